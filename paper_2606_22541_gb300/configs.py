@@ -1,0 +1,83 @@
+"""The five layer configurations the MoE layer is exercised on.
+
+Shapes follow the model the paper evaluates (DeepSeek-V3.2: 256 routed experts
+plus one shared expert, top-8, hidden 7168, 16-bit data; ASAP Table 1 and
+Section 5.1) and two smaller families (a tiny correctness case and a
+Mixtral-8x7B-shaped layer).  Micro-batches stand for token batches arriving
+independently from attention DP groups (Section 3.3); each runs on its own CUDA
+stream with no host barrier between them (Section 3.4.2).
+"""
+from dataclasses import dataclass, field, asdict
+from typing import List, Optional
+
+GATING = {"softmax": 0, "softmax_renorm": 1, "sigmoid_grouped": 2}
+DTYPE = {"bf16": 0, "fp8_e4m3_block128": 1}
+
+
+@dataclass(frozen=True)
+class LayerConfig:
+    name: str
+    hidden: int            # H
+    n_experts: int         # E routed experts
+    top_k: int             # k
+    inter: int             # I, routed expert intermediate
+    n_shared: int          # 0 or 1
+    shared_inter: int      # I_s
+    gating: str
+    n_groups: int = 1
+    topk_groups: int = 1
+    route_scale: float = 1.0
+    dtype: str = "bf16"
+    microbatches: List[int] = field(default_factory=list)
+    zipf_s: Optional[float] = None   # expert-popularity skew of the inputs
+    seed: int = 1000
+
+    @property
+    def n_tokens(self):
+        return sum(self.microbatches)
+
+    @property
+    def max_microbatch(self):
+        return max(self.microbatches) if self.microbatches else 0
+
+    def oracle_cfg(self):
+        """Plain mapping handed to the oracle."""
+        return dict(n_experts=self.n_experts, top_k=self.top_k, gating=self.gating,
+                    n_groups=self.n_groups, topk_groups=self.topk_groups,
+                    route_scale=self.route_scale)
+
+    def flops_per_token(self):
+        """Multiply-adds x 2 of the expert FFNs (router excluded)."""
+        return 6 * self.hidden * self.inter * self.top_k + 6 * self.hidden * self.shared_inter * self.n_shared
+
+    def router_flops_per_token(self):
+        return 2 * self.hidden * self.n_experts
+
+    def as_dict(self):
+        return asdict(self)
+
+
+def _stress_lengths(seed, count=8, mu=7.5, sigma=1.0, lo=128, hi=16384):
+    import numpy as np
+    rng = np.random.Generator(np.random.PCG64(seed))
+    v = np.round(rng.lognormal(mu, sigma, size=count)).astype(int)
+    return [int(min(max(a, lo), hi)) for a in v]
+
+
+TINY = LayerConfig("tiny", hidden=256, n_experts=8, top_k=2, inter=128, n_shared=0,
+                   shared_inter=0, gating="softmax", microbatches=[96, 160], seed=1000)
+MIXTRAL = LayerConfig("mixtral", hidden=4096, n_experts=8, top_k=2, inter=14336, n_shared=0,
+                      shared_inter=0, gating="softmax_renorm",
+                      microbatches=[1024, 1536, 2048, 3584], seed=1001)
+DSV3 = LayerConfig("dsv3_bf16", hidden=7168, n_experts=256, top_k=8, inter=2048, n_shared=1,
+                   shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                   route_scale=2.5, microbatches=[4096] * 4, seed=1002)
+STRESS = LayerConfig("dsv3_stress", hidden=7168, n_experts=256, top_k=8, inter=2048, n_shared=1,
+                     shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                     route_scale=2.5, microbatches=_stress_lengths(1003), zipf_s=1.1, seed=1003)
+DSV3_FP8 = LayerConfig("dsv3_fp8", hidden=7168, n_experts=256, top_k=8, inter=2048, n_shared=1,
+                       shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                       route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[4096] * 8,
+                       zipf_s=1.1, seed=1004)
+
+CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8)}

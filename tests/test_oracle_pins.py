@@ -1,0 +1,395 @@
+"""Pins of the float64 oracle against things other than itself: library
+conversions, brute force on tiny inputs, closed forms, invariants and a
+hand-worked example.  CPU only."""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import formats, gating, layer
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------- formats
+
+def test_bf16_decoder_matches_torch_on_every_pattern():
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    ours = formats.bf16_bits_to_f64(bits)
+    ref = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(torch.float64).numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(ours), nan)
+    assert np.array_equal(ours[~nan], ref[~nan])
+
+
+def test_bf16_decoder_known_values():
+    f = formats.bf16_bits_to_f64
+    assert f(np.uint16(0x3F80)) == 1.0
+    assert f(np.uint16(0xC000)) == -2.0
+    assert f(np.uint16(0x0001)) == 2.0 ** -133
+    assert f(np.uint16(0x7F7F)) == (2 - 2 ** -7) * 2.0 ** 127
+    assert np.isinf(f(np.uint16(0x7F80)))
+
+
+def test_e4m3_decoder_matches_torch_on_every_pattern():
+    bits = np.arange(256, dtype=np.uint8)
+    ours = formats.e4m3_bits_to_f64(bits)
+    ref = torch.from_numpy(bits).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(ours), nan)
+    assert np.array_equal(ours[~nan], ref[~nan])
+    assert formats.e4m3_bits_to_f64(np.uint8(0x7E)) == 448.0
+    assert formats.e4m3_bits_to_f64(np.uint8(0x01)) == 2.0 ** -9
+
+
+def test_e4m3_rounding_matches_torch_cast_in_range():
+    rng = np.random.default_rng(5)
+    v = np.concatenate([rng.normal(0, 30, 20000), rng.normal(0, 0.01, 5000),
+                        rng.uniform(-448, 448, 5000)])
+    ours = formats.round_to_e4m3_sat(v)
+    ref = torch.from_numpy(v).to(torch.float8_e4m3fn).to(torch.float64).numpy()
+    assert np.array_equal(ours, ref)
+
+
+def test_e4m3_rounding_ties_and_saturation():
+    r = formats.round_to_e4m3_sat
+    assert r(1.0625) == 1.0          # halfway between 1 and 1.125 -> even
+    assert r(1.1875) == 1.25         # halfway between 1.125 and 1.25 -> even
+    assert r(464.0) == 448.0         # tie between 448 and (absent) 480
+    assert r(1e6) == 448.0 and r(-1e6) == -448.0
+    assert r(2.0 ** -10) == 0.0      # half the smallest subnormal -> even (0)
+    assert r(3 * 2.0 ** -10) == 2 * 2.0 ** -9
+
+
+# ---------------------------------------------------------------- gating
+
+def _brute_topk_softmax(l, k, renorm):
+    """Max-sum subset, ties -> lexicographically smallest index set; slots by
+    (-value, index); weights from the softmax written out directly."""
+    E = len(l)
+    best = None
+    for S in itertools.combinations(range(E), k):
+        key = (sum(l[i] for i in S), tuple(-i for i in S))
+        if best is None or key > best[0]:
+            best = (key, S)
+    S = sorted(best[1], key=lambda i: (-l[i], i))
+    z = sum(math.exp(v) for v in l)
+    w = [math.exp(l[i]) / z for i in S]
+    if renorm:
+        tot = sum(w)
+        w = [v / tot for v in w]
+    return S, w
+
+
+@pytest.mark.parametrize("renorm", [False, True])
+def test_softmax_topk_matches_brute_force(renorm):
+    rng = np.random.default_rng(11)
+    for _ in range(300):
+        l = rng.normal(0, 1.5, 8)
+        idx, w = gating.route_token_softmax(l, 2, renorm)
+        S, wb = _brute_topk_softmax(list(l), 2, renorm)
+        assert list(idx) == S
+        assert np.allclose(w, wb, rtol=1e-13, atol=0)
+
+
+def test_softmax_topk_exact_ties_lower_index_wins():
+    l = np.array([0.5, 1.0, 1.0, 0.2, 1.0, -1.0, 0.0, 1.0])
+    idx, _ = gating.route_token_softmax(l, 2, False)
+    assert list(idx) == [1, 2]
+    S, _ = _brute_topk_softmax(list(l), 3, False)
+    idx3, _ = gating.route_token_softmax(l, 3, False)
+    assert list(idx3) == S == [1, 2, 4]
+
+
+def _brute_grouped(l, k, G, kg, scale):
+    s = [1 / (1 + math.exp(-v)) for v in l]
+    E = len(l)
+    gsz = E // G
+    gscore = []
+    for g in range(G):
+        mem = range(g * gsz, (g + 1) * gsz)
+        gscore.append(max(s[a] + s[b] for a, b in itertools.combinations(mem, 2)))
+    best = None
+    for Gs in itertools.combinations(range(G), kg):
+        key = (sum(gscore[g] for g in Gs), tuple(-g for g in Gs))
+        if best is None or key > best[0]:
+            best = (key, Gs)
+    cand = [e for g in best[1] for e in range(g * gsz, (g + 1) * gsz)]
+    bestS = None
+    for S in itertools.combinations(cand, k):
+        key = (sum(s[i] for i in S), tuple(-i for i in sorted(S)))
+        if bestS is None or key > bestS[0]:
+            bestS = (key, S)
+    S = sorted(bestS[1], key=lambda i: (-s[i], i))
+    tot = sum(s[i] for i in S)
+    return S, [s[i] / tot * scale for i in S]
+
+
+def test_grouped_sigmoid_matches_brute_force():
+    rng = np.random.default_rng(12)
+    for _ in range(150):
+        l = rng.normal(0, 1.0, 16)
+        idx, w = gating.route_token_sigmoid_grouped(l, 4, 4, 2, 2.5)
+        S, wb = _brute_grouped(list(l), 4, 4, 2, 2.5)
+        assert list(idx) == S
+        assert np.allclose(w, wb, rtol=1e-13, atol=0)
+
+
+def test_grouped_sigmoid_group_tie_lower_group_wins():
+    # groups of 4; groups 1 and 2 tie on the top-2 sum, group 0 is best
+    l = np.array([3.0, 2.9, -5, -5,   1.0, 0.5, -5, -5,   0.5, 1.0, -5, -5,   -3, -3, -3, -3])
+    idx, _ = gating.route_token_sigmoid_grouped(l, 4, 4, 2, 1.0)
+    assert list(idx) == [0, 1, 4, 5]
+    S, _ = _brute_grouped(list(l), 4, 4, 2, 1.0)
+    assert S == [0, 1, 4, 5]
+
+
+def test_softmax_renorm_with_k_equal_E_is_full_softmax():
+    rng = np.random.default_rng(13)
+    l = rng.normal(0, 2, 8)
+    idx, w = gating.route_token_softmax(l, 8, True)
+    p = np.exp(l) / np.exp(l).sum()
+    assert np.allclose(w, p[idx], rtol=1e-13)
+    assert sorted(idx) == list(range(8))
+
+
+def test_softmax_variants_agree_on_idx():
+    rng = np.random.default_rng(14)
+    L = rng.normal(0, 1, (64, 8))
+    a, _ = gating.route(L, dict(gating="softmax", top_k=2))
+    b, _ = gating.route(L, dict(gating="softmax_renorm", top_k=2))
+    assert np.array_equal(a, b)
+
+
+def test_certified_comparison():
+    cfg = dict(gating="softmax", top_k=2)
+    l = np.array([1.0, 0.9, 0.5, 0.4, 0.0, -1, -2, -3])
+    eps = np.full(8, 1e-3)
+    assert gating.token_decided(l, eps, cfg)
+    assert gating.token_feasible(l, eps, cfg, [0, 1])
+    assert not gating.token_feasible(l, eps, cfg, [1, 0])
+    assert not gating.token_feasible(l, eps, cfg, [0, 2])
+    l2 = l.copy()
+    l2[2] = 0.9 - 5e-4                      # near tie at the k boundary
+    assert not gating.token_decided(l2, eps, cfg)
+    assert gating.token_feasible(l2, eps, cfg, [0, 2])   # either may win
+    assert gating.token_feasible(l2, eps, cfg, [0, 1])
+    gcfg = dict(gating="sigmoid_grouped", top_k=4, n_groups=4, topk_groups=2, route_scale=1.0)
+    rng = np.random.default_rng(15)
+    n_decided = 0
+    for _ in range(50):
+        lg = rng.normal(0, 1, 16)
+        idx, _ = gating.route_token_sigmoid_grouped(lg, 4, 4, 2, 1.0)
+        e = np.full(16, 1e-6)
+        assert gating.token_feasible(lg, e, gcfg, idx)
+        if gating.token_decided(lg, e, gcfg):
+            n_decided += 1
+            # the next-best expert of the kept groups swapped into the last
+            # slot, or a slot swap, must be infeasible for a decided token
+            groups = sorted(set((idx // 4).tolist()) | set())
+            s = 1 / (1 + np.exp(-lg))
+            cand = [c for g in range(4) for c in range(4 * g, 4 * g + 4)
+                    if c not in idx and (c // 4) in groups]
+            if cand:
+                nxt = max(cand, key=lambda c: (s[c], -c))
+                wrong = idx.copy()
+                wrong[-1] = nxt
+                assert not gating.token_feasible(lg, e, gcfg, wrong)
+            assert not gating.token_feasible(lg, e, gcfg, idx[[1, 0, 2, 3]])
+    assert n_decided > 40
+
+
+# ---------------------------------------------------------------- counts / permutation
+
+def _random_idx(rng, n, E, k):
+    return np.array([rng.permutation(E)[:k] for _ in range(n)], np.int64).reshape(n, k)
+
+
+def test_counts_offsets_invariants():
+    rng = np.random.default_rng(21)
+    for n, E, k in [(0, 8, 2), (1, 8, 2), (37, 8, 2), (200, 256, 8)]:
+        idx = _random_idx(rng, n, E, k).reshape(n, k)
+        c = layer.expert_counts(idx, E)
+        o = layer.expert_offsets(c)
+        assert c.sum() == n * k and (c >= 0).all()
+        assert o[0] == 0 and o[-1] == n * k and (np.diff(o) == c).all()
+        assert np.array_equal(c, np.bincount(idx.reshape(-1), minlength=E))
+
+
+def test_permutation_is_a_stable_bijection():
+    rng = np.random.default_rng(22)
+    n, E, k = 150, 16, 4
+    idx = _random_idx(rng, n, E, k)
+    src, dst = layer.permutation(idx, E)
+    assert sorted(dst.reshape(-1).tolist()) == list(range(n * k))
+    off = layer.expert_offsets(layer.expert_counts(idx, E))
+    for t in range(n):
+        for j in range(k):
+            p = dst[t, j]
+            assert src[p] == t
+            e = idx[t, j]
+            assert off[e] <= p < off[e + 1]
+    # stable: inside each segment the (t, j) pairs increase
+    pairs = {int(dst[t, j]): (t, j) for t in range(n) for j in range(k)}
+    for e in range(E):
+        seg = [pairs[p] for p in range(off[e], off[e + 1])]
+        assert seg == sorted(seg)
+
+
+def test_identity_experts_return_k_times_x():
+    rng = np.random.default_rng(23)
+    n, E, k, H = 64, 8, 2, 32
+    bits = rng.integers(0, 65536, (n, H)).astype(np.uint16)
+    bits = (bits & 0x3FFF) | 0x3000           # finite, moderate bf16 values
+    x = formats.bf16_bits_to_f64(bits)
+    idx = _random_idx(rng, n, E, k)
+    src, dst = layer.permutation(idx, E)
+    xp = layer.dispatch(x, src)
+    out = layer.combine(xp, np.ones((n, k)), dst)
+    assert np.array_equal(out, k * x)
+
+
+# ---------------------------------------------------------------- FFN / layer
+
+def test_single_expert_k1_equals_dense_swiglu():
+    rng = np.random.default_rng(31)
+    n, H, I = 20, 48, 24
+    x = rng.normal(0, 1, (n, H))
+    wg = rng.normal(0, 0.2, (1, I, H))
+    wu = rng.normal(0, 0.2, (1, I, H))
+    wd = rng.normal(0, 0.2, (1, H, I))
+    wr = rng.normal(0, 0.2, (1, H))
+    cfg = dict(n_experts=1, top_k=1, gating="softmax", n_groups=1, topk_groups=1, route_scale=1.0)
+    r = layer.moe_layer(x, wr, wg, wu, wd, cfg)
+    # dense SwiGLU written independently: per token, per channel sums
+    g = np.einsum("ih,nh->ni", wg[0], x)
+    u = np.einsum("ih,nh->ni", wu[0], x)
+    h = g * u / (1 + np.exp(-g))
+    ref = np.einsum("hi,ni->nh", wd[0], h)
+    assert np.allclose(r["w"], 1.0)
+    assert np.allclose(r["y"], ref, rtol=1e-12, atol=1e-12)
+
+
+def test_worked_example():
+    d = json.load(open(os.path.join(GOLDEN, "worked_layer_example.json")))
+    a = lambda k: np.array(d[k], np.float64)
+    cfg = dict(n_experts=2, top_k=1, gating="softmax", n_groups=1, topk_groups=1, route_scale=1.0)
+    r = layer.moe_layer(a("x"), a("router_w"), a("w_gate"), a("w_up"), a("w_down"), cfg,
+                        shared=(a("sh_gate"), a("sh_up"), a("sh_down")))
+    p0 = 1 / (1 + math.exp(-2))
+    h = 2 / (1 + math.exp(-2))
+    hs = -1 / (1 + math.exp(1))
+    assert r["idx"].tolist() == d["expected_idx"]
+    assert np.allclose(r["y"], [[p0 * h + 2 * hs, 3 * p0 * h]], rtol=1e-14, atol=0)
+
+
+def test_per_token_independence():
+    rng = np.random.default_rng(32)
+    n, H, E, k, I = 60, 32, 8, 2, 16
+    x = rng.normal(0, 1, (n, H))
+    wr = rng.normal(0, 0.3, (E, H))
+    wg = rng.normal(0, 0.2, (E, I, H))
+    wu = rng.normal(0, 0.2, (E, I, H))
+    wd = rng.normal(0, 0.2, (E, H, I))
+    cfg = dict(n_experts=E, top_k=k, gating="softmax_renorm", n_groups=1, topk_groups=1, route_scale=1.0)
+    full = layer.moe_layer(x, wr, wg, wu, wd, cfg)["y"]
+    parts = [layer.moe_layer(x[a:b], wr, wg, wu, wd, cfg)["y"] for a, b in [(0, 7), (7, 33), (33, 60)]]
+    assert np.allclose(np.concatenate(parts), full, rtol=1e-12, atol=1e-12)
+    some = [3, 17, 59]
+    r = layer.moe_layer(x, wr, wg, wu, wd, cfg)
+    tok = layer.moe_layer_tokens(x[some], r["idx"][some], r["w"][some], wg, wu, wd)
+    assert np.allclose(tok, full[some], rtol=1e-12, atol=1e-12)
+
+
+def test_shared_expert_enters_once():
+    rng = np.random.default_rng(33)
+    n, H, E, k, I = 10, 16, 4, 2, 8
+    x = rng.normal(0, 1, (n, H))
+    wr = rng.normal(0, 0.3, (E, H))
+    wg, wu = rng.normal(0, 0.2, (2, E, I, H))
+    wd = rng.normal(0, 0.2, (E, H, I))
+    sh = (rng.normal(0, 0.2, (I, H)), rng.normal(0, 0.2, (I, H)), rng.normal(0, 0.2, (H, I)))
+    cfg = dict(n_experts=E, top_k=k, gating="softmax", n_groups=1, topk_groups=1, route_scale=1.0)
+    a = layer.moe_layer(x, wr, wg, wu, wd, cfg)["y"]
+    b = layer.moe_layer(x, wr, wg, wu, wd, cfg, shared=sh)["y"]
+    assert np.allclose(b - a, layer.swiglu(x, *sh), rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- FP8 emulation
+
+def test_row_quantisation_properties():
+    rng = np.random.default_rng(41)
+    v = rng.normal(0, 3, (7, 384))
+    q, s = layer.quantize_rows_e4m3(v)
+    assert s.shape == (7, 3)
+    # every q is an e4m3 value and the block max maps to exactly 448
+    assert np.array_equal(formats.round_to_e4m3_sat(q), q)
+    for b in range(3):
+        assert np.allclose(np.abs(q[:, b * 128:(b + 1) * 128]).max(1), 448.0)
+    back = q * np.repeat(s, 128, 1)
+    # relative error of e4m3 normals is at most 2^-4; subnormals add 2^-10*s
+    err = np.abs(back - v)
+    bound = np.abs(v) * 2.0 ** -4 + np.repeat(s, 128, 1) * 2.0 ** -10
+    assert (err <= bound * (1 + 1e-12)).all()
+
+
+def test_dequant_blocks_layout():
+    q = np.ones((256, 384))
+    s = np.arange(6, dtype=np.float64).reshape(2, 3)
+    w = layer.dequant_blocks(q, s)
+    assert w[0, 0] == 0 and w[127, 383] == 2 and w[128, 0] == 3 and w[255, 383] == 5
+
+
+def test_fp8_swiglu_is_close_to_exact_and_exact_on_representable_input():
+    rng = np.random.default_rng(42)
+    H, I = 256, 128
+    x = rng.normal(0, 1, (3, H))
+    wg, wu = rng.normal(0, 1 / 16, (2, I, H))
+    wd = rng.normal(0, 1 / 11.3, (H, I))
+    a = layer.swiglu_fp8(x, wg, wu, wd)
+    b = layer.swiglu(x, wg, wu, wd)
+    assert np.linalg.norm(a - b) / np.linalg.norm(b) < 0.08
+
+
+# ---------------------------------------------------------------- paper constants
+
+def test_table1_shapes_are_the_dsv3_configs():
+    d = json.load(open(os.path.join(GOLDEN, "table1_dsv3.json")))
+    from paper_2606_22541_gb300.configs import DSV3, STRESS, DSV3_FP8
+    for c in (DSV3, STRESS, DSV3_FP8):
+        assert c.n_experts == d["E_total"] == d["routed_experts"]
+        assert c.top_k == d["K"] == d["active_routed_per_token"]
+        assert c.hidden == d["H"]
+        assert c.n_shared == d["shared_experts"] == d["active_shared_per_token"]
+
+
+# ---------------------------------------------------------------- planted mistakes
+
+def test_pins_catch_planted_mistakes(monkeypatch):
+    """Plant plausible mistakes in the oracle and check a pin notices."""
+    rng = np.random.default_rng(51)
+    n, H, I = 6, 16, 8
+    x = rng.normal(0, 1, (n, H))
+    wg, wu = rng.normal(0, 0.3, (2, 1, I, H))
+    wd = rng.normal(0, 0.3, (1, H, I))
+    cfg = dict(n_experts=1, top_k=1, gating="softmax", n_groups=1, topk_groups=1, route_scale=1.0)
+    g = np.einsum("ih,nh->ni", wg[0], x)
+    u = np.einsum("ih,nh->ni", wu[0], x)
+    ref = np.einsum("hi,ni->nh", wd[0], g * u / (1 + np.exp(-g)))
+    good = layer.moe_layer(x, rng.normal(0, 1, (1, H)), wg, wu, wd, cfg)["y"]
+    assert np.allclose(good, ref)
+    monkeypatch.setattr(layer, "silu", lambda v: v / (1.0 + np.exp(v)))   # sign slip
+    bad = layer.moe_layer(x, rng.normal(0, 1, (1, H)), wg, wu, wd, cfg)["y"]
+    assert not np.allclose(bad, ref)
+    monkeypatch.undo()
+    # transposed router operand order would reorder top-k: brute force sees it
+    l = np.array([0.1, 2.0, -1.0, 1.5, 0.0, 0.3, -0.2, 0.9])
+    S, _ = _brute_topk_softmax(list(l), 2, False)
+    monkeypatch.setattr(gating, "_order", lambda keys: np.lexsort((np.arange(len(keys)), np.asarray(keys))))
+    idx, _ = gating.route_token_softmax(l, 2, False)
+    assert list(idx) != S
