@@ -1,0 +1,224 @@
+/*
+ * asap_moe.h -- C ABI of the expert-side MoE layer of ASAP's data-parallel
+ * prefill path, for one NVIDIA GB300 (sm_103a).
+ *
+ * The layer (ASAP Sections 3.2 and 3.4.2; shapes from Table 1 and Section 5.1):
+ *
+ *   route     : logits L = x Wr^T; top-k gating -> idx[n,k], w[n,k];
+ *               per-expert token counts and their exclusive prefix offsets
+ *               (the "token metadata" the MoE side receives, Section 3.2.1)
+ *   dispatch  : hidden states grouped per expert, x_perm[offsets[e] + r] = x[t]
+ *               (the "token payload", Section 3.2.1)
+ *   expert_ffn: grouped GEMM, hidden states on the left and one layer's expert
+ *               weights on the right (Section 3.4.2):
+ *               h = silu(X_e Wg_e^T) * (X_e Wu_e^T);  y = h Wd_e^T,
+ *               plus the always-active shared expert on every token (Section 5.1)
+ *   combine   : out[t] = sum_j w[t,j] y_perm[perm_dst[t,j]] + y_shared[t]
+ *               (expert results returned through the expert IDs, Section 3.2.2)
+ *
+ * Conventions for every call below:
+ *  - Tensors are row-major device pointers owned by the caller, except the
+ *    packed weight copies a handle makes in asap_moe_create.  Inputs and
+ *    outputs of a call must not overlap.
+ *  - Calls other than create / destroy / status only ENQUEUE work on the given
+ *    stream: no host synchronisation, no allocation, no read-back of counts.
+ *    Micro-batches from different attention DP groups can therefore be
+ *    submitted on different streams with no host barrier between them
+ *    (Section 3.4.2, bubble-free dispatching).
+ *  - Each call in flight needs its own workspace (asap_moe_workspace_size);
+ *    two calls that run at the same time must not share one.
+ *  - n == 0 is a successful no-op.  n > max_tokens, NULL pointers for
+ *    required tensors or a workspace smaller than required return
+ *    ASAP_ERR_INVALID / ASAP_ERR_WORKSPACE without enqueuing anything.
+ *  - Launch failures return ASAP_ERR_CUDA.  asap_moe_last_error() returns a
+ *    thread-local message describing the last failure of this thread.
+ *  - A handle is immutable after create; concurrent calls on different
+ *    streams with different workspaces are safe.
+ *  - Kernels that detect a bad index or a wait that exceeds its time limit
+ *    record it in a device status word of the handle instead of trapping;
+ *    asap_moe_status reads and clears it.
+ *
+ * Layouts (bf16 unless stated; H hidden, E experts, k top-k, I intermediate):
+ *   x        [n, H]          hidden states of one micro-batch
+ *   idx      [n, k] int32    expert of (token, slot); slot order = descending
+ *                            selection score, ties by lower expert index
+ *   w        [n, k] fp32     routing weight of (token, slot)
+ *   counts   [E]    int32    tokens per expert
+ *   offsets  [E+1]  int32    exclusive prefix sum of counts, offsets[E] = n*k
+ *   perm_src [n*k]  int32    position -> token
+ *   perm_dst [n*k]  int32    (token t, slot j) at t*k + j -> position; inside
+ *                            a segment positions follow increasing (t, j)
+ *   x_perm   [n*k, H]        expert-grouped hidden states
+ *   y_perm   [n*k, H]        expert outputs, same order as x_perm
+ *   y_shared [n, H]          shared-expert output (unused when n_shared == 0)
+ *   out      [n, H]          layer output
+ */
+#ifndef ASAP_MOE_H
+#define ASAP_MOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ASAP_MOE_MAX_EXPERTS 256
+#define ASAP_MOE_MAX_TOPK 8
+
+typedef enum {
+  ASAP_OK = 0,
+  ASAP_ERR_INVALID = -1,      /* bad argument or configuration */
+  ASAP_ERR_UNSUPPORTED = -2,  /* valid request this build does not implement */
+  ASAP_ERR_WORKSPACE = -3,    /* workspace missing or too small */
+  ASAP_ERR_CUDA = -4,         /* a CUDA runtime call or launch failed */
+  ASAP_ERR_DEVICE_STATUS = -5 /* a kernel recorded an error (asap_moe_status) */
+} asap_status;
+
+/* Gating rules (the paper names the model, not the rule; these are the
+ * published definitions of the model families):
+ *  SOFTMAX          p = softmax(L); top-k of p; w = p (no renormalisation)
+ *  SOFTMAX_RENORM   as SOFTMAX, then w = p / sum of the selected p
+ *  SIGMOID_GROUPED  s = sigmoid(L); selection score s + bias; n_groups equal
+ *                   contiguous groups scored by the sum of their two best
+ *                   selection scores; keep topk_groups groups; top-k of their
+ *                   experts; w = s / sum of selected s * route_scale.
+ * Ties go to the lower expert (group) index.                                */
+typedef enum {
+  ASAP_GATE_SOFTMAX = 0,
+  ASAP_GATE_SOFTMAX_RENORM = 1,
+  ASAP_GATE_SIGMOID_GROUPED = 2
+} asap_gating;
+
+typedef enum {
+  ASAP_BF16 = 0,              /* bf16 storage, fp32 accumulation */
+  ASAP_FP8_E4M3_BLOCK128 = 1  /* e4m3 weights with one fp32 scale per 128x128
+                                 block; activations e4m3 per token per 128
+                                 channels (reserved: ASAP_ERR_UNSUPPORTED) */
+} asap_dtype;
+
+/* Shape and gating of one MoE layer.  Table 1 of the paper: E_total = 256,
+ * K = 8, H = 7168, 16-bit data; Section 5.1: one shared expert.
+ * Requirements: hidden % 256 == 0; inter % 128 == 0; shared_inter % 128 == 0
+ * when n_shared == 1; 1 <= n_experts <= 256; 1 <= top_k <= min(8, n_experts);
+ * for SIGMOID_GROUPED n_experts % n_groups == 0, group size >= 2 and
+ * top_k <= topk_groups * group size; max_tokens * top_k < 2^31.            */
+typedef struct {
+  int32_t hidden;        /* H */
+  int32_t n_experts;     /* E, routed experts */
+  int32_t top_k;         /* k */
+  int32_t inter;         /* I, routed-expert intermediate size */
+  int32_t n_shared;      /* 0 or 1 shared expert */
+  int32_t shared_inter;  /* I_s */
+  int32_t gating;        /* asap_gating */
+  int32_t n_groups;      /* SIGMOID_GROUPED only */
+  int32_t topk_groups;   /* SIGMOID_GROUPED only */
+  float route_scale;     /* SIGMOID_GROUPED only */
+  int32_t dtype;         /* asap_dtype */
+  int32_t max_tokens;    /* largest micro-batch a call may pass */
+} asap_moe_config;
+
+/* Device pointers to one layer's weights (bf16, row-major).  They are copied
+ * (and re-packed) by asap_moe_create; the caller may free them afterwards.
+ *   router_w  [E, H]
+ *   router_bias [E] fp32 or NULL: selection-only correction bias
+ *   w_gate, w_up [E][I, H];  w_down [E][H, I]
+ *   sh_gate, sh_up [I_s, H]; sh_down [H, I_s]   (NULL when n_shared == 0)
+ *   s_* : fp32 block scales of the FP8 configuration (NULL for bf16)        */
+typedef struct {
+  const void* router_w;
+  const float* router_bias;
+  const void* w_gate;
+  const void* w_up;
+  const void* w_down;
+  const float* s_gate;
+  const float* s_up;
+  const float* s_down;
+  const void* sh_gate;
+  const void* sh_up;
+  const void* sh_down;
+  const float* sh_s_gate;
+  const float* sh_s_up;
+  const float* sh_s_down;
+} asap_moe_weights;
+
+typedef struct asap_moe_s* asap_moe_t;
+
+/* Validate cfg, allocate the handle's device memory on the current device,
+ * copy and pack the weights (gate/up rows interleaved in blocks of 128 so one
+ * 256-wide GEMM tile holds matching gate and up columns) and build the weight
+ * TMA descriptors.  Synchronous.  On failure *out is NULL. */
+int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* weights,
+                    asap_moe_t* out);
+
+/* Free everything create allocated.  Synchronises the device first.  NULL is
+ * accepted. */
+int asap_moe_destroy(asap_moe_t h);
+
+/* Pure host computation: bytes of workspace one call with n tokens needs.  The
+ * same size serves every enqueuing call below.  Needs no GPU. */
+int asap_moe_workspace_size(const asap_moe_config* cfg, int32_t n_tokens, size_t* bytes);
+
+/* Pure host computation: ASAP_OK when cfg satisfies the requirements above,
+ * otherwise ASAP_ERR_INVALID / ASAP_ERR_UNSUPPORTED and a message.  Needs no
+ * GPU. */
+int asap_moe_check_config(const asap_moe_config* cfg);
+
+/* Router logits only: logits[n, E] (fp32) = x Wr^T, fp32 accumulation of
+ * bf16 products. */
+int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, float* logits,
+                           void* ws, size_t ws_bytes, void* stream);
+
+/* Routing (Table 1: top-K of E_total experts; Section 3.2.1: per-expert token
+ * counts): logits, gating, idx/w, counts, offsets.  counts and offsets are
+ * deterministic. */
+int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
+                   int32_t* counts, int32_t* offsets, void* ws, size_t ws_bytes,
+                   void* stream);
+
+/* Routing from given fp32 logits [n, E] (lets exact ties be tested). */
+int asap_moe_route_logits(asap_moe_t h, const float* logits, int32_t n, int32_t* idx,
+                          float* w, int32_t* counts, int32_t* offsets, void* ws,
+                          size_t ws_bytes, void* stream);
+
+/* Dispatch (Section 3.2.1 token payload): from idx, build perm_src/perm_dst
+ * and copy every token row into its k expert segments of x_perm.  idx values
+ * outside [0, E) are recorded in the status word and the entry is skipped.
+ * x_perm_scales is reserved for the FP8 configuration (pass NULL). */
+int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx,
+                      void* x_perm, float* x_perm_scales, int32_t* perm_src,
+                      int32_t* perm_dst, void* ws, size_t ws_bytes, void* stream);
+
+/* Expert FFN (Section 3.4.2 GMM): y_perm rows of expert e's segment
+ * [offsets[e], offsets[e+1]) = SwiGLU_e(x_perm rows); y_shared = shared
+ * SwiGLU of x (ignored when n_shared == 0).  The grouped GEMMs find their
+ * tiles on the device from offsets (offsets[E] must equal n*k). */
+int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
+                        const int32_t* offsets, const void* x, int32_t n, void* y_perm,
+                        void* y_shared, void* ws, size_t ws_bytes, void* stream);
+
+/* Combine (Section 3.2.2): out[t] = sum_{j<k} w[t,j] y_perm[perm_dst[t*k+j]]
+ * (+ y_shared[t]), fp32 in slot order then the shared row, rounded to bf16.
+ * y_shared may be NULL. */
+int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared,
+                     const float* w, const int32_t* perm_dst, int32_t n, void* out,
+                     void* stream);
+
+/* The whole layer for one micro-batch: route -> dispatch -> expert_ffn ->
+ * combine, enqueued on one stream with no host synchronisation.  Bit-identical
+ * to the four calls composed. */
+int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
+                   size_t ws_bytes, void* stream);
+
+/* Synchronise the device, return ASAP_OK or ASAP_ERR_DEVICE_STATUS, write the
+ * raw status word (0 = clean) to *word if non-NULL, then clear it. */
+int asap_moe_status(asap_moe_t h, uint32_t* word);
+
+/* Thread-local text of this thread's last failure ("" if none). */
+const char* asap_moe_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASAP_MOE_H */

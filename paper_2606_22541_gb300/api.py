@@ -1,0 +1,147 @@
+"""Python binding of the C ABI, one function per entry point with the same name.
+
+Tensors are torch CUDA tensors (the binding passes their device pointers);
+``stream`` is a torch.cuda.Stream or None for the current stream.  Every step
+of the layer runs in libasap_moe's kernels; nothing here computes.
+"""
+import ctypes
+
+import torch
+
+from . import _native
+from ._native import AsapMoeConfig, AsapMoeWeights, check, lib
+from .configs import GATING, DTYPE
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def make_config(cfg, max_tokens):
+    """C config from a configs.LayerConfig."""
+    return AsapMoeConfig(hidden=cfg.hidden, n_experts=cfg.n_experts, top_k=cfg.top_k, inter=cfg.inter,
+                         n_shared=cfg.n_shared, shared_inter=cfg.shared_inter, gating=GATING[cfg.gating],
+                         n_groups=cfg.n_groups, topk_groups=cfg.topk_groups,
+                         route_scale=float(cfg.route_scale), dtype=DTYPE[cfg.dtype],
+                         max_tokens=int(max_tokens))
+
+
+class Handle:
+    """Owns an asap_moe_t; destroyed on close() or garbage collection."""
+
+    def __init__(self, ptr, cfg, ccfg):
+        self.ptr = ptr
+        self.cfg = cfg
+        self.ccfg = ccfg
+
+    @property
+    def max_tokens(self):
+        return self.ccfg.max_tokens
+
+    def close(self):
+        if self.ptr:
+            lib().asap_moe_destroy(self.ptr)
+            self.ptr = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def asap_moe_check_config(cfg, max_tokens=1):
+    c = make_config(cfg, max_tokens)
+    return lib().asap_moe_check_config(ctypes.byref(c))
+
+
+def asap_moe_create(cfg, weights, max_tokens):
+    """weights: dict of CUDA tensors named like asap_moe_weights' fields."""
+    c = make_config(cfg, max_tokens)
+    w = AsapMoeWeights()
+    for name, _ in AsapMoeWeights._fields_:
+        t = weights.get(name)
+        setattr(w, name, None if t is None else t.data_ptr())
+    out = ctypes.c_void_p()
+    check("asap_moe_create", lib().asap_moe_create(ctypes.byref(c), ctypes.byref(w), ctypes.byref(out)))
+    return Handle(out, cfg, c)
+
+
+def asap_moe_destroy(h):
+    h.close()
+
+
+def asap_moe_workspace_size(cfg, n_tokens, max_tokens=None):
+    c = make_config(cfg, max_tokens if max_tokens is not None else max(n_tokens, 1))
+    out = ctypes.c_size_t()
+    check("asap_moe_workspace_size", lib().asap_moe_workspace_size(ctypes.byref(c), int(n_tokens), ctypes.byref(out)))
+    return out.value
+
+
+def workspace(h, n_tokens, device="cuda"):
+    """A workspace tensor large enough for one call with n_tokens tokens."""
+    nbytes = asap_moe_workspace_size(h.cfg, n_tokens, h.max_tokens)
+    return torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+
+
+def _ws(ws):
+    return (_ptr(ws), ctypes.c_size_t(0 if ws is None else ws.numel() * ws.element_size()))
+
+
+def asap_moe_router_logits(h, x, logits, ws=None, stream=None):
+    p, n = _ws(ws)
+    check("asap_moe_router_logits",
+          lib().asap_moe_router_logits(h.ptr, _ptr(x), x.shape[0], _ptr(logits), p, n, _stream(stream)))
+
+
+def asap_moe_route(h, x, idx, w, counts, offsets, ws, stream=None):
+    p, n = _ws(ws)
+    check("asap_moe_route", lib().asap_moe_route(h.ptr, _ptr(x), x.shape[0], _ptr(idx), _ptr(w), _ptr(counts),
+                                                 _ptr(offsets), p, n, _stream(stream)))
+
+
+def asap_moe_route_logits(h, logits, idx, w, counts, offsets, ws, stream=None):
+    p, n = _ws(ws)
+    check("asap_moe_route_logits",
+          lib().asap_moe_route_logits(h.ptr, _ptr(logits), logits.shape[0], _ptr(idx), _ptr(w), _ptr(counts),
+                                      _ptr(offsets), p, n, _stream(stream)))
+
+
+def asap_moe_dispatch(h, x, idx, x_perm, perm_src, perm_dst, ws, stream=None, x_perm_scales=None):
+    p, n = _ws(ws)
+    check("asap_moe_dispatch",
+          lib().asap_moe_dispatch(h.ptr, _ptr(x), x.shape[0], _ptr(idx), _ptr(x_perm), _ptr(x_perm_scales),
+                                  _ptr(perm_src), _ptr(perm_dst), p, n, _stream(stream)))
+
+
+def asap_moe_expert_ffn(h, x_perm, offsets, x, y_perm, y_shared, ws, stream=None, x_perm_scales=None):
+    p, n = _ws(ws)
+    check("asap_moe_expert_ffn",
+          lib().asap_moe_expert_ffn(h.ptr, _ptr(x_perm), _ptr(x_perm_scales), _ptr(offsets), _ptr(x),
+                                    x.shape[0], _ptr(y_perm), _ptr(y_shared), p, n, _stream(stream)))
+
+
+def asap_moe_combine(h, y_perm, y_shared, w, perm_dst, out, stream=None):
+    check("asap_moe_combine", lib().asap_moe_combine(h.ptr, _ptr(y_perm), _ptr(y_shared), _ptr(w), _ptr(perm_dst),
+                                                     out.shape[0], _ptr(out), _stream(stream)))
+
+
+def asap_moe_layer(h, x, out, ws, stream=None):
+    p, n = _ws(ws)
+    check("asap_moe_layer", lib().asap_moe_layer(h.ptr, _ptr(x), x.shape[0], _ptr(out), p, n, _stream(stream)))
+
+
+def asap_moe_status(h):
+    """(code, raw status word); code is ASAP_OK or ASAP_ERR_DEVICE_STATUS."""
+    word = ctypes.c_uint32()
+    code = lib().asap_moe_status(h.ptr, ctypes.byref(word))
+    return code, word.value
+
+
+def asap_moe_last_error():
+    return lib().asap_moe_last_error().decode(errors="replace")

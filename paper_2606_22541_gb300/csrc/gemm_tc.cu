@@ -1,0 +1,459 @@
+// Grouped GEMM on the sm_103a tensor core (tcgen05 + TMEM), fed by TMA.
+//
+// This is the expert computation of the MoE layer: a grouped matrix
+// multiplication with the token hidden states on the left and one layer's
+// expert weights on the right (ASAP Section 3.4.2).  Each expert e owns the
+// row segment [offsets[e], offsets[e+1]) of the grouped activations; the tile
+// list is derived on the device from those offsets, so the host never reads
+// the per-expert counts back (the bubble-free principle of Section 3.4.2).
+//
+// Design (one CTA per SM, persistent, warp-specialised, 192 threads):
+//   warp 0   : TMA producer.  A box [128 rows, 64 K] and B box [256 rows, 64 K],
+//              128-byte swizzle, into a 4-stage shared-memory ring.
+//   warp 1   : TMEM allocator and MMA issuer (one thread): 4 x
+//              tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) per stage,
+//              fp32 accumulator in TMEM, two accumulators (2 x 256 columns) so
+//              the epilogue of one tile overlaps the main loop of the next.
+//   warps 2-5: epilogue.  tcgen05.ld 32x32b (warp w reads TMEM lanes
+//              32*(w%4) ...), fused SwiGLU (gate and up columns of a tile are
+//              the two 128-column halves), bf16 or fp32 store.
+// Tile order: expert-major; inside an expert the m-tiles of one n-tile are
+// adjacent so CTAs running at the same time share the weight tile through L2.
+// Rows of a tile past the segment end belong to the next expert (or are
+// zero-filled by TMA past the tensor end) and are masked at the store.
+#include "common.cuh"
+#include "internal.h"
+
+#include <mutex>
+
+namespace asap {
+
+namespace {
+
+constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 2 * BN;
+constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+
+struct Sched {
+  int tile_start[kMaxExperts + 1];
+  int mtiles[kMaxExperts];
+  int row_base[kMaxExperts];
+  int mrows[kMaxExperts];
+};
+
+constexpr int kBarBytes = 256;  // 12 mbarriers + tmem slot + abort flag
+constexpr size_t kSmemBytes = 1024 + STAGES * (A_BYTES + B_BYTES) + kBarBytes + sizeof(Sched);
+
+struct Tile {
+  int a_row, b_row, rows, n_tile, kit;
+  bool p1;
+};
+
+__device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int total0,
+                                            const GemmArgs& a, Tile& T) {
+  if (t < total0) {
+    int lo = 0, hi = G;  // largest g with tile_start[g] <= t
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (s->tile_start[mid] <= t) lo = mid; else hi = mid;
+    }
+    const int g = lo;
+    const int local = t - s->tile_start[g];
+    const int mt = s->mtiles[g];
+    const int nt = local / mt;
+    const int mi = local - nt * mt;
+    T.a_row = s->row_base[g] + mi * BM;
+    T.rows = min(BM, s->mrows[g] - mi * BM);
+    T.b_row = g * a.b_stride0 + nt * BN;
+    T.n_tile = nt;
+    T.kit = a.k_iters0;
+    T.p1 = false;
+  } else {
+    const int u = t - total0;
+    const int mt = (a.m1 + BM - 1) / BM;
+    const int nt = u / mt;
+    const int mi = u - nt * mt;
+    T.a_row = mi * BM;
+    T.rows = min(BM, a.m1 - mi * BM);
+    T.b_row = nt * BN;
+    T.n_tile = nt;
+    T.kit = a.k_iters1;
+    T.p1 = true;
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr,
+                                              int row) {
+  const bool valid = row < T.rows;
+  const long long orow = static_cast<long long>(T.a_row) + row;
+  if constexpr (EPI == EPI_SWIGLU) {
+    uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
+    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
+    uint16_t* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * (BN / 2);
+#pragma unroll 1
+    for (int c = 0; c < BN / 2; c += 16) {
+      uint32_t g[16], u[16];
+      tmem_ld16(taddr + c, g);
+      tmem_ld16(taddr + BN / 2 + c, u);
+      tmem_ld_wait();
+      if (valid) {
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+          const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+          const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
+          const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
+          pk[i] = pack_bf16x2(h0, h1);
+        }
+        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+        d4[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        d4[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      }
+    }
+  } else if constexpr (EPI == EPI_BF16) {
+    uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
+    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
+    uint16_t* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * BN;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t v0[16], v1[16];
+      tmem_ld16(taddr + c, v0);
+      tmem_ld16(taddr + c + 16, v1);
+      tmem_ld_wait();
+      if (valid) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          pk[i] = pack_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
+          pk[8 + i] = pack_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
+        }
+        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) d4[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+      }
+    }
+  } else {
+    float* out = static_cast<float*>(T.p1 ? a.out1 : a.out0);
+    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
+    float* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * BN;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 16) {
+      uint32_t v[16];
+      tmem_ld16(taddr + c, v);
+      tmem_ld_wait();
+      if (valid) {
+        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) d4[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+    }
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                        const __grid_constant__ CUtensorMap tmB0,
+                        const __grid_constant__ CUtensorMap tmA1,
+                        const __grid_constant__ CUtensorMap tmB1, const GemmArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sA = base;
+  const uint32_t sB = base + STAGES * A_BYTES;
+  uint8_t* bar_area = gbase + STAGES * (A_BYTES + B_BYTES);
+  const uint32_t bar0 = smem_u32(bar_area);
+  // mbarriers (8 bytes each): full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * STAGES + 5));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int G = args.offsets ? args.groups : 1;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int s = 0; s < STAGES; ++s) {
+        mbar_init(full_bar(s), 1);
+        mbar_init(empty_bar(s), 1);
+      }
+      for (int a = 0; a < 2; ++a) {
+        mbar_init(tfull_bar(a), 1);
+        mbar_init(tempty_bar(a), 128);
+      }
+      mbar_init(drain_bar, 1);
+      *abort_flag = 0;
+      fence_barrier_init();
+      tma_prefetch_desc(&tmA0);
+      tma_prefetch_desc(&tmB0);
+      if (args.m1 > 0) {
+        tma_prefetch_desc(&tmA1);
+        tma_prefetch_desc(&tmB1);
+      }
+    }
+    // Per-group m-tile counts and their exclusive prefix (warp scan; each
+    // lane owns up to 8 consecutive groups).  Bad offsets -> empty group.
+    int local = 0;
+    int cnt[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int g = lane * 8 + i;
+      cnt[i] = 0;
+      if (g < G) {
+        int lo = 0, m = args.m0;
+        if (args.offsets) {
+          lo = __ldg(args.offsets + g);
+          const int hi = __ldg(args.offsets + g + 1);
+          m = hi - lo;
+          if (lo < 0 || m < 0 || hi > args.m0) {
+            record_status(args.status, ST_BAD_OFFSETS);
+            lo = 0;
+            m = 0;
+          }
+        }
+        sch->row_base[g] = lo;
+        sch->mrows[g] = m;
+        cnt[i] = (m + BM - 1) / BM;
+        sch->mtiles[g] = cnt[i];
+        local += cnt[i] * args.n_tiles0;
+      }
+    }
+    int incl = local;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    int run = incl - local;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int g = lane * 8 + i;
+      if (g < G) {
+        sch->tile_start[g] = run;
+        run += cnt[i] * args.n_tiles0;
+      }
+    }
+    if (lane == 31) sch->tile_start[G] = incl;
+  } else if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total0 = sch->tile_start[G];
+  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ producer
+    const uint64_t pol_a = l2_policy(args.hint_a);
+    const uint64_t pol_b = l2_policy(args.hint_b);
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t pending = 0, issued_phase = 0;  // bit s: stage s has a load in flight
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      const CUtensorMap* mA = T.p1 ? &tmA1 : &tmA0;
+      const CUtensorMap* mB = T.p1 ? &tmB1 : &tmB0;
+      for (int kb = 0; kb < T.kit; ++kb) {
+        if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(full_bar(stage), A_BYTES + B_BYTES);
+        tma_load_2d(sA + stage * A_BYTES, mA, full_bar(stage), kb * BK, T.a_row, pol_a);
+        tma_load_2d(sB + stage * B_BYTES, mB, full_bar(stage), kb * BK, T.b_row, pol_b);
+        pending |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      record_status(args.status, ST_WAIT_TIMEOUT);
+      // let the copies already issued land before the CTA's memory goes away
+      int dummy = 0;
+      for (int s = 0; s < STAGES; ++s)
+        if (pending & (1u << s)) mbar_wait(full_bar(s), (issued_phase >> s) & 1u, &dummy);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true, issued = false;
+    int it = 0;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d = tmem_base + acc * BN;
+      for (int kb = 0; kb < T.kit; ++kb) {
+        if (!mbar_wait(full_bar(stage), phase, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_addr = sA + stage * A_BYTES;
+        const uint32_t b_addr = sB + stage * B_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          tc_mma_bf16(d, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kIdesc,
+                      (kb | kk) != 0);
+        }
+        issued = true;
+        tc_commit(empty_bar(stage));
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (ok) tc_commit(tfull_bar(acc));
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      record_status(args.status, ST_WAIT_TIMEOUT);
+      if (issued) {
+        int dummy = 0;
+        tc_commit(drain_bar);
+        mbar_wait(drain_bar, 0, &dummy);
+      }
+    }
+  } else if (warp >= 2) {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    int it = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(tfull_bar(acc), acc_phase, abort_flag));
+      if (!ok) {
+        if (lane == 0) {
+          *abort_flag = 1;
+          record_status(args.status, ST_WAIT_TIMEOUT);
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      epilogue_tile<EPI>(T, args, taddr, row);
+      tc_fence_before();
+      mbar_arrive(tempty_bar(acc));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+template <int EPI>
+cudaError_t set_attr() {
+  return cudaFuncSetAttribute(grouped_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(kSmemBytes));
+}
+
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                              CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                              CUtensorMapFloatOOBfill);
+
+EncodeFn get_encode_fn() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(p);
+  });
+  return fn;
+}
+
+}  // namespace
+
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(sizeof(Sched) + 0 <= 8192, "schedule table");
+
+cudaError_t gemm_set_attributes() {
+  cudaError_t e = set_attr<EPI_SWIGLU>();
+  if (e == cudaSuccess) e = set_attr<EPI_BF16>();
+  if (e == cudaSuccess) e = set_attr<EPI_F32>();
+  return e;
+}
+
+cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, int grid,
+                        cudaStream_t stream) {
+  if (grid <= 0) return cudaSuccess;
+  const dim3 g(grid), b(kThreads);
+  switch (epi) {
+    case EPI_SWIGLU:
+      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      break;
+    case EPI_BF16:
+      grouped_gemm_kernel<EPI_BF16><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      break;
+    default:
+      grouped_gemm_kernel<EPI_F32><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      break;
+  }
+  return cudaGetLastError();
+}
+
+bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
+                      uint32_t box_rows, std::string* err) {
+  EncodeFn fn = get_encode_fn();
+  if (!fn) {
+    if (err) *err = "cuTensorMapEncodeTiled is not available from the driver";
+    return false;
+  }
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0 || (cols * 2) % 16 != 0 || rows == 0) {
+    if (err) *err = "tensor for TMA must be 16-byte aligned with 16-byte row stride and >= 1 row";
+    return false;
+  }
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (err) *err = "cuTensorMapEncodeTiled failed with CUresult " + std::to_string(static_cast<int>(r));
+    return false;
+  }
+  return true;
+}
+
+}  // namespace asap

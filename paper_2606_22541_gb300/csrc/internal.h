@@ -1,0 +1,81 @@
+// Host-side declarations shared by the translation units of libasap_moe.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+namespace asap {
+
+// ------------------------------------------------------------ grouped GEMM
+// One launch computes up to two problems with the same epilogue:
+//  problem 0: ``groups`` row segments of A (segment g = rows
+//             [offsets[g], offsets[g+1]) ), each multiplied by its own B block
+//             (rows g*b_stride0 ... of the B tensor); or, with offsets ==
+//             nullptr, one plain GEMM of m0 rows.
+//  problem 1: one plain GEMM of m1 rows (the shared expert), optional.
+// C = A B^T with A [rows, K] and B [N, K] both K-major bf16.
+enum { EPI_SWIGLU = 0, EPI_BF16 = 1, EPI_F32 = 2 };
+
+struct GemmArgs {
+  const int32_t* offsets;  // [groups + 1] or nullptr
+  int groups;              // 1 when offsets == nullptr
+  int m0;                  // rows of A0 (segment ends are checked against it)
+  int b_stride0;           // B0 rows between consecutive groups
+  int n_tiles0;            // 256-wide N tiles per group
+  int k_iters0;            // K0 / 64
+  void* out0;
+  long long ldo0;          // elements between output rows
+  int m1;                  // rows of problem 1 (0 = none)
+  int n_tiles1;
+  int k_iters1;
+  void* out1;
+  long long ldo1;
+  uint32_t* status;
+  int hint_a, hint_b;      // L2 priority of A / B loads: 0 normal, 1 first, 2 last
+};
+
+constexpr int kGemmBM = 128;
+constexpr int kGemmBN = 256;
+constexpr int kGemmBK = 64;
+
+cudaError_t gemm_set_attributes();
+// maps: A0, B0, A1, B1 (A1/B1 may repeat A0/B0 when m1 == 0)
+cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, int grid,
+                        cudaStream_t stream);
+// Encode a 2-D row-major bf16 tensor [rows, cols] for 128-byte-swizzled
+// boxes of [box_rows, 64].  Returns false and fills *err on failure.
+bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
+                      uint32_t box_rows, std::string* err);
+
+// ------------------------------------------------------------ routing
+struct GateParams {
+  int n_experts, top_k, gating, n_groups, topk_groups;
+  float route_scale;
+  const float* bias;  // [E] or nullptr
+};
+cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int E, float* logits,
+                                cudaStream_t s);
+cudaError_t launch_gate(const float* logits, int n, const GateParams& p, int32_t* idx, float* w,
+                        int32_t* hist, cudaStream_t s);
+cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
+                        cudaStream_t s);
+cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
+                        int32_t* chunk_base, cudaStream_t s);
+
+// ------------------------------------------------------------ permute
+cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                            const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
+                            int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float* w,
+                           const int32_t* perm_dst, int n, int H, int k, void* out,
+                           uint32_t* status, cudaStream_t s);
+// packed[e][b*256 + r] = gate[e][b*128 + r] (r < 128), up[...] for r >= 128
+cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, int H, void* packed,
+                                cudaStream_t s);
+
+inline int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
+
+}  // namespace asap

@@ -1,0 +1,83 @@
+"""The C-ABI library loads on a machine without a GPU, exports every entry
+point the header declares, and its pure-host calls (config checks, workspace
+sizing, argument validation) behave as documented.  No compute calls."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_22541_gb300 import _native, build as build_mod
+from paper_2606_22541_gb300.configs import CONFIGS, DSV3, TINY
+from paper_2606_22541_gb300 import api
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "asap_moe.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    build_mod.build()
+    return _native.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(asap_moe_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("asap_moe_route", "asap_moe_dispatch", "asap_moe_expert_ffn",
+                     "asap_moe_combine", "asap_moe_layer", "asap_moe_create", "asap_moe_destroy"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    assert set(declared_functions()) == set(_native.SIGNATURES)
+
+
+def test_check_config(L):
+    for c in CONFIGS.values():
+        code = api.asap_moe_check_config(c, 4096)
+        if c.dtype == "bf16":
+            assert code == _native.ASAP_OK, api.asap_moe_last_error()
+        else:
+            assert code == _native.ASAP_ERR_UNSUPPORTED
+    from dataclasses import replace
+    bad = [replace(TINY, hidden=200), replace(TINY, top_k=9), replace(TINY, inter=100),
+           replace(DSV3, n_groups=7), replace(DSV3, topk_groups=0), replace(TINY, n_experts=300),
+           replace(TINY, gating="softmax", top_k=0)]
+    for b in bad:
+        assert api.asap_moe_check_config(b, 16) == _native.ASAP_ERR_INVALID
+    assert api.asap_moe_check_config(TINY, 0) == _native.ASAP_ERR_INVALID
+
+
+def test_workspace_size(L):
+    assert api.asap_moe_workspace_size(TINY, 0, 100) == 0
+    a = api.asap_moe_workspace_size(DSV3, 4096)
+    b = api.asap_moe_workspace_size(DSV3, 4097)
+    assert b > a > 4096 * 8 * 7168 * 2   # at least the grouped hidden states
+    assert a % 256 == 0
+    with pytest.raises(_native.AsapError):
+        api.asap_moe_workspace_size(TINY, 10, 5)
+
+
+def test_create_rejects_bad_arguments_before_touching_cuda(L):
+    c = api.make_config(TINY, 16)
+    w = _native.AsapMoeWeights()
+    out = ctypes.c_void_p(1234)
+    assert L.asap_moe_create(ctypes.byref(c), ctypes.byref(w), ctypes.byref(out)) == _native.ASAP_ERR_INVALID
+    assert out.value is None
+    assert "required" in api.asap_moe_last_error()
+    assert L.asap_moe_create(None, ctypes.byref(w), ctypes.byref(out)) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_destroy(None) == _native.ASAP_OK
+
+
+def test_calls_reject_null_handle(L):
+    assert L.asap_moe_layer(None, None, 1, None, None, 0, None) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_combine(None, None, None, None, None, 1, None, None) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_status(None, None) == _native.ASAP_ERR_INVALID

@@ -1,0 +1,388 @@
+"""Parity of the CUDA path (through the C ABI) with the float64 oracle, on
+seeded inputs: each step and the whole layer, shapes spanning several tiles
+with ragged tails, edge cases, and the multi-stream submission model."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_22541_gb300 import api, inputs
+from paper_2606_22541_gb300.configs import TINY, MIXTRAL, DSV3, STRESS
+
+from _helpers import bf16_to_f64, weights_f64, compare_rows, routing_check
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+# Reduced shapes of the Mixtral and DeepSeek-V3 layers: several 128-row tiles,
+# ragged segments, empty experts, the tensor-core router (E = 256) and the
+# shared expert, small enough for the oracle to finish in seconds.
+MX_SMALL = inputs.small_variant(MIXTRAL, name="mixtral_small", hidden=1024, inter=512, microbatches=[1000, 333])
+DS_SMALL = inputs.small_variant(DSV3, name="dsv3_small", hidden=512, inter=256, shared_inter=256,
+                                microbatches=[300, 77])
+ST_SMALL = inputs.small_variant(STRESS, name="stress_small", hidden=512, inter=256, shared_inter=256,
+                                microbatches=[700, 129, 1])
+SMALL = [TINY, MX_SMALL, DS_SMALL, ST_SMALL]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+class Case:
+    """Weights on the GPU, their float64 copies and a handle."""
+    _cache = {}
+
+    @classmethod
+    def get(cls, cfg):
+        if cfg.name not in cls._cache:
+            cls._cache[cfg.name] = cls(cfg)
+        return cls._cache[cfg.name]
+
+    def __init__(self, cfg):
+        self.cfg = cfg
+        self.w = inputs.make_weights(cfg, DEV)
+        self.h = api.asap_moe_create(cfg, self.w, max(cfg.microbatches))
+        self.wf = weights_f64(self.w)
+        self.ocfg = cfg.oracle_cfg()
+        self.shared = (self.wf["sh_gate"], self.wf["sh_up"], self.wf["sh_down"]) if cfg.n_shared else None
+
+    def tokens(self, i, n=None):
+        n = self.cfg.microbatches[i] if n is None else n
+        return inputs.make_tokens(self.cfg, n, i, DEV)
+
+    def ws(self, n):
+        return api.workspace(self.h, n)
+
+
+def run_route(c, x):
+    n = x.shape[0]
+    k, E = c.cfg.top_k, c.cfg.n_experts
+    idx = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    w = torch.empty((n, k), dtype=torch.float32, device=DEV)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    api.asap_moe_route(c.h, x, idx, w, counts, offsets, c.ws(n))
+    torch.cuda.synchronize()
+    return idx, w, counts, offsets
+
+
+def assert_clean(c):
+    code, word = api.asap_moe_status(c.h)
+    assert code == 0 and word == 0, f"device status word {word:#x}"
+
+
+# ---------------------------------------------------------------- routing
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+def test_router_logits_within_bound(cfg):
+    c = Case.get(cfg)
+    x = c.tokens(0)
+    logits = torch.empty((x.shape[0], cfg.n_experts), dtype=torch.float32, device=DEV)
+    api.asap_moe_router_logits(c.h, x, logits)
+    torch.cuda.synchronize()
+    xf = bf16_to_f64(x)
+    L = oracle.router_logits(xf, c.wf["router_w"])
+    eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+    err = np.abs(logits.cpu().numpy().astype(np.float64) - L)
+    assert (err <= eps).all(), f"max err/bound {float((err / eps).max()):.3f}"
+    assert_clean(c)
+
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+def test_route_matches_oracle(cfg):
+    c = Case.get(cfg)
+    for i in range(len(cfg.microbatches)):
+        x = c.tokens(i)
+        idx, w, counts, offsets = run_route(c, x)
+        xf = bf16_to_f64(x)
+        L = oracle.router_logits(xf, c.wf["router_w"])
+        eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+        idx_ref, w_ref = oracle.route(L, c.ocfg)
+        ig = idx.cpu().numpy().astype(np.int64)
+        decided = routing_check(L, eps, c.ocfg, ig, w.cpu().numpy().astype(np.float64), w_ref, idx_ref)
+        # counts / offsets: the histogram of the returned idx and its scan
+        cg = counts.cpu().numpy()
+        og = offsets.cpu().numpy()
+        assert np.array_equal(cg, np.bincount(ig.reshape(-1), minlength=cfg.n_experts))
+        assert og[0] == 0 and np.array_equal(np.diff(og), cg) and og[-1] == ig.size
+        if decided.all():
+            assert np.array_equal(cg, oracle.expert_counts(idx_ref, cfg.n_experts))
+            assert np.array_equal(og, oracle.expert_offsets(oracle.expert_counts(idx_ref, cfg.n_experts)))
+    assert_clean(c)
+
+
+def test_route_logits_exact_ties():
+    c = Case.get(TINY)
+    n, E = 130, TINY.n_experts
+    rng = np.random.default_rng(7)
+    L = np.round(rng.normal(0, 1, (n, E)) * 2) / 2          # many exact ties
+    L[5] = 0.0                                              # every expert tied
+    L[6] = [1, 1, 1, 0, 0, 0, 0, 0]
+    lg = torch.tensor(L, dtype=torch.float32, device=DEV)
+    idx = torch.empty((n, 2), dtype=torch.int32, device=DEV)
+    w = torch.empty((n, 2), dtype=torch.float32, device=DEV)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    api.asap_moe_route_logits(c.h, lg, idx, w, counts, offsets, c.ws(n))
+    torch.cuda.synchronize()
+    idx_ref, w_ref = oracle.route(L, c.ocfg)
+    assert np.array_equal(idx.cpu().numpy(), idx_ref)
+    assert np.allclose(w.cpu().numpy(), w_ref, rtol=1e-6, atol=0)
+    assert list(idx_ref[5]) == [0, 1] and list(idx_ref[6]) == [0, 1]
+    assert np.array_equal(counts.cpu().numpy(), oracle.expert_counts(idx_ref, E))
+    assert np.array_equal(offsets.cpu().numpy(), oracle.expert_offsets(oracle.expert_counts(idx_ref, E)))
+
+
+def test_route_logits_grouped_exact_ties_and_all_to_one_group():
+    c = Case.get(DS_SMALL)
+    n, E = 70, 256
+    rng = np.random.default_rng(8)
+    L = np.round(rng.normal(0, 1, (n, E)) * 4) / 4
+    L[0] = 0.0                       # everything tied: groups 0-3, experts 0..7
+    L[1] = -5.0
+    L[1, 64:72] = 3.0                # one group holds all 8 picks
+    L[2] = -5.0
+    L[2, 200] = 4.0                  # a single hot expert
+    lg = torch.tensor(L, dtype=torch.float32, device=DEV)
+    idx = torch.empty((n, 8), dtype=torch.int32, device=DEV)
+    w = torch.empty((n, 8), dtype=torch.float32, device=DEV)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    api.asap_moe_route_logits(c.h, lg, idx, w, counts, offsets, c.ws(n))
+    torch.cuda.synchronize()
+    idx_ref, w_ref = oracle.route(L, c.ocfg)
+    # float32 sigmoid may merge logits the float64 one separates; the
+    # quarter-step logits here keep every tie exact or well separated
+    eps = np.zeros_like(L)
+    ig = idx.cpu().numpy().astype(np.int64)
+    routing_check(L, eps, c.ocfg, ig, w.cpu().numpy().astype(np.float64), w_ref, idx_ref)
+    assert list(idx_ref[0]) == list(range(8))
+    assert list(idx_ref[1]) == list(range(64, 72))
+    # constructed exact ties resolve bit-exactly by the lower-index rule
+    for t in range(3):
+        assert list(ig[t]) == list(idx_ref[t])
+
+
+# ---------------------------------------------------------------- dispatch / combine
+
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
+def test_dispatch_exact(cfg):
+    c = Case.get(cfg)
+    n, k, E, H = 333, cfg.top_k, cfg.n_experts, cfg.hidden
+    if n > max(cfg.microbatches):
+        n = max(cfg.microbatches)
+    rng = np.random.default_rng(9)
+    idx_np = np.array([rng.permutation(E)[:k] for _ in range(n)], np.int64).reshape(n, k)
+    idx_np[: n // 3, 0] = 1                     # make expert 1 hot
+    idx_np[: n // 3, 1:] = np.array([rng.permutation(np.arange(2, E))[:k - 1] for _ in range(n // 3)])
+    x = c.tokens(0, n)
+    idx = torch.tensor(idx_np, dtype=torch.int32, device=DEV)
+    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(c.h, x, idx, x_perm, perm_src, perm_dst, c.ws(n))
+    torch.cuda.synchronize()
+    src_ref, dst_ref = oracle.permutation(idx_np, E)
+    assert np.array_equal(perm_src.cpu().numpy(), src_ref)
+    assert np.array_equal(perm_dst.cpu().numpy(), dst_ref)
+    assert np.array_equal(bf16_to_f64(x_perm), oracle.dispatch(bf16_to_f64(x), src_ref))
+    assert_clean(c)
+
+
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
+def test_identity_experts_return_k_x(cfg):
+    """dispatch then combine with y_perm = x_perm and unit weights gives k*x
+    exactly (k a power of two, so k*x is a bf16 value)."""
+    c = Case.get(cfg)
+    n, k, E, H = max(cfg.microbatches), cfg.top_k, cfg.n_experts, cfg.hidden
+    x = c.tokens(1 if len(cfg.microbatches) > 1 else 0, n)
+    idx, w, counts, offsets = run_route(c, x)
+    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(c.h, x, idx, x_perm, perm_src, perm_dst, c.ws(n))
+    out = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+    ones = torch.ones((n, k), dtype=torch.float32, device=DEV)
+    api.asap_moe_combine(c.h, x_perm, None, ones, perm_dst, out)
+    torch.cuda.synchronize()
+    assert np.array_equal(bf16_to_f64(out), k * bf16_to_f64(x))
+    assert_clean(c)
+
+
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
+def test_combine_matches_oracle(cfg):
+    c = Case.get(cfg)
+    n, k, H = 150, cfg.top_k, cfg.hidden
+    n = min(n, max(cfg.microbatches))
+    rng = np.random.default_rng(10)
+    y_perm = inputs.randn_bf16((n * k, H), 1.0, 77, DEV)
+    y_sh = inputs.randn_bf16((n, H), 1.0, 78, DEV)
+    perm = rng.permutation(n * k).reshape(n, k)
+    w_np = rng.uniform(0.01, 1.0, (n, k)).astype(np.float32)
+    out = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+    api.asap_moe_combine(c.h, y_perm, y_sh, torch.tensor(w_np, device=DEV),
+                         torch.tensor(perm, dtype=torch.int32, device=DEV), out)
+    torch.cuda.synchronize()
+    ref = oracle.combine(bf16_to_f64(y_perm), w_np.astype(np.float64), perm, bf16_to_f64(y_sh))
+    g = bf16_to_f64(out)
+    # fp32 accumulation then one bf16 rounding: within one bf16 ulp of the
+    # exact sum plus the fp32 accumulation error
+    tol = np.abs(ref) * 2.0 ** -8 + 1e-5 * (np.abs(bf16_to_f64(y_perm)).max() * k + 1)
+    assert (np.abs(g - ref) <= tol).all()
+    assert_clean(c)
+
+
+# ---------------------------------------------------------------- expert FFN
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+def test_expert_ffn_matches_oracle(cfg):
+    """Grouped GEMMs on oracle-made segments: empty experts, one hot expert,
+    segments that are not multiples of 128 rows."""
+    c = Case.get(cfg)
+    n, k, E, H = max(cfg.microbatches), cfg.top_k, cfg.n_experts, cfg.hidden
+    rng = np.random.default_rng(11)
+    counts = rng.multinomial(n * k, np.r_[0.3, np.full(E - 1, 0.7 / (E - 1))])
+    counts[E // 2 + 1] += counts[E // 2]      # one empty expert, total kept at n*k
+    counts[E // 2] = 0
+    offsets_np = oracle.expert_offsets(counts)
+    x = c.tokens(0, n)
+    x_perm = inputs.randn_bf16((n * k, H), 1.0, 90, DEV)
+    y_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=DEV) if cfg.n_shared else None
+    offsets = torch.tensor(offsets_np, dtype=torch.int32, device=DEV)
+    api.asap_moe_expert_ffn(c.h, x_perm, offsets, x, y_perm, y_sh, c.ws(n))
+    torch.cuda.synchronize()
+    ref = oracle.expert_ffn(bf16_to_f64(x_perm), offsets_np, c.wf["w_gate"], c.wf["w_up"], c.wf["w_down"])
+    compare_rows(bf16_to_f64(y_perm), ref)
+    if cfg.n_shared:
+        compare_rows(bf16_to_f64(y_sh), oracle.swiglu(bf16_to_f64(x), *c.shared))
+    assert_clean(c)
+
+
+# ---------------------------------------------------------------- whole layer
+
+def oracle_layer(c, x):
+    return oracle.moe_layer(bf16_to_f64(x), c.wf["router_w"], c.wf["w_gate"], c.wf["w_up"], c.wf["w_down"],
+                            c.ocfg, shared=c.shared)
+
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+def test_layer_matches_oracle(cfg):
+    c = Case.get(cfg)
+    for i, n in enumerate(cfg.microbatches):
+        x = c.tokens(i)
+        out = torch.empty((n, cfg.hidden), dtype=torch.bfloat16, device=DEV)
+        api.asap_moe_layer(c.h, x, out, c.ws(n))
+        torch.cuda.synchronize()
+        r = oracle_layer(c, x)
+        idx, w, _, _ = run_route(c, x)
+        xf = bf16_to_f64(x)
+        eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+        decided = routing_check(r["logits"], eps, c.ocfg, idx.cpu().numpy().astype(np.int64),
+                                w.cpu().numpy().astype(np.float64), r["w"], r["idx"])
+        compare_rows(bf16_to_f64(out)[decided], r["y"][decided])
+    assert_clean(c)
+
+
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
+def test_layer_equals_composed_calls_bit_for_bit(cfg):
+    c = Case.get(cfg)
+    n, k, E, H = cfg.microbatches[0], cfg.top_k, cfg.n_experts, cfg.hidden
+    x = c.tokens(0)
+    ws = c.ws(n)
+    out = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+    api.asap_moe_layer(c.h, x, out, ws)
+    idx, w, counts, offsets = run_route(c, x)
+    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(c.h, x, idx, x_perm, perm_src, perm_dst, ws)
+    y_perm = torch.empty_like(x_perm)
+    y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=DEV) if cfg.n_shared else None
+    api.asap_moe_expert_ffn(c.h, x_perm, offsets, x, y_perm, y_sh, ws)
+    out2 = torch.empty_like(out)
+    api.asap_moe_combine(c.h, y_perm, y_sh, w, perm_dst, out2)
+    torch.cuda.synchronize()
+    assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
+    assert_clean(c)
+
+
+@pytest.mark.parametrize("cfg", [DS_SMALL, ST_SMALL], ids=lambda c: c.name)
+def test_streams_concurrent_equals_serial_and_token_independent(cfg):
+    """Micro-batches submitted on their own streams with no host barrier give
+    the same bits as one stream; a token's output does not depend on the
+    micro-batch it arrived in."""
+    c = Case.get(cfg)
+    xs = [c.tokens(i) for i in range(len(cfg.microbatches))]
+    wss = [c.ws(x.shape[0]) for x in xs]
+    serial = []
+    for x, ws in zip(xs, wss):
+        o = torch.empty_like(x)
+        api.asap_moe_layer(c.h, x, o, ws)
+        serial.append(o)
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream() for _ in xs]
+    conc = [torch.empty_like(x) for x in xs]
+    for x, o, ws, s in zip(xs, conc, wss, streams):
+        s.wait_stream(torch.cuda.current_stream())
+        api.asap_moe_layer(c.h, x, o, ws, stream=s)
+    torch.cuda.synchronize()
+    for a, b in zip(serial, conc):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    # regroup: the first 50 tokens of micro-batch 0 as a batch of their own
+    x0 = xs[0][:50].contiguous()
+    o0 = torch.empty_like(x0)
+    api.asap_moe_layer(c.h, x0, o0, c.ws(50))
+    torch.cuda.synchronize()
+    assert torch.equal(o0.view(torch.int16), serial[0][:50].view(torch.int16))
+    assert_clean(c)
+
+
+def test_edge_sizes():
+    c = Case.get(DS_SMALL)
+    H = DS_SMALL.hidden
+    # n = 0 is a no-op
+    x = c.tokens(0, 1)
+    out = torch.full((1, H), 7.0, dtype=torch.bfloat16, device=DEV)
+    api.asap_moe_layer(c.h, x[:0], out[:0], None)
+    # n = 1 and the maximum n
+    for n in (1, max(DS_SMALL.microbatches)):
+        x = c.tokens(0, n)
+        out = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+        api.asap_moe_layer(c.h, x, out, c.ws(n))
+        torch.cuda.synchronize()
+        r = oracle_layer(c, x)
+        eps = oracle.logit_error_bound(bf16_to_f64(x), c.wf["router_w"])
+        dec = np.array([oracle.token_decided(r["logits"][t], eps[t], c.ocfg) for t in range(n)])
+        compare_rows(bf16_to_f64(out)[dec], r["y"][dec])
+    # n > max_tokens and a short workspace are rejected without launching
+    from paper_2606_22541_gb300._native import AsapError
+    big = c.tokens(0, max(DS_SMALL.microbatches) + 1)
+    with pytest.raises(AsapError):
+        api.asap_moe_layer(c.h, big, torch.empty_like(big), c.ws(max(DS_SMALL.microbatches)))
+    x = c.tokens(0, 10)
+    with pytest.raises(AsapError):
+        api.asap_moe_layer(c.h, x, torch.empty_like(x), c.ws(5))
+    assert_clean(c)
+
+
+def test_bad_indices_are_reported_not_trapped():
+    c = Case.get(TINY)
+    n, k, H = 20, 2, TINY.hidden
+    x = c.tokens(0, n)
+    idx = torch.zeros((n, k), dtype=torch.int32, device=DEV)
+    idx[:, 1] = 1
+    idx[3, 0] = 99                                           # out of range
+    x_perm = torch.zeros((n * k, H), dtype=torch.bfloat16, device=DEV)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(c.h, x, idx, x_perm, perm_src, perm_dst, c.ws(n))
+    code, word = api.asap_moe_status(c.h)
+    assert code != 0 and (word & 1)
+    assert perm_dst[3, 0].item() == -1
+    code, word = api.asap_moe_status(c.h)                   # cleared by the read
+    assert code == 0 and word == 0
