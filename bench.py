@@ -1,0 +1,544 @@
+#!/usr/bin/env python
+"""Throughput of the expert-side MoE layer on one GB300 (and N replicas).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Workload (default): the DeepSeek-V3-shaped BF16 MoE layer of the paper's
+evaluation model (ASAP Table 1 and Section 5.1: H = 7168, 256 routed experts
+plus 1 shared, top-8; intermediate 2048), 16384 tokens per step as 4
+micro-batches of 4096 tokens, each submitted through asap_moe_layer on its
+own CUDA stream with no host barrier between them (Section 3.4.2).  Inputs
+are seeded synthetic tensors; 22.6 GB of expert weights make every step's
+working set far larger than the 129 MB L2.
+
+One JSON line on rank 0: tokens/s over the timed steps, plus the roofline of
+the dominant kernel (the gate/up grouped GEMM), per-kernel timings measured
+with CUDA events on the stream each kernel runs on, the float64 oracle timed
+on the host cores on a bounded sample, the end-to-end figure through host
+buffers, and the SM clocks sampled during the timed region.
+
+``--impl reference`` times the float64 oracle instead (host cores, bounded
+sample per step) on the same workload and metric.
+"""
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MoE-layer prefill tokens/s on 1 GB300; grouped-GEMM % of tensor peak"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="dsv3_bf16")
+    ap.add_argument("--kernel-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-tokens", type=int, default=2)
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------ distributed plumbing
+
+class Dist:
+    """Control plane of N independent replicas: barrier and max-reduce only."""
+
+    def __init__(self):
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.init_process_group("gloo")
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, v):
+        if not self.pg:
+            return v
+        import torch
+        t = torch.tensor([float(v)], dtype=torch.float64)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(parts[1]), max=float(parts[2]), power=float(parts[3]),
+                                 hw=parts[5], hwt=parts[6], swt=parts[7], swp=parts[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        load = [r for r in rows if r["power"] > 300.0] or rows
+        reasons = set()
+        for r in load:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("swp", "sw_power_cap")):
+                if r[key].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r["sm"] for r in load), "sm_max_mhz": max(r["max"] for r in rows),
+                "samples": len(rows), "samples_under_load": len(load),
+                "power_w_max": max(r["power"] for r in rows), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------ oracle baseline (host cores)
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_tokens(cfg, x_tokens, device):
+    """Run the float64 oracle on a few tokens of the workload: routing over all
+    experts, then each token's 8 routed experts and the shared expert, with
+    every weight matrix decoded from bf16 by the oracle as it reads it.
+    Returns the outputs (float64)."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2606_22541_gb300 import inputs
+
+    def f64(t):
+        return oracle.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16))
+
+    xf = f64(x_tokens)
+    wr = f64(inputs.router_weights_bf16(cfg, device))
+    L = oracle.router_logits(xf, wr)
+    idx, w = oracle.route(L, cfg.oracle_cfg())
+    shared = tuple(f64(t) for t in inputs.shared_weights_bf16(cfg, device)) if cfg.n_shared else None
+
+    def expert(e, which):
+        return f64(inputs.expert_weights_bf16(cfg, e, device)[which])
+
+    # per-expert callables decode on demand, as the oracle's layer functions allow
+    return oracle.moe_layer_tokens(xf, idx, w, lambda e: expert(e, 0), lambda e: expert(e, 1),
+                                   lambda e: expert(e, 2), shared)
+
+
+def cpu_baseline(cfg, device, n_tokens):
+    from paper_2606_22541_gb300 import inputs
+    x = inputs.make_tokens(cfg, n_tokens, 0, device)
+    t0 = time.perf_counter()
+    oracle_tokens(cfg, x, device)
+    dt = time.perf_counter() - t0
+    return {"value": n_tokens / dt, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
+            "sample": f"{n_tokens} tokens of micro-batch 0: float64 routing over all {cfg.n_experts} experts, "
+                      f"then each token's {cfg.top_k} routed experts and the shared expert with weights decoded "
+                      f"from bf16 per expert ({dt:.1f} s); numpy elementwise work on one thread, BLAS on up to "
+                      f"{host_cores()} threads"}
+
+
+# ------------------------------------------------------------ roofline evidence
+
+def profile_traffic(name, source_files):
+    """Per-launch DRAM bytes from a committed ncu summary, or None when the
+    summary is missing or the kernel's sources changed since it was taken."""
+    path = os.path.join(ROOT, "profiles", name)
+    if not os.path.exists(path):
+        return None, None
+    text = open(path).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    h = re.search(r"source_sha256:\s*([0-9a-f]+)", text)
+    if not m or not h:
+        return None, None
+    if h.group(1) != sources_sha256(source_files):
+        return None, "stale"
+    return float(m.group(1)), path
+
+
+def sources_sha256(files):
+    d = hashlib.sha256()
+    for f in files:
+        d.update(open(os.path.join(ROOT, f), "rb").read())
+    return d.hexdigest()
+
+
+GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb300/csrc/common.cuh"]
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ------------------------------------------------------------ our arm
+
+def run_ours(args, dist):
+    import numpy as np
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_22541_gb300 import api, inputs
+    from paper_2606_22541_gb300.configs import CONFIGS
+
+    cfg = CONFIGS[args.workload]
+    torch.cuda.set_device(dist.local_rank)
+    dev = f"cuda:{dist.local_rank}"
+    mbs = cfg.microbatches
+    n_max = max(mbs)
+    weights = inputs.make_weights(cfg, dev)
+    h = api.asap_moe_create(cfg, weights, n_max)
+    del weights
+    torch.cuda.empty_cache()
+    xs = inputs.make_microbatches(cfg, dev)
+    outs = [torch.empty_like(x) for x in xs]
+    wss = [api.workspace(h, x.shape[0], dev) for x in xs]
+    streams = [torch.cuda.Stream(device=dev) for _ in xs]
+    main = torch.cuda.current_stream()
+    tokens_per_step = sum(mbs)
+
+    def step():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for x, o, ws, s in zip(xs, outs, wss, streams):
+            s.wait_event(ev)                       # device-side ordering only
+            api.asap_moe_layer(h, x, o, ws, stream=s)
+        for s in streams:
+            main.wait_stream(s)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(dist.local_rank)
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(main)
+    for _ in range(args.steps):
+        step()
+    t_end.record(main)
+    torch.cuda.synchronize()
+    dist.barrier()
+    clk = clocks.stop()
+    elapsed_ms = dist.max(t_start.elapsed_time(t_end))
+    code, word = api.asap_moe_status(h)
+    if code != 0:
+        raise RuntimeError(f"device status word {word:#x} after the timed region")
+    launches_per_mb = 7   # router GEMM, gate, scan, dispatch, gate/up GEMM, down GEMM, combine
+    result = {
+        "metric": METRIC,
+        "value": dist.world * tokens_per_step * args.steps / (elapsed_ms / 1e3),
+        "unit": "tokens/s",
+        "n_gpus": dist.world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": elapsed_ms / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded normal inputs, random-init weights of the layer's shape)",
+        "config": {"workload": f"{cfg.name}: DeepSeek-V3-shaped MoE layer, H={cfg.hidden}, E={cfg.n_experts} routed + "
+                               f"{cfg.n_shared} shared, I={cfg.inter}, top-{cfg.top_k}, grouped sigmoid gating "
+                               f"({cfg.n_groups} groups, top-{cfg.topk_groups}), {len(mbs)} micro-batches x "
+                               f"{mbs[0]} tokens, one CUDA stream each",
+                   "tokens_per_step": tokens_per_step, "microbatches": mbs,
+                   "parallelism": f"replicas x{dist.world} (no data-path collective)",
+                   "l2": "inputs larger than L2: 22.6 GB of expert weights streamed every step"},
+        "gpu_launches": launches_per_mb * len(mbs) * args.steps,
+        "clocks": clk,
+    }
+
+    # ---------------- per-kernel timings, each on the stream it runs on
+    kern = kernel_pass(args, h, cfg, xs, dev)
+    peaks, peaks_src = load_peaks()
+    result["kernels"] = kern["table"]
+    result["roofline"] = roofline(kern, peaks, peaks_src)
+    gemm_flops = kern["gemm_flops"]
+    gemm_ms = kern["gemm_ms"]
+    result["grouped_gemm_tensor_frac"] = {
+        "achieved_tflops": gemm_flops / (gemm_ms / 1e3) / 1e12,
+        "of_burst_measured": gemm_flops / (gemm_ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+        "of_sustained_measured": gemm_flops / (gemm_ms / 1e3) / 1e12 / peaks["bf16_tflops_sustained"],
+        "peaks": peaks_src,
+        "note": "algorithmic FLOPs of both grouped GEMMs (routed + shared) over their event-timed durations"}
+
+    # ---------------- end to end through host buffers
+    result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
+
+    # ---------------- float64 oracle on the host cores
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(cfg, dev, args.cpu_sample_tokens)
+    else:
+        result["cpu_baseline"] = None
+    h.close()
+    return result
+
+
+def kernel_pass(args, h, cfg, xs, dev):
+    """The same work as the timed steps, launched call by call on one stream
+    with CUDA events between the calls, so every kernel's duration is taken on
+    the stream it runs on without overlap from the other micro-batches."""
+    import numpy as np
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    n = max(x.shape[0] for x in xs)
+    k, E, H, I, Is = cfg.top_k, cfg.n_experts, cfg.hidden, cfg.inter, cfg.shared_inter
+    s = torch.cuda.current_stream()
+    logits = torch.empty((n, E), dtype=torch.float32, device=dev)
+    idx = torch.empty((n, k), dtype=torch.int32, device=dev)
+    w = torch.empty((n, k), dtype=torch.float32, device=dev)
+    counts = torch.empty(E, dtype=torch.int32, device=dev)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=dev)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=dev)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=dev)
+    hbuf = torch.empty((n * k, I), dtype=torch.bfloat16, device=dev)
+    hsh = torch.empty((n, Is), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
+    y_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=dev)
+    y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
+    out = torch.empty((n, H), dtype=torch.bfloat16, device=dev)
+    ws = api.workspace(h, n, dev)
+    names = ["router_gemm", "gate_scan", "dispatch", "gemm_gate_up_swiglu", "gemm_down", "combine"]
+    times = {nm: [] for nm in names}
+    active = []   # experts with tokens, per micro-batch (for the weight bytes)
+    for it in range(args.kernel_steps + 1):
+        rec = []
+        for x in xs:
+            m = x.shape[0]
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+            ev[0].record(s)
+            api.asap_moe_router_logits(h, x, logits[:m], stream=s)
+            ev[1].record(s)
+            api.asap_moe_route_logits(h, logits[:m], idx[:m], w[:m], counts, offsets, ws, stream=s)
+            ev[2].record(s)
+            api.asap_moe_dispatch(h, x, idx[:m], x_perm[:m * k], perm_src[:m * k], perm_dst[:m], ws, stream=s)
+            ev[3].record(s)
+            api.asap_moe_expert_gate_up(h, x_perm[:m * k], offsets, x, hbuf[:m * k],
+                                        hsh[:m] if hsh is not None else None, stream=s)
+            ev[4].record(s)
+            api.asap_moe_expert_down(h, hbuf[:m * k], offsets, hsh[:m] if hsh is not None else None, m,
+                                     y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s)
+            ev[5].record(s)
+            api.asap_moe_combine(h, y_perm[:m * k], y_sh[:m] if y_sh is not None else None, w[:m], perm_dst[:m],
+                                 out[:m], stream=s)
+            ev[6].record(s)
+            rec.append(ev)
+            if it == 0:
+                torch.cuda.synchronize()
+                active.append(int((counts > 0).sum().item()))
+        torch.cuda.synchronize()
+        if it == 0:
+            continue   # warm-up round
+        for ev in rec:
+            for j, nm in enumerate(names):
+                times[nm].append(ev[j].elapsed_time(ev[j + 1]))
+    avg = {nm: sum(v) / len(v) for nm, v in times.items()}
+    m = xs[0].shape[0]
+    nk = m * k
+    mean_active = sum(active) / len(active)
+    # algorithmic bytes / FLOPs per launch (one micro-batch of m tokens)
+    wb = 2  # bf16
+    alg = {
+        "router_gemm": dict(bytes=m * H * wb + E * H * wb + m * E * 4, flops=2.0 * m * H * E),
+        "gate_scan": dict(bytes=m * E * 4 + nk * 8, flops=0.0),
+        "dispatch": dict(bytes=m * H * wb + nk * H * wb + nk * 12, flops=0.0),
+        "gemm_gate_up_swiglu": dict(
+            bytes=mean_active * 2 * I * H * wb + (2 * Is * H * wb if cfg.n_shared else 0)
+            + nk * H * wb + (m * H * wb if cfg.n_shared else 0) + nk * I * wb + (m * Is * wb if cfg.n_shared else 0),
+            flops=2.0 * nk * H * 2 * I + (2.0 * m * H * 2 * Is if cfg.n_shared else 0.0)),
+        "gemm_down": dict(
+            bytes=mean_active * H * I * wb + (H * Is * wb if cfg.n_shared else 0)
+            + nk * I * wb + (m * Is * wb if cfg.n_shared else 0) + nk * H * wb + (m * H * wb if cfg.n_shared else 0),
+            flops=2.0 * nk * I * H + (2.0 * m * Is * H if cfg.n_shared else 0.0)),
+        "combine": dict(bytes=nk * H * wb + (m * H * wb if cfg.n_shared else 0) + m * H * wb + nk * 8, flops=0.0),
+    }
+    table = {}
+    for nm in names:
+        sec = avg[nm] / 1e3
+        table[nm] = {"ms": avg[nm], "alg_bytes": alg[nm]["bytes"], "alg_flops": alg[nm]["flops"],
+                     "gbs": alg[nm]["bytes"] / sec / 1e9, "tflops": alg[nm]["flops"] / sec / 1e12}
+    total_ms = sum(avg.values())
+    for nm in names:
+        table[nm]["share"] = avg[nm] / total_ms
+    gemm_flops = alg["gemm_gate_up_swiglu"]["flops"] + alg["gemm_down"]["flops"]
+    gemm_ms = avg["gemm_gate_up_swiglu"] + avg["gemm_down"]
+    return {"table": table, "avg": avg, "alg": alg, "gemm_flops": gemm_flops, "gemm_ms": gemm_ms,
+            "active_experts": mean_active, "serial_ms_per_microbatch": total_ms}
+
+
+def roofline(kern, peaks, peaks_src):
+    nm = max(kern["avg"], key=kern["avg"].get)
+    a = kern["alg"][nm]
+    sec = kern["avg"][nm] / 1e3
+    t_hbm = a["bytes"] / (peaks["hbm_gbs"] * 1e9)
+    t_tc = a["flops"] / (peaks["bf16_tflops_sustained"] * 1e12) if a["flops"] else 0.0
+    traffic, src = profile_traffic("gemm_gate_up_swiglu_dsv3.md", GEMM_SOURCES) if nm.startswith("gemm") else (None, None)
+    if t_tc >= t_hbm:
+        achieved = a["flops"] / sec / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        r = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak}
+    else:
+        achieved = a["bytes"] / sec / 1e9
+        peak = peaks["hbm_gbs"]
+        r = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak}
+    r.update({"traffic": traffic, "kernel": nm, "alg_bytes_per_launch": a["bytes"],
+              "alg_flops_per_launch": a["flops"], "avg_launch_ms": kern["avg"][nm],
+              "peak_source": f"{peaks_src} ({'sustained bf16 tensor' if r['bound'] == 'tensor' else 'HBM copy'})",
+              "hbm_frac_of_measured": a["bytes"] / sec / 1e9 / peaks["hbm_gbs"],
+              "tensor_frac_of_sustained_measured": (a["flops"] / sec / 1e12 / peaks["bf16_tflops_sustained"])
+              if a["flops"] else None,
+              "traffic_source": src})
+    return r
+
+
+def e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist):
+    """tokens/s through asap_moe_layer with the inputs in pinned host memory:
+    every step copies each micro-batch host->device on its stream, runs the
+    layer and copies the output back."""
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    hx = [x.cpu().pin_memory() for x in xs]
+    ho = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    dx = [torch.empty_like(x) for x in xs]
+
+    def step():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for i, s in enumerate(streams):
+            s.wait_event(ev)
+            with torch.cuda.stream(s):
+                dx[i].copy_(hx[i], non_blocking=True)
+            api.asap_moe_layer(h, dx[i], outs[i], wss[i], stream=s)
+            with torch.cuda.stream(s):
+                ho[i].copy_(outs[i], non_blocking=True)
+        for s in streams:
+            main.wait_stream(s)
+
+    steps = max(3, args.steps // 2)
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(main)
+    for _ in range(steps):
+        step()
+    b.record(main)
+    torch.cuda.synchronize()
+    ms = dist.max(a.elapsed_time(b))
+    tokens = sum(x.shape[0] for x in xs)
+    return {"value": dist.world * tokens * steps / (ms / 1e3), "unit": "tokens/s",
+            "h2d_bytes_per_step": sum(x.numel() * x.element_size() for x in hx),
+            "d2h_bytes_per_step": sum(o.numel() * o.element_size() for o in ho), "steps": steps}
+
+
+# ------------------------------------------------------------ reference arm (the oracle)
+
+def run_reference(args, dist):
+    import torch
+    from paper_2606_22541_gb300 import inputs
+    from paper_2606_22541_gb300.configs import CONFIGS
+
+    cfg = CONFIGS[args.workload]
+    dev = f"cuda:{dist.local_rank}" if torch.cuda.is_available() else "cpu"
+    per_step = 1
+    x = inputs.make_tokens(cfg, (args.warmup + args.steps) * per_step, 0, dev)
+    for i in range(args.warmup):
+        oracle_tokens(cfg, x[i:i + 1], dev)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        j = args.warmup + i
+        oracle_tokens(cfg, x[j:j + 1], dev)
+    dt = time.perf_counter() - t0
+    value = args.steps * per_step / dt
+    sample = (f"{per_step} token per step of micro-batch 0 (float64 routing over all experts, its "
+              f"{cfg.top_k} routed experts and the shared expert, weights decoded from bf16 per expert)")
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": dist.world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded normal inputs, random-init weights of the layer's shape)",
+            "config": {"workload": cfg.name, "tokens_per_step": per_step},
+            "cpu_baseline": {"kind": "oracle", "cores": host_cores(), "sample": sample, "value": value,
+                             "unit": "tokens/s"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    dist = Dist()
+    if args.impl == "reference":
+        if dist.rank == 0:
+            print(json.dumps(run_reference(args, dist)), flush=True)
+        dist.close()
+        return
+    res = run_ours(args, dist)
+    if dist.rank == 0:
+        print(json.dumps(res), flush=True)
+    dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -197,6 +197,20 @@ int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_sc
                         const int32_t* offsets, const void* x, int32_t n, void* y_perm,
                         void* y_shared, void* ws, size_t ws_bytes, void* stream);
 
+/* The two halves of asap_moe_expert_ffn, for callers that keep the
+ * intermediate activations or time the GEMMs separately (same kernels, same
+ * bits):
+ *   gate_up: h_perm [n*k, I] = silu(X_e Wg_e^T) * (X_e Wu_e^T) per segment,
+ *            h_shared [n, I_s] likewise for the shared expert on x;
+ *   down   : y_perm = h_perm Wd_e^T per segment, y_shared = h_shared Ws_d^T.
+ * No workspace.  *_scales are reserved for the FP8 configuration (NULL). */
+int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
+                            const int32_t* offsets, const void* x, int32_t n, void* h_perm,
+                            void* h_shared, void* stream);
+int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float* h_perm_scales,
+                         const int32_t* offsets, const void* h_shared, int32_t n, void* y_perm,
+                         void* y_shared, void* stream);
+
 /* Combine (Section 3.2.2): out[t] = sum_{j<k} w[t,j] y_perm[perm_dst[t*k+j]]
  * (+ y_shared[t]), fp32 in slot order then the shared row, rounded to bf16.
  * y_shared may be NULL. */

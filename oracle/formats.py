@@ -15,8 +15,8 @@ be pinned against an independent library conversion.
 import numpy as np
 
 
-def bf16_bits_to_f64(bits):
-    """bfloat16 bit patterns (uint16) -> float64, exactly.
+def _bf16_fields_to_f64(bits):
+    """bfloat16 bit patterns (uint16) -> float64, exactly, from the fields.
 
     Layout: 1 sign bit, 8 exponent bits (bias 127), 7 fraction bits.
     exponent 0      : subnormal, value = (-1)^s * 2^-126 * f/128
@@ -32,6 +32,18 @@ def bf16_bits_to_f64(bits):
     mag = np.where(e == 0, sub, normal)
     mag = np.where(e == 255, np.where(f == 0, np.inf, np.nan), mag)
     return sign * mag
+
+
+_BF16_TABLE = None
+
+
+def bf16_bits_to_f64(bits):
+    """bfloat16 bit patterns (uint16) -> float64, exactly: a lookup in the
+    table of all 65536 patterns decoded by ``_bf16_fields_to_f64``."""
+    global _BF16_TABLE
+    if _BF16_TABLE is None:
+        _BF16_TABLE = _bf16_fields_to_f64(np.arange(65536, dtype=np.uint32).astype(np.uint16))
+    return _BF16_TABLE[np.asarray(bits, dtype=np.uint16)]
 
 
 def e4m3_bits_to_f64(bits):

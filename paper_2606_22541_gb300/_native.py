@@ -47,6 +47,8 @@ SIGNATURES = {
     "asap_moe_route_logits": [_P, _P, _I, _P, _P, _P, _P, _P, _SZ, _P],
     "asap_moe_dispatch": [_P, _P, _I, _P, _P, _P, _P, _P, _P, _SZ, _P],
     "asap_moe_expert_ffn": [_P, _P, _P, _P, _P, _I, _P, _P, _P, _SZ, _P],
+    "asap_moe_expert_gate_up": [_P, _P, _P, _P, _P, _I, _P, _P, _P],
+    "asap_moe_expert_down": [_P, _P, _P, _P, _P, _I, _P, _P, _P],
     "asap_moe_combine": [_P, _P, _P, _P, _P, _I, _P, _P],
     "asap_moe_layer": [_P, _P, _I, _P, _P, _SZ, _P],
     "asap_moe_status": [_P, ctypes.POINTER(ctypes.c_uint32)],

@@ -161,86 +161,102 @@ int run_gate_scan(asap_moe_t h, const float* logits, int n, int32_t* idx, float*
   return ASAP_OK;
 }
 
-int run_expert_ffn(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n,
-                   void* y_perm, void* y_sh, void* hbuf, void* hsh, cudaStream_t st) {
+int ub_mtiles(const asap_moe_config& c, long long nk) {
+  return asap::ceil_div(nk, asap::kGemmBM) + static_cast<int>(std::min<long long>(c.n_experts, nk));
+}
+
+// GEMM1: h = silu(X Wg^T) * (X Wu^T) on the routed segments, plus the shared
+// expert on x (problem 1 of the same launch).
+int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n, void* hbuf,
+                void* hsh, cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
-  std::string err;
   const bool sh = c.n_shared != 0;
-  const int ub_mtiles = asap::ceil_div(nk, asap::kGemmBM) + static_cast<int>(std::min<long long>(c.n_experts, nk));
-  // GEMM1: h = silu(X Wg^T) * (X Wu^T), routed segments + shared expert on x
-  {
-    CUtensorMap maps[4];
-    if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
-      return fail(ASAP_ERR_INVALID, "x_perm: " + err);
-    maps[1] = h->tm_gate_up;
-    if (sh) {
-      if (!asap::encode_tmap_bf16(&maps[2], x, n, c.hidden, asap::kGemmBM, &err))
-        return fail(ASAP_ERR_INVALID, "x: " + err);
-      maps[3] = h->tm_sh_gate_up;
-    } else {
-      maps[2] = maps[0];
-      maps[3] = maps[1];
-    }
-    asap::GemmArgs a{};
-    a.offsets = offsets;
-    a.groups = c.n_experts;
-    a.m0 = static_cast<int>(nk);
-    a.b_stride0 = 2 * c.inter;
-    a.n_tiles0 = c.inter / 128;
-    a.k_iters0 = c.hidden / asap::kGemmBK;
-    a.out0 = hbuf;
-    a.ldo0 = c.inter;
-    a.m1 = sh ? n : 0;
-    a.n_tiles1 = sh ? c.shared_inter / 128 : 0;
-    a.k_iters1 = c.hidden / asap::kGemmBK;
-    a.out1 = hsh;
-    a.ldo1 = c.shared_inter;
-    a.status = h->status;
-    a.hint_a = 2;
-    a.hint_b = 1;
-    const long long tiles = static_cast<long long>(ub_mtiles) * a.n_tiles0 +
-                            (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
-    CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
-           "gate/up GEMM launch");
+  std::string err;
+  CUtensorMap maps[4];
+  if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
+    return fail(ASAP_ERR_INVALID, "x_perm: " + err);
+  maps[1] = h->tm_gate_up;
+  if (sh) {
+    if (!asap::encode_tmap_bf16(&maps[2], x, n, c.hidden, asap::kGemmBM, &err))
+      return fail(ASAP_ERR_INVALID, "x: " + err);
+    maps[3] = h->tm_sh_gate_up;
+  } else {
+    maps[2] = maps[0];
+    maps[3] = maps[1];
   }
-  // GEMM2: y = h Wd^T
-  {
-    CUtensorMap maps[4];
-    if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
-      return fail(ASAP_ERR_INVALID, "h: " + err);
-    maps[1] = h->tm_down;
-    if (sh) {
-      if (!asap::encode_tmap_bf16(&maps[2], hsh, n, c.shared_inter, asap::kGemmBM, &err))
-        return fail(ASAP_ERR_INVALID, "h_shared: " + err);
-      maps[3] = h->tm_sh_down;
-    } else {
-      maps[2] = maps[0];
-      maps[3] = maps[1];
-    }
-    asap::GemmArgs a{};
-    a.offsets = offsets;
-    a.groups = c.n_experts;
-    a.m0 = static_cast<int>(nk);
-    a.b_stride0 = c.hidden;
-    a.n_tiles0 = c.hidden / asap::kGemmBN;
-    a.k_iters0 = c.inter / asap::kGemmBK;
-    a.out0 = y_perm;
-    a.ldo0 = c.hidden;
-    a.m1 = sh ? n : 0;
-    a.n_tiles1 = sh ? c.hidden / asap::kGemmBN : 0;
-    a.k_iters1 = sh ? c.shared_inter / asap::kGemmBK : 0;
-    a.out1 = y_sh;
-    a.ldo1 = c.hidden;
-    a.status = h->status;
-    a.hint_a = 2;
-    a.hint_b = 1;
-    const long long tiles = static_cast<long long>(ub_mtiles) * a.n_tiles0 +
-                            (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
-    CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
-           "down GEMM launch");
-  }
+  asap::GemmArgs a{};
+  a.offsets = offsets;
+  a.groups = c.n_experts;
+  a.m0 = static_cast<int>(nk);
+  a.b_stride0 = 2 * c.inter;
+  a.n_tiles0 = c.inter / 128;
+  a.k_iters0 = c.hidden / asap::kGemmBK;
+  a.out0 = hbuf;
+  a.ldo0 = c.inter;
+  a.m1 = sh ? n : 0;
+  a.n_tiles1 = sh ? c.shared_inter / 128 : 0;
+  a.k_iters1 = c.hidden / asap::kGemmBK;
+  a.out1 = hsh;
+  a.ldo1 = c.shared_inter;
+  a.status = h->status;
+  a.hint_a = 2;
+  a.hint_b = 1;
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
+  CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+         "gate/up GEMM launch");
   return ASAP_OK;
+}
+
+// GEMM2: y = h Wd^T on the routed segments, plus the shared expert.
+int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void* hsh, int n, void* y_perm,
+             void* y_sh, cudaStream_t st) {
+  const asap_moe_config& c = h->cfg;
+  const long long nk = static_cast<long long>(n) * c.top_k;
+  const bool sh = c.n_shared != 0;
+  std::string err;
+  CUtensorMap maps[4];
+  if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
+    return fail(ASAP_ERR_INVALID, "h: " + err);
+  maps[1] = h->tm_down;
+  if (sh) {
+    if (!asap::encode_tmap_bf16(&maps[2], hsh, n, c.shared_inter, asap::kGemmBM, &err))
+      return fail(ASAP_ERR_INVALID, "h_shared: " + err);
+    maps[3] = h->tm_sh_down;
+  } else {
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+  }
+  asap::GemmArgs a{};
+  a.offsets = offsets;
+  a.groups = c.n_experts;
+  a.m0 = static_cast<int>(nk);
+  a.b_stride0 = c.hidden;
+  a.n_tiles0 = c.hidden / asap::kGemmBN;
+  a.k_iters0 = c.inter / asap::kGemmBK;
+  a.out0 = y_perm;
+  a.ldo0 = c.hidden;
+  a.m1 = sh ? n : 0;
+  a.n_tiles1 = sh ? c.hidden / asap::kGemmBN : 0;
+  a.k_iters1 = sh ? c.shared_inter / asap::kGemmBK : 0;
+  a.out1 = y_sh;
+  a.ldo1 = c.hidden;
+  a.status = h->status;
+  a.hint_a = 2;
+  a.hint_b = 1;
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
+  CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+         "down GEMM launch");
+  return ASAP_OK;
+}
+
+int run_expert_ffn(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n,
+                   void* y_perm, void* y_sh, void* hbuf, void* hsh, cudaStream_t st) {
+  int r = run_gate_up(h, x_perm, offsets, x, n, hbuf, hsh, st);
+  if (r != ASAP_OK) return r;
+  return run_down(h, hbuf, offsets, hsh, n, y_perm, y_sh, st);
 }
 
 }  // namespace
@@ -453,6 +469,32 @@ ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* 
   const Layout L = layout(h->cfg, n);
   return run_expert_ffn(h, x_perm, offsets, x, n, y_perm, y_shared, at<void>(ws, L.h), at<void>(ws, L.h_sh),
                         S(stream));
+}
+
+ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
+                                     const int32_t* offsets, const void* x, int32_t n, void* h_perm,
+                                     void* h_shared, void* stream) {
+  (void)x_perm_scales;
+  int r = check_call(h, n, nullptr, 0, false);
+  if (r != ASAP_OK || n == 0) return r;
+  if (!x_perm || !offsets || !h_perm || !aligned16(x_perm) || !aligned16(h_perm))
+    return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+  if (h->cfg.n_shared && (!x || !h_shared || !aligned16(x) || !aligned16(h_shared)))
+    return fail(ASAP_ERR_INVALID, "x and h_shared are required for the shared expert");
+  return run_gate_up(h, x_perm, offsets, x, n, h_perm, h_shared, S(stream));
+}
+
+ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float* h_perm_scales,
+                                  const int32_t* offsets, const void* h_shared, int32_t n, void* y_perm,
+                                  void* y_shared, void* stream) {
+  (void)h_perm_scales;
+  int r = check_call(h, n, nullptr, 0, false);
+  if (r != ASAP_OK || n == 0) return r;
+  if (!h_perm || !offsets || !y_perm || !aligned16(h_perm) || !aligned16(y_perm))
+    return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+  if (h->cfg.n_shared && (!h_shared || !y_shared || !aligned16(h_shared) || !aligned16(y_shared)))
+    return fail(ASAP_ERR_INVALID, "h_shared and y_shared are required for the shared expert");
+  return run_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, S(stream));
 }
 
 ASAP_API int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared, const float* w,

@@ -85,12 +85,7 @@ def make_weights(cfg, device):
     """Router, routed-expert and shared-expert weights of one layer."""
     H, E, I, Is = cfg.hidden, cfg.n_experts, cfg.inter, cfg.shared_inter
     base = cfg.seed * 1000
-    r_std = 0.02 if cfg.name == "tiny" else 1.0 / np.sqrt(H)
-    wr = randn_bf16((E, H), r_std, base + 1, device)
-    if cfg.zipf_s is not None:
-        b = torch.tensor(zipf_logit_bias(E, cfg.zipf_s, cfg.seed), dtype=torch.float32, device=device)
-        wr[:, 0] = b.to(torch.bfloat16)
-    w = dict(router_w=wr, router_bias=None)
+    w = dict(router_w=router_weights_bf16(cfg, device), router_bias=None)
     if cfg.dtype == "bf16":
         w["w_gate"] = expert_stack_bf16(E, I, H, 1 / np.sqrt(H), base + 2, device)
         w["w_up"] = expert_stack_bf16(E, I, H, 1 / np.sqrt(H), base + 3, device)
@@ -110,6 +105,35 @@ def make_weights(cfg, device):
             w.update(sh_gate=sg[0], sh_s_gate=ssg[0], sh_up=su[0], sh_s_up=ssu[0],
                      sh_down=sd[0], sh_s_down=ssd[0])
     return w
+
+
+def expert_weights_bf16(cfg, e, device):
+    """(Wg_e [I, H], Wu_e [I, H], Wd_e [H, I]) of one routed expert, the same
+    values make_weights draws for it (bf16 configurations)."""
+    H, I = cfg.hidden, cfg.inter
+    base = cfg.seed * 1000
+    return (randn_bf16((I, H), 1 / np.sqrt(H), (base + 2) * 1000 + e, device),
+            randn_bf16((I, H), 1 / np.sqrt(H), (base + 3) * 1000 + e, device),
+            randn_bf16((H, I), 1 / np.sqrt(I), (base + 4) * 1000 + e, device))
+
+
+def router_weights_bf16(cfg, device):
+    """The router weights make_weights draws (bf16 configurations)."""
+    H, E = cfg.hidden, cfg.n_experts
+    r_std = 0.02 if cfg.name == "tiny" else 1.0 / np.sqrt(H)
+    wr = randn_bf16((E, H), r_std, cfg.seed * 1000 + 1, device)
+    if cfg.zipf_s is not None:
+        b = torch.tensor(zipf_logit_bias(E, cfg.zipf_s, cfg.seed), dtype=torch.float32, device=device)
+        wr[:, 0] = b.to(torch.bfloat16)
+    return wr
+
+
+def shared_weights_bf16(cfg, device):
+    H, Is = cfg.hidden, cfg.shared_inter
+    base = cfg.seed * 1000
+    return (randn_bf16((Is, H), 1 / np.sqrt(H), base + 5, device),
+            randn_bf16((Is, H), 1 / np.sqrt(H), base + 6, device),
+            randn_bf16((H, Is), 1 / np.sqrt(Is), base + 7, device))
 
 
 def make_tokens(cfg, n, mb_index, device):
