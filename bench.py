@@ -47,7 +47,9 @@ def parse_args():
     ap.add_argument("--workload", default="dsv3_bf16")
     ap.add_argument("--kernel-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample-tokens", type=int, default=2)
+    ap.add_argument("--cpu-sample-tokens", type=int, default=6)
+    ap.add_argument("--microbatches", default=None,
+                    help="comma-separated micro-batch sizes overriding the workload's")
     return ap.parse_args()
 
 
@@ -151,44 +153,55 @@ def host_cores():
         return os.cpu_count() or 1
 
 
-def oracle_tokens(cfg, x_tokens, device):
-    """Run the float64 oracle on a few tokens of the workload: routing over all
-    experts, then each token's 8 routed experts and the shared expert, with
-    every weight matrix decoded from bf16 by the oracle as it reads it.
-    Returns the outputs (float64)."""
+def oracle_inputs(cfg, x_tokens, device):
+    """Raw bf16 bit patterns (host numpy) of everything the oracle reads for
+    a few tokens: the tokens, the router, the shared expert and the routed
+    experts those tokens select (found by a first, untimed oracle routing)."""
     import numpy as np
     import torch
     import oracle
     from paper_2606_22541_gb300 import inputs
 
-    def f64(t):
-        return oracle.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16))
+    def bits(t):
+        return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
-    xf = f64(x_tokens)
-    wr = f64(inputs.router_weights_bf16(cfg, device))
-    L = oracle.router_logits(xf, wr)
+    xb = bits(x_tokens)
+    wrb = bits(inputs.router_weights_bf16(cfg, device))
+    idx, _ = oracle.route(oracle.router_logits(oracle.bf16_bits_to_f64(xb), oracle.bf16_bits_to_f64(wrb)),
+                          cfg.oracle_cfg())
+    experts = {int(e): tuple(bits(t) for t in inputs.expert_weights_bf16(cfg, int(e), device))
+               for e in np.unique(idx)}
+    shared = tuple(bits(t) for t in inputs.shared_weights_bf16(cfg, device)) if cfg.n_shared else None
+    return dict(x=xb, router=wrb, experts=experts, shared=shared)
+
+
+def oracle_run(cfg, inp):
+    """The float64 oracle on prepared inputs: bf16 decode, routing over all
+    experts, each token's routed experts (decoded one at a time) and the
+    shared expert."""
+    import oracle
+    f64 = oracle.bf16_bits_to_f64
+    xf = f64(inp["x"])
+    L = oracle.router_logits(xf, f64(inp["router"]))
     idx, w = oracle.route(L, cfg.oracle_cfg())
-    shared = tuple(f64(t) for t in inputs.shared_weights_bf16(cfg, device)) if cfg.n_shared else None
-
-    def expert(e, which):
-        return f64(inputs.expert_weights_bf16(cfg, e, device)[which])
-
-    # per-expert callables decode on demand, as the oracle's layer functions allow
-    return oracle.moe_layer_tokens(xf, idx, w, lambda e: expert(e, 0), lambda e: expert(e, 1),
-                                   lambda e: expert(e, 2), shared)
+    shared = tuple(f64(b) for b in inp["shared"]) if inp["shared"] is not None else None
+    ex = inp["experts"]
+    return oracle.moe_layer_tokens(xf, idx, w, lambda e: f64(ex[e][0]), lambda e: f64(ex[e][1]),
+                                   lambda e: f64(ex[e][2]), shared)
 
 
 def cpu_baseline(cfg, device, n_tokens):
     from paper_2606_22541_gb300 import inputs
     x = inputs.make_tokens(cfg, n_tokens, 0, device)
+    inp = oracle_inputs(cfg, x, device)
     t0 = time.perf_counter()
-    oracle_tokens(cfg, x, device)
+    oracle_run(cfg, inp)
     dt = time.perf_counter() - t0
     return {"value": n_tokens / dt, "unit": "tokens/s", "cores": host_cores(), "kind": "oracle",
             "sample": f"{n_tokens} tokens of micro-batch 0: float64 routing over all {cfg.n_experts} experts, "
-                      f"then each token's {cfg.top_k} routed experts and the shared expert with weights decoded "
-                      f"from bf16 per expert ({dt:.1f} s); numpy elementwise work on one thread, BLAS on up to "
-                      f"{host_cores()} threads"}
+                      f"then each token's {cfg.top_k} routed experts and the shared expert, weights decoded "
+                      f"from bf16 as the oracle reads them ({dt:.1f} s); numpy elementwise work on one thread, "
+                      f"BLAS on up to {host_cores()} threads"}
 
 
 # ------------------------------------------------------------ roofline evidence
@@ -219,6 +232,10 @@ def sources_sha256(files):
 GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb300/csrc/common.cuh"]
 
 
+def weight_gb(cfg):
+    return (cfg.n_experts * 3 * cfg.hidden * cfg.inter + cfg.n_shared * 3 * cfg.hidden * cfg.shared_inter) * 2 / 1e9
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -239,6 +256,9 @@ def run_ours(args, dist):
     from paper_2606_22541_gb300.configs import CONFIGS
 
     cfg = CONFIGS[args.workload]
+    if args.microbatches:
+        from paper_2606_22541_gb300.inputs import small_variant
+        cfg = small_variant(cfg, microbatches=[int(v) for v in args.microbatches.split(",")])
     torch.cuda.set_device(dist.local_rank)
     dev = f"cuda:{dist.local_rank}"
     mbs = cfg.microbatches
@@ -283,7 +303,7 @@ def run_ours(args, dist):
     code, word = api.asap_moe_status(h)
     if code != 0:
         raise RuntimeError(f"device status word {word:#x} after the timed region")
-    launches_per_mb = 7   # router GEMM, gate, scan, dispatch, gate/up GEMM, down GEMM, combine
+    launches_per_mb = 7   # router, gate, scan, dispatch, gate/up GEMM, down GEMM, combine
     result = {
         "metric": METRIC,
         "value": dist.world * tokens_per_step * args.steps / (elapsed_ms / 1e3),
@@ -297,13 +317,13 @@ def run_ours(args, dist):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded normal inputs, random-init weights of the layer's shape)",
-        "config": {"workload": f"{cfg.name}: DeepSeek-V3-shaped MoE layer, H={cfg.hidden}, E={cfg.n_experts} routed + "
-                               f"{cfg.n_shared} shared, I={cfg.inter}, top-{cfg.top_k}, grouped sigmoid gating "
-                               f"({cfg.n_groups} groups, top-{cfg.topk_groups}), {len(mbs)} micro-batches x "
-                               f"{mbs[0]} tokens, one CUDA stream each",
+        "config": {"workload": f"{cfg.name}: MoE layer, H={cfg.hidden}, E={cfg.n_experts} routed + "
+                               f"{cfg.n_shared} shared, I={cfg.inter}, top-{cfg.top_k}, {cfg.gating} gating"
+                               + (f" ({cfg.n_groups} groups, top-{cfg.topk_groups})" if cfg.n_groups > 1 else "")
+                               + f", {len(mbs)} micro-batches ({','.join(map(str, mbs))} tokens), one CUDA stream each",
                    "tokens_per_step": tokens_per_step, "microbatches": mbs,
                    "parallelism": f"replicas x{dist.world} (no data-path collective)",
-                   "l2": "inputs larger than L2: 22.6 GB of expert weights streamed every step"},
+                   "l2": f"inputs larger than L2: {weight_gb(cfg):.1f} GB of expert weights streamed every step"},
         "gpu_launches": launches_per_mb * len(mbs) * args.steps,
         "clocks": clk,
     }
@@ -506,13 +526,13 @@ def run_reference(args, dist):
     dev = f"cuda:{dist.local_rank}" if torch.cuda.is_available() else "cpu"
     per_step = 1
     x = inputs.make_tokens(cfg, (args.warmup + args.steps) * per_step, 0, dev)
-    for i in range(args.warmup):
-        oracle_tokens(cfg, x[i:i + 1], dev)
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        j = args.warmup + i
-        oracle_tokens(cfg, x[j:j + 1], dev)
-    dt = time.perf_counter() - t0
+    dt = 0.0
+    for i in range(args.warmup + args.steps):
+        inp = oracle_inputs(cfg, x[i * per_step:(i + 1) * per_step], dev)   # input preparation, untimed
+        t0 = time.perf_counter()
+        oracle_run(cfg, inp)
+        if i >= args.warmup:
+            dt += time.perf_counter() - t0
     value = args.steps * per_step / dt
     sample = (f"{per_step} token per step of micro-batch 0 (float64 routing over all experts, its "
               f"{cfg.top_k} routed experts and the shared expert, weights decoded from bf16 per expert)")

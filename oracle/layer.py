@@ -89,7 +89,7 @@ def expert_ffn(x_perm, offsets, wg, wu, wd):
     large weight sets can be decoded one expert at a time)."""
     x_perm = np.asarray(x_perm, np.float64)
     E = len(offsets) - 1
-    y = np.zeros((x_perm.shape[0], _dim(wd, 1)), np.float64)
+    y = np.zeros_like(x_perm)   # an expert maps H channels back to H
     for e in range(E):
         a, b = offsets[e], offsets[e + 1]
         if b > a:
@@ -112,11 +112,6 @@ def combine(y_perm, w, perm_dst, y_shared=None):
 
 def _get(wset, e):
     return wset(e) if callable(wset) else wset[e]
-
-
-def _dim(wset, axis):
-    m = _get(wset, 0)
-    return m.shape[axis - 1] if m.ndim == 2 else m.shape[axis]
 
 
 def moe_layer(x, router_w, wg, wu, wd, cfg, shared=None, router_bias=None):
@@ -148,7 +143,7 @@ def moe_layer_tokens(x_tok, idx, w, wg, wu, wd, shared=None):
     x_tok: [m, H]; idx, w: [m, k]."""
     x_tok = np.asarray(x_tok, np.float64)
     m, k = np.asarray(idx).shape
-    out = np.zeros((m, _dim(wd, 1)), np.float64)
+    out = np.zeros_like(x_tok)
     for t in range(m):
         for j in range(k):
             e = int(idx[t, j])
@@ -208,7 +203,7 @@ def moe_layer_tokens_fp8(x_tok, idx, w, wg, wu, wd, shared=None, block=128):
     matrices (or per-expert callables returning them)."""
     x_tok = np.asarray(x_tok, np.float64)
     m, k = np.asarray(idx).shape
-    out = np.zeros((m, _dim(wd, 1)), np.float64)
+    out = np.zeros_like(x_tok)
     for t in range(m):
         for j in range(k):
             e = int(idx[t, j])

@@ -80,4 +80,11 @@ DSV3_FP8 = LayerConfig("dsv3_fp8", hidden=7168, n_experts=256, top_k=8, inter=20
                        route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[4096] * 8,
                        zipf_s=1.1, seed=1004)
 
-CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8)}
+# Profiling case of the DeepSeek-V3 layer's grouped GEMMs: the same per-expert
+# shape (M_e ~ 128 rows, K = 7168, N = 2 x 2048) with 32 experts, so one
+# launch's weights (2.8 GB) exceed L2 while the device holds a few GB.
+DSV3_E32 = LayerConfig("dsv3_e32_profile", hidden=7168, n_experts=32, top_k=8, inter=2048, n_shared=1,
+                       shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                       route_scale=2.5, microbatches=[512], seed=1002)
+
+CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32)}
