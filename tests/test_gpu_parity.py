@@ -386,3 +386,41 @@ def test_bad_indices_are_reported_not_trapped():
     assert perm_dst[3, 0].item() == -1
     code, word = api.asap_moe_status(c.h)                   # cleared by the read
     assert code == 0 and word == 0
+
+
+@pytest.mark.parametrize("cfg", [MX_SMALL, DS_SMALL], ids=lambda c: c.name)
+def test_ffn_halves_equal_expert_ffn_and_h_matches_oracle(cfg):
+    """gate_up then down give the same bits as expert_ffn; the intermediate h
+    matches silu(X Wg^T) * (X Wu^T) of the oracle."""
+    c = Case.get(cfg)
+    n, k, H, I = max(cfg.microbatches), cfg.top_k, cfg.hidden, cfg.inter
+    x = c.tokens(0, n)
+    idx, w, counts, offsets = run_route(c, x)
+    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    perm_src = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    perm_dst = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    ws = c.ws(n)
+    api.asap_moe_dispatch(c.h, x, idx, x_perm, perm_src, perm_dst, ws)
+    y1 = torch.empty_like(x_perm)
+    ysh1 = torch.empty((n, H), dtype=torch.bfloat16, device=DEV) if cfg.n_shared else None
+    api.asap_moe_expert_ffn(c.h, x_perm, offsets, x, y1, ysh1, ws)
+    hb = torch.empty((n * k, I), dtype=torch.bfloat16, device=DEV)
+    hsh = torch.empty((n, cfg.shared_inter), dtype=torch.bfloat16, device=DEV) if cfg.n_shared else None
+    api.asap_moe_expert_gate_up(c.h, x_perm, offsets, x, hb, hsh)
+    y2 = torch.empty_like(x_perm)
+    ysh2 = torch.empty_like(ysh1) if cfg.n_shared else None
+    api.asap_moe_expert_down(c.h, hb, offsets, hsh, n, y2, ysh2)
+    torch.cuda.synchronize()
+    assert torch.equal(y1.view(torch.int16), y2.view(torch.int16))
+    if cfg.n_shared:
+        assert torch.equal(ysh1.view(torch.int16), ysh2.view(torch.int16))
+    off = offsets.cpu().numpy()
+    xp = bf16_to_f64(x_perm)
+    hg = bf16_to_f64(hb)
+    for e in range(cfg.n_experts):
+        a, b = off[e], off[e + 1]
+        if b > a:
+            X = xp[a:b]
+            ref = oracle.silu(X @ c.wf["w_gate"][e].T) * (X @ c.wf["w_up"][e].T)
+            compare_rows(hg[a:b], ref, rel_norm=5e-3)
+    assert_clean(c)
