@@ -224,6 +224,30 @@ int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared,
 int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
                    size_t ws_bytes, void* stream);
 
+/* asap_moe_route without any device allocation (no counterpart in the
+ * paper; this entry point exists for callers that cannot allocate).
+ *
+ * Some callers cannot call cudaMalloc when they route: their device memory is
+ * owned entirely by another allocator (for example a serving framework's pool
+ * that reserved the GPU at start-up), or allocation on that path is forbidden
+ * or would synchronise the device.  This call takes the same inputs and
+ * outputs as asap_moe_route but keeps its scratch (router logits, per-chunk
+ * histograms and chunk bases) in one static device array of the library:
+ * 4096 tokens x 256 experts, 4 MiB + 128 KiB, held by every GPU that loads
+ * libasap_moe until the process exits.  It calls no cudaMalloc, cudaFree or
+ * other allocating routine.
+ *  - n > 4096 (or n > max_tokens) returns ASAP_ERR_INVALID with a message.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call shares the one array, so calls whose work overlaps on the
+ *    GPU (for example on two streams without ordering between them) race and
+ *    may return wrong routing; order them on one stream or with events.
+ *  - The array keeps the last call's contents; every element a call reads is
+ *    written earlier by the same call.                                      */
+int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
+                           int32_t* counts, int32_t* offsets, void* stream);
+
 /* Synchronise the device, return ASAP_OK or ASAP_ERR_DEVICE_STATUS, write the
  * raw status word (0 = clean) to *word if non-NULL, then clear it. */
 int asap_moe_status(asap_moe_t h, uint32_t* word);

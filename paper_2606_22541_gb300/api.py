@@ -148,6 +148,14 @@ def asap_moe_layer(h, x, out, ws, stream=None):
     check("asap_moe_layer", lib().asap_moe_layer(h.ptr, _ptr(x), x.shape[0], _ptr(out), p, n, _stream(stream)))
 
 
+def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
+    """asap_moe_route with its scratch in the library's static device array
+    (at most 4096 tokens; calls overlapping on the GPU race)."""
+    check("asap_moe_route_noalloc",
+          lib().asap_moe_route_noalloc(h.ptr, _ptr(x), x.shape[0], _ptr(idx), _ptr(w), _ptr(counts),
+                                       _ptr(offsets), _stream(stream)))
+
+
 def asap_moe_status(h):
     """(code, raw status word); code is ASAP_OK or ASAP_ERR_DEVICE_STATUS."""
     word = ctypes.c_uint32()

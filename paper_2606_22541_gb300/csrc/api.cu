@@ -7,6 +7,7 @@
 
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 
 #define ASAP_API extern "C" __attribute__((visibility("default")))
@@ -554,5 +555,86 @@ ASAP_API int asap_moe_status(asap_moe_t h, uint32_t* word) {
   if (e != cudaSuccess) return cuda_fail(e, "status read");
   if (word) *word = v;
   if (v != 0) return fail(ASAP_ERR_DEVICE_STATUS, "device status word " + std::to_string(v));
+  return ASAP_OK;
+}
+
+// ============================================================ routing without allocation
+//
+// Some callers cannot allocate device memory when they route a micro-batch:
+// a process whose HBM is owned entirely by another allocator (a serving
+// framework's caching pool that reserved the device at start-up), or code on
+// a path where a cudaMalloc would implicitly synchronise the device or is not
+// permitted at all.  asap_moe_route_noalloc gives them the routing step with
+// its scratch (router logits, per-chunk histograms, chunk bases) in a
+// file-scope device array instead of a caller workspace.  The array is
+// kStaticRouteMaxTokens tokens x 256 experts and is held by every GPU that
+// loads this library until the process exits.
+
+namespace {
+
+constexpr int kStaticRouteMaxTokens = 4096;
+constexpr size_t kStaticLogitsBytes =
+    static_cast<size_t>(kStaticRouteMaxTokens) * ASAP_MOE_MAX_EXPERTS * sizeof(float);   // 4 MiB
+constexpr size_t kStaticChunkBytes = static_cast<size_t>(kStaticRouteMaxTokens / asap::kChunkTokens) *
+                                     ASAP_MOE_MAX_EXPERTS * sizeof(int32_t);                  // 64 KiB
+constexpr size_t kStaticRouteBytes = kStaticLogitsBytes + 2 * kStaticChunkBytes;
+
+constexpr int kStaticMaxDevices = 64;
+std::mutex g_static_route_mu;
+void* g_static_route_ptr[kStaticMaxDevices] = {};
+
+}  // namespace
+
+// Host code must not use this symbol as a device address: it is a host-side
+// stand-in.  The device address comes from cudaGetSymbolAddress below.
+static __device__ __align__(256) unsigned char g_static_route_scratch[kStaticRouteBytes];
+
+namespace {
+
+// Device address of the static scratch on ``device``, looked up once per
+// device with that device current.
+int static_route_scratch(int device, unsigned char** out) {
+  if (device < 0 || device >= kStaticMaxDevices)
+    return fail(ASAP_ERR_UNSUPPORTED, "device ordinal beyond the static routing scratch table");
+  std::lock_guard<std::mutex> lock(g_static_route_mu);
+  if (!g_static_route_ptr[device]) {
+    int prev = 0;
+    cudaError_t e = cudaGetDevice(&prev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (prev != device && (e = cudaSetDevice(device)) != cudaSuccess) return cuda_fail(e, "cudaSetDevice");
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_route_scratch);
+    if (prev != device) cudaSetDevice(prev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the static routing scratch");
+    g_static_route_ptr[device] = p;
+  }
+  *out = static_cast<unsigned char*>(g_static_route_ptr[device]);
+  return ASAP_OK;
+}
+
+}  // namespace
+
+ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
+                                    int32_t* counts, int32_t* offsets, void* stream) {
+  int r = check_call(h, n, nullptr, 0, false);
+  if (r != ASAP_OK || n == 0) return r;
+  if (n > kStaticRouteMaxTokens)
+    return fail(ASAP_ERR_INVALID, "n = " + std::to_string(n) + " exceeds the " +
+                                      std::to_string(kStaticRouteMaxTokens) +
+                                      " tokens the static routing scratch holds; use asap_moe_route");
+  if (!x || !idx || !w || !counts || !offsets || !aligned16(x)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+  unsigned char* scratch = nullptr;
+  if ((r = static_route_scratch(h->device, &scratch)) != ASAP_OK) return r;
+  float* logits = reinterpret_cast<float*>(scratch);
+  int32_t* hist = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes);
+  int32_t* base = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + kStaticChunkBytes);
+  cudaStream_t st = S(stream);
+  // every scratch element read below is written earlier on the same stream
+  // (logits by the router, all E entries of each chunk's histogram by the
+  // gate kernel), so nothing has to be cleared between calls
+  if ((r = run_router_logits(h, x, n, logits, st)) != ASAP_OK) return r;
+  CU_TRY(asap::launch_gate(logits, n, gate_params(h), idx, w, hist, st), "gate launch");
+  CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base, st),
+         "scan launch");
   return ASAP_OK;
 }
