@@ -147,7 +147,9 @@ typedef struct asap_moe_s* asap_moe_t;
 /* Validate cfg, allocate the handle's device memory on the current device,
  * copy and pack the weights (gate/up rows interleaved in blocks of 128 so one
  * 256-wide GEMM tile holds matching gate and up columns) and build the weight
- * TMA descriptors.  Synchronous.  On failure *out is NULL. */
+ * TMA descriptors.  Synchronous: it first synchronises the device, so weights
+ * still being written on any stream are complete before they are read.  On
+ * failure *out is NULL. */
 int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* weights,
                     asap_moe_t* out);
 
@@ -165,7 +167,9 @@ int asap_moe_workspace_size(const asap_moe_config* cfg, int32_t n_tokens, size_t
 int asap_moe_check_config(const asap_moe_config* cfg);
 
 /* Router logits only: logits[n, E] (fp32) = x Wr^T, fp32 accumulation of
- * bf16 products. */
+ * bf16 products.  Needs a workspace: the tensor-core router splits K into
+ * slices and adds them in slice order, exactly as asap_moe_route does, so
+ * asap_moe_route_logits on these logits reproduces asap_moe_route. */
 int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, float* logits,
                            void* ws, size_t ws_bytes, void* stream);
 
@@ -233,7 +237,7 @@ int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
  * or would synchronise the device.  This call takes the same inputs and
  * outputs as asap_moe_route but keeps its scratch (router logits, per-chunk
  * histograms and chunk bases) in one static device array of the library:
- * 4096 tokens x 256 experts, 4 MiB + 128 KiB, held by every GPU that loads
+ * 4096 tokens x 256 experts, 4 MiB + 256 KiB, held by every GPU that loads
  * libasap_moe until the process exits.  It calls no cudaMalloc, cudaFree or
  * other allocating routine.
  *  - n > 4096 (or n > max_tokens) returns ASAP_ERR_INVALID with a message.

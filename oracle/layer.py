@@ -153,6 +153,23 @@ def moe_layer_tokens(x_tok, idx, w, wg, wu, wd, shared=None):
     return out
 
 
+def moe_layer_tokens_by_expert(x_tok, idx, w, get_expert, shared=None):
+    """``moe_layer_tokens`` looping over experts instead of tokens, so a large
+    weight set is fetched (decoded) once per expert: get_expert(e) returns
+    (Wg_e, Wu_e, Wd_e).  Same definition; the terms of a token are added in
+    expert order, then the shared expert."""
+    x_tok = np.asarray(x_tok, np.float64)
+    idx = np.asarray(idx, np.int64)
+    out = np.zeros_like(x_tok)
+    for e in np.unique(idx):
+        rows, slots = np.nonzero(idx == e)
+        wg, wu, wd = get_expert(int(e))
+        out[rows] += w[rows, slots][:, None] * swiglu(x_tok[rows], wg, wu, wd)
+    if shared is not None:
+        out += swiglu(x_tok, *shared)
+    return out
+
+
 # --------------------------------------------------------------------------
 # FP8 (e4m3) configuration.  Weights arrive quantised (e4m3 values with one
 # float32 scale per 128 x 128 block); activations are quantised on the fly per

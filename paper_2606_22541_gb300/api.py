@@ -93,7 +93,7 @@ def _ws(ws):
     return (_ptr(ws), ctypes.c_size_t(0 if ws is None else ws.numel() * ws.element_size()))
 
 
-def asap_moe_router_logits(h, x, logits, ws=None, stream=None):
+def asap_moe_router_logits(h, x, logits, ws, stream=None):
     p, n = _ws(ws)
     check("asap_moe_router_logits",
           lib().asap_moe_router_logits(h.ptr, _ptr(x), x.shape[0], _ptr(logits), p, n, _stream(stream)))

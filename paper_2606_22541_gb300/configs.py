@@ -58,10 +58,18 @@ class LayerConfig:
 
 
 def _stress_lengths(seed, count=8, mu=7.5, sigma=1.0, lo=128, hi=16384):
+    """The recipe of the stress workload's micro-batch lengths: round(lognormal
+    (mu, sigma)) clipped to [lo, hi] from numpy's PCG64 stream.  numpy does
+    not keep its lognormal stream stable across versions, so the workload uses
+    the lengths this recipe gave once (STRESS_LENGTHS), not a fresh draw."""
     import numpy as np
     rng = np.random.Generator(np.random.PCG64(seed))
     v = np.round(rng.lognormal(mu, sigma, size=count)).astype(int)
     return [int(min(max(a, lo), hi)) for a in v]
+
+
+# _stress_lengths(1003) with numpy 2.5
+STRESS_LENGTHS = [4014, 1179, 8045, 5228, 362, 1108, 2591, 5185]
 
 
 TINY = LayerConfig("tiny", hidden=256, n_experts=8, top_k=2, inter=128, n_shared=0,
@@ -74,7 +82,7 @@ DSV3 = LayerConfig("dsv3_bf16", hidden=7168, n_experts=256, top_k=8, inter=2048,
                    route_scale=2.5, microbatches=[4096] * 4, seed=1002)
 STRESS = LayerConfig("dsv3_stress", hidden=7168, n_experts=256, top_k=8, inter=2048, n_shared=1,
                      shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
-                     route_scale=2.5, microbatches=_stress_lengths(1003), zipf_s=1.1, seed=1003)
+                     route_scale=2.5, microbatches=list(STRESS_LENGTHS), zipf_s=1.1, seed=1003)
 DSV3_FP8 = LayerConfig("dsv3_fp8", hidden=7168, n_experts=256, top_k=8, inter=2048, n_shared=1,
                        shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
                        route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[4096] * 8,

@@ -63,7 +63,7 @@ Layout layout(const asap_moe_config& c, long long n) {
   };
   const long long nk = n * c.top_k;
   const long long chunks = (n + asap::kChunkTokens - 1) / asap::kChunkTokens;
-  L.logits = take(static_cast<size_t>(n) * c.n_experts * 4);
+  L.logits = take(static_cast<size_t>(asap::kMaxRouterSplits) * n * c.n_experts * 4);  // K-slice planes
   L.idx = take(static_cast<size_t>(nk) * 4);
   L.w = take(static_cast<size_t>(nk) * 4);
   L.hist = take(static_cast<size_t>(chunks) * c.n_experts * 4);
@@ -106,7 +106,22 @@ int check_call(asap_moe_t h, int32_t n, void* ws, size_t ws_bytes, bool needs_ws
 
 // ------------------------------------------------------------ launch helpers
 
-int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, cudaStream_t st) {
+// Number of K slices of the tensor-core router GEMM for n tokens: enough
+// CTAs to cover the SMs (one 128-row tile x one 256-expert tile per slice),
+// at least 8 k-blocks per slice.
+int router_splits(asap_moe_t h, int n) {
+  if (!h->tc_router) return 1;
+  const int mtiles = asap::ceil_div(n, asap::kGemmBM);
+  const int kit = h->cfg.hidden / asap::kGemmBK;
+  int s = h->num_sms / std::max(mtiles, 1);
+  s = std::min(s, kit / 8);
+  s = std::min(s, asap::kMaxRouterSplits);
+  return std::max(s, 1);
+}
+
+// Router logits as ``splits`` planes of partial sums [splits][n][E] (planes
+// are added in order by the consumer); splits == 1 writes the logits.
+int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int splits, cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   if (h->tc_router) {
     CUtensorMap maps[4];
@@ -129,7 +144,9 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, cudaStr
     a.status = h->status;
     a.hint_a = 0;
     a.hint_b = 2;
-    const int tiles = asap::ceil_div(n, asap::kGemmBM);
+    a.k_splits = splits;
+    a.split_rows0 = n;
+    const int tiles = asap::ceil_div(n, asap::kGemmBM) * splits;
     CU_TRY(asap::gemm_launch(asap::EPI_F32, maps, a, std::min(tiles, h->num_sms), st), "router GEMM launch");
   } else {
     CU_TRY(asap::launch_router_small(x, h->router_w, n, c.hidden, c.n_experts, logits, st), "router launch");
@@ -150,12 +167,12 @@ asap::GateParams gate_params(asap_moe_t h) {
   return p;
 }
 
-int run_gate_scan(asap_moe_t h, const float* logits, int n, int32_t* idx, float* w, int32_t* counts,
+int run_gate_scan(asap_moe_t h, const float* logits, int splits, int n, int32_t* idx, float* w, int32_t* counts,
                   int32_t* offsets, void* ws, cudaStream_t st) {
   const Layout L = layout(h->cfg, n);
   int32_t* hist = at<int32_t>(ws, L.hist);
   int32_t* base = at<int32_t>(ws, L.chunk_base);
-  CU_TRY(asap::launch_gate(logits, n, gate_params(h), idx, w, hist, st), "gate launch");
+  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
                            st),
          "scan launch");
@@ -203,6 +220,7 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   a.status = h->status;
   a.hint_a = 2;
   a.hint_b = 1;
+  a.k_splits = 1;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -246,6 +264,7 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.status = h->status;
   a.hint_a = 2;
   a.hint_b = 1;
+  a.k_splits = 1;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -343,6 +362,10 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
   };
   cudaError_t e = cudaGetDevice(&h->device);
   if (e != cudaSuccess) return bail(cuda_fail(e, "cudaGetDevice"));
+  // The weights may still be in flight on any of the caller's streams; the
+  // copies below run on a private non-blocking stream, so wait for all of it.
+  e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return bail(cuda_fail(e, "synchronise before reading the weights"));
   e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
   if (e != cudaSuccess) return bail(cuda_fail(e, "SM count"));
   int cc_major = 0, cc_minor = 0;
@@ -408,11 +431,18 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
 
 ASAP_API int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, float* logits, void* ws,
                                     size_t ws_bytes, void* stream) {
-  int r = check_call(h, n, ws, ws_bytes, false);
+  int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !logits || !aligned16(x) || !aligned16(logits))
     return fail(ASAP_ERR_INVALID, "x and logits must be non-NULL and 16-byte aligned");
-  return run_router_logits(h, x, n, logits, S(stream));
+  const int splits = router_splits(h, n);
+  if (splits == 1) return run_router_logits(h, x, n, logits, 1, S(stream));
+  // the same K slices and the same order of addition as asap_moe_route
+  float* parts = at<float>(ws, layout(h->cfg, n).logits);
+  if ((r = run_router_logits(h, x, n, parts, splits, S(stream))) != ASAP_OK) return r;
+  CU_TRY(asap::launch_reduce_splits(parts, splits, static_cast<long long>(n) * h->cfg.n_experts, logits, S(stream)),
+         "logit reduction launch");
+  return ASAP_OK;
 }
 
 ASAP_API int asap_moe_route_logits(asap_moe_t h, const float* logits, int32_t n, int32_t* idx, float* w,
@@ -420,7 +450,7 @@ ASAP_API int asap_moe_route_logits(asap_moe_t h, const float* logits, int32_t n,
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!logits || !idx || !w || !counts || !offsets) return fail(ASAP_ERR_INVALID, "NULL tensor");
-  return run_gate_scan(h, logits, n, idx, w, counts, offsets, ws, S(stream));
+  return run_gate_scan(h, logits, 1, n, idx, w, counts, offsets, ws, S(stream));
 }
 
 ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w, int32_t* counts,
@@ -429,9 +459,10 @@ ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !idx || !w || !counts || !offsets || !aligned16(x)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   float* logits = at<float>(ws, layout(h->cfg, n).logits);
-  r = run_router_logits(h, x, n, logits, S(stream));
+  const int splits = router_splits(h, n);
+  r = run_router_logits(h, x, n, logits, splits, S(stream));
   if (r != ASAP_OK) return r;
-  return run_gate_scan(h, logits, n, idx, w, counts, offsets, ws, S(stream));
+  return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, S(stream));
 }
 
 ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx, void* x_perm,
@@ -528,8 +559,9 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
   void* x_perm = at<void>(ws, L.x_perm);
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
-  if ((r = run_router_logits(h, x, n, logits, st)) != ASAP_OK) return r;
-  if ((r = run_gate_scan(h, logits, n, idx, w, counts, offsets, ws, st)) != ASAP_OK) return r;
+  const int splits = router_splits(h, n);
+  if ((r = run_router_logits(h, x, n, logits, splits, st)) != ASAP_OK) return r;
+  if ((r = run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, st)) != ASAP_OK) return r;
   CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base), x_perm,
                                perm_src, perm_dst, h->status, st),
          "dispatch launch");
@@ -576,7 +608,7 @@ constexpr int kStaticRouteMaxTokens = 4096;
 constexpr size_t kStaticLogitsBytes =
     static_cast<size_t>(kStaticRouteMaxTokens) * ASAP_MOE_MAX_EXPERTS * sizeof(float);   // 4 MiB
 constexpr size_t kStaticChunkBytes = static_cast<size_t>(kStaticRouteMaxTokens / asap::kChunkTokens) *
-                                     ASAP_MOE_MAX_EXPERTS * sizeof(int32_t);                  // 64 KiB
+                                     ASAP_MOE_MAX_EXPERTS * sizeof(int32_t);                  // 128 KiB
 constexpr size_t kStaticRouteBytes = kStaticLogitsBytes + 2 * kStaticChunkBytes;
 
 constexpr int kStaticMaxDevices = 64;
@@ -632,8 +664,8 @@ ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int3
   // every scratch element read below is written earlier on the same stream
   // (logits by the router, all E entries of each chunk's histogram by the
   // gate kernel), so nothing has to be cleared between calls
-  if ((r = run_router_logits(h, x, n, logits, st)) != ASAP_OK) return r;
-  CU_TRY(asap::launch_gate(logits, n, gate_params(h), idx, w, hist, st), "gate launch");
+  if ((r = run_router_logits(h, x, n, logits, 1, st)) != ASAP_OK) return r;
+  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base, st),
          "scan launch");
   return ASAP_OK;

@@ -24,7 +24,8 @@ __device__ __forceinline__ void record_status(uint32_t* st, uint32_t bits) {
   if (st) atomicOr(st, bits);
 }
 
-constexpr int kChunkTokens = 64;  // tokens per routing / dispatch chunk
+constexpr int kChunkTokens = 32;  // tokens per routing / dispatch chunk (one warp each)
+constexpr int kMaxRouterSplits = 8;  // K slices of the tensor-core router GEMM
 constexpr int kMaxExperts = 256;
 constexpr int kMaxTopK = 8;
 

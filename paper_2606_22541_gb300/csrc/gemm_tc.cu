@@ -48,7 +48,7 @@ constexpr int kBarBytes = 256;  // 12 mbarriers + tmem slot + abort flag
 constexpr size_t kSmemBytes = 1024 + STAGES * (A_BYTES + B_BYTES) + kBarBytes + sizeof(Sched);
 
 struct Tile {
-  int a_row, b_row, rows, n_tile, kit;
+  int a_row, b_row, rows, n_tile, kb0, kb1, split;
   bool p1;
 };
 
@@ -61,15 +61,20 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
       if (s->tile_start[mid] <= t) lo = mid; else hi = mid;
     }
     const int g = lo;
-    const int local = t - s->tile_start[g];
+    int local = t - s->tile_start[g];
     const int mt = s->mtiles[g];
+    const int per_split = mt * a.n_tiles0;
+    const int split = local / per_split;   // K slice (split-K of problem 0)
+    local -= split * per_split;
     const int nt = local / mt;
     const int mi = local - nt * mt;
     T.a_row = s->row_base[g] + mi * BM;
     T.rows = min(BM, s->mrows[g] - mi * BM);
     T.b_row = g * a.b_stride0 + nt * BN;
     T.n_tile = nt;
-    T.kit = a.k_iters0;
+    T.split = split;
+    T.kb0 = static_cast<int>(static_cast<long long>(a.k_iters0) * split / a.k_splits);
+    T.kb1 = static_cast<int>(static_cast<long long>(a.k_iters0) * (split + 1) / a.k_splits);
     T.p1 = false;
   } else {
     const int u = t - total0;
@@ -80,7 +85,9 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
     T.rows = min(BM, a.m1 - mi * BM);
     T.b_row = nt * BN;
     T.n_tile = nt;
-    T.kit = a.k_iters1;
+    T.split = 0;
+    T.kb0 = 0;
+    T.kb1 = a.k_iters1;
     T.p1 = true;
   }
 }
@@ -89,7 +96,8 @@ template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr,
                                               int row) {
   const bool valid = row < T.rows;
-  const long long orow = static_cast<long long>(T.a_row) + row;
+  // split-K slices of problem 0 write separate output planes
+  const long long orow = static_cast<long long>(T.a_row) + row + (T.p1 ? 0 : T.split * a.split_rows0);
   if constexpr (EPI == EPI_SWIGLU) {
     uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
     const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
@@ -227,7 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         sch->mrows[g] = m;
         cnt[i] = (m + BM - 1) / BM;
         sch->mtiles[g] = cnt[i];
-        local += cnt[i] * args.n_tiles0;
+        local += cnt[i] * args.n_tiles0 * args.k_splits;
       }
     }
     int incl = local;
@@ -242,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int g = lane * 8 + i;
       if (g < G) {
         sch->tile_start[g] = run;
-        run += cnt[i] * args.n_tiles0;
+        run += cnt[i] * args.n_tiles0 * args.k_splits;
       }
     }
     if (lane == 31) sch->tile_start[G] = incl;
@@ -270,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       decode_tile(t, sch, G, total0, args, T);
       const CUtensorMap* mA = T.p1 ? &tmA1 : &tmA0;
       const CUtensorMap* mB = T.p1 ? &tmB1 : &tmB0;
-      for (int kb = 0; kb < T.kit; ++kb) {
+      for (int kb = T.kb0; kb < T.kb1; ++kb) {
         if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag)) {
           ok = false;
           break;
@@ -311,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_after();
       const uint32_t d = tmem_base + acc * BN;
-      for (int kb = 0; kb < T.kit; ++kb) {
+      for (int kb = T.kb0; kb < T.kb1; ++kb) {
         if (!mbar_wait(full_bar(stage), phase, abort_flag)) {
           ok = false;
           break;
@@ -322,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
           tc_mma_bf16(d, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kIdesc,
-                      (kb | kk) != 0);
+                      (kb > T.kb0 || kk > 0) ? 1u : 0u);
         }
         issued = true;
         tc_commit(empty_bar(stage));

@@ -35,6 +35,8 @@ struct GemmArgs {
   long long ldo1;
   uint32_t* status;
   int hint_a, hint_b;      // L2 priority of A / B loads: 0 normal, 1 first, 2 last
+  int k_splits;            // problem 0 split into this many K slices (>= 1)
+  long long split_rows0;   // output rows between the planes of consecutive K slices
 };
 
 constexpr int kGemmBM = 128;
@@ -58,8 +60,11 @@ struct GateParams {
 };
 cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int E, float* logits,
                                 cudaStream_t s);
-cudaError_t launch_gate(const float* logits, int n, const GateParams& p, int32_t* idx, float* w,
+// logits: ``splits`` planes of [n, E] partial sums, added in plane order.
+// hist is written expert-major: hist[e * n_chunks + chunk].
+cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                         int32_t* hist, cudaStream_t s);
+cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane, float* out, cudaStream_t s);
 cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
                         cudaStream_t s);
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,

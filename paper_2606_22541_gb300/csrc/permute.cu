@@ -15,19 +15,22 @@ namespace asap {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kDispatchWarps = 16;  // 512 threads >= kChunkTokens * kMaxTopK entries
+constexpr int kDispatchWarps = kChunkTokens;  // one warp per token for the copies
+constexpr int kRankWarps = kChunkTokens * kMaxTopK / 32;  // warps that rank the chunk's entries
 
 // One CTA per chunk of kChunkTokens tokens.  Entry i = t_local * k + j is
-// handled by thread i, so warp order and lane order follow (t, j); the rank
-// of an entry inside its expert is (entries of that expert in earlier
-// chunks) + (in earlier warps of this chunk) + (in earlier lanes of this
-// warp): positions increase with (t, j) inside every segment.
+// ranked by thread i, so warp order and lane order follow (t, j); the rank of
+// an entry inside its expert is (entries of that expert in earlier chunks)
+// + (in earlier warps of this chunk) + (in earlier lanes of this warp):
+// positions increase with (t, j) inside every segment.  chunk_base is
+// expert-major: chunk_base[e * n_chunks + chunk].  Then one warp per token
+// reads its row once and writes it to its k positions.
 __global__ void __launch_bounds__(kDispatchWarps * 32)
     dispatch_kernel(const uint4* __restrict__ x, int n, int V, int k, int E,
-                    const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base,
+                    const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
                     uint4* __restrict__ x_perm, int32_t* __restrict__ perm_src,
                     int32_t* __restrict__ perm_dst, uint32_t* status) {
-  __shared__ int wcnt[kDispatchWarps][kMaxExperts];
+  __shared__ int wcnt[kRankWarps][kMaxExperts];
   __shared__ int spos[kChunkTokens * kMaxTopK];
   const int c = blockIdx.x;
   const int t0 = c * kChunkTokens;
@@ -35,26 +38,28 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
   const int ne = nt * k;
   const int nk = n * k;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = threadIdx.x; i < kDispatchWarps * E; i += blockDim.x) (&wcnt[0][0])[(i / E) * kMaxExperts + i % E] = 0;
+  for (int i = threadIdx.x; i < kRankWarps * E; i += blockDim.x) wcnt[i / E][i % E] = 0;
   __syncthreads();
 
   const int i = threadIdx.x;
-  int e = -1;
-  if (i < ne) {
-    e = idx[static_cast<long long>(t0) * k + i];
-    if (e < 0 || e >= E) {
-      record_status(status, ST_BAD_EXPERT_INDEX);
-      e = -1;
+  int e = -1, rank = 0;
+  if (warp < kRankWarps) {
+    if (i < ne) {
+      e = idx[static_cast<long long>(t0) * k + i];
+      if (e < 0 || e >= E) {
+        record_status(status, ST_BAD_EXPERT_INDEX);
+        e = -1;
+      }
     }
+    const unsigned peers = __match_any_sync(kFull, e);
+    rank = __popc(peers & ((1u << lane) - 1u));
+    if (e >= 0 && lane == __ffs(peers) - 1) wcnt[warp][e] = __popc(peers);
   }
-  const unsigned peers = __match_any_sync(kFull, e);
-  const int rank = __popc(peers & ((1u << lane) - 1u));
-  if (e >= 0 && lane == __ffs(peers) - 1) wcnt[warp][e] = __popc(peers);
   __syncthreads();
   for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
-    int run = chunk_base[static_cast<long long>(c) * E + ee];
+    int run = chunk_base[static_cast<long long>(ee) * n_chunks + c];
 #pragma unroll
-    for (int w = 0; w < kDispatchWarps; ++w) {
+    for (int w = 0; w < kRankWarps; ++w) {
       const int v = wcnt[w][ee];
       wcnt[w][ee] = run;
       run += v;
@@ -76,16 +81,28 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
   }
   __syncthreads();
   // row copies: one warp per token, read once, write k times
-  for (int lt = warp; lt < nt; lt += kDispatchWarps) {
-    const uint4* src = x + static_cast<long long>(t0 + lt) * V;
+  if (warp < nt) {
+    const uint4* src = x + static_cast<long long>(t0 + warp) * V;
     int p[kMaxTopK];
 #pragma unroll
-    for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[lt * k + j] : -1;
-    for (int v = lane; v < V; v += 32) {
-      const uint4 val = __ldg(src + v);
+    for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[warp * k + j] : -1;
+    int v = lane;
+    for (; v + 32 < V; v += 64) {
+      const uint4 a = __ldg(src + v);
+      const uint4 b = __ldg(src + v + 32);
 #pragma unroll
       for (int j = 0; j < kMaxTopK; ++j)
-        if (p[j] >= 0) x_perm[static_cast<long long>(p[j]) * V + v] = val;
+        if (p[j] >= 0) {
+          uint4* d = x_perm + static_cast<long long>(p[j]) * V;
+          d[v] = a;
+          d[v + 32] = b;
+        }
+    }
+    for (; v < V; v += 32) {
+      const uint4 a = __ldg(src + v);
+#pragma unroll
+      for (int j = 0; j < kMaxTopK; ++j)
+        if (p[j] >= 0) x_perm[static_cast<long long>(p[j]) * V + v] = a;
     }
   }
 }
@@ -117,6 +134,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
       }
     }
   }
+#pragma unroll 2
   for (int v = lane; v < V; v += 32) {
     uint4 yv[kMaxTopK];
 #pragma unroll
@@ -181,9 +199,10 @@ cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int
                             const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  dispatch_kernel<<<ceil_div(n, kChunkTokens), kDispatchWarps * 32, 0, s>>>(
-      static_cast<const uint4*>(x), n, H / 8, k, E, idx, chunk_base, static_cast<uint4*>(x_perm), perm_src,
-      perm_dst, status);
+  const int chunks = ceil_div(n, kChunkTokens);
+  dispatch_kernel<<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
+                                                         chunk_base, chunks, static_cast<uint4*>(x_perm), perm_src,
+                                                         perm_dst, status);
   return cudaGetLastError();
 }
 

@@ -12,6 +12,8 @@
 
 #include <math_constants.h>
 
+#include <algorithm>
+
 namespace asap {
 
 namespace {
@@ -79,14 +81,18 @@ __device__ __forceinline__ void warp_argmax(float& v, int& i) {
   }
 }
 
-constexpr int kGateWarps = 8;
+constexpr int kGateWarps = kChunkTokens;  // one warp per token of the chunk
 
-// One CTA per chunk of kChunkTokens tokens, one warp per token at a time.
-// Lane l holds experts l, l+32, ..., so expert order and (i, lane) order agree.
-__global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __restrict__ logits, int n,
-                                                               GateParams p, int32_t* __restrict__ idx,
+// One CTA per chunk of kChunkTokens tokens, one warp per token.  The logits
+// arrive as ``splits`` partial planes (K slices of the router GEMM) that are
+// added in slice order.  Lane l holds experts l, l+32, ..., so expert order
+// and (i, lane) order agree.  The chunk's expert histogram is written
+// transposed: hist[e * n_chunks + chunk].
+__global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __restrict__ logits, int splits,
+                                                               long long plane, int n, GateParams p,
+                                                               int32_t* __restrict__ idx,
                                                                float* __restrict__ wout,
-                                                               int32_t* __restrict__ hist) {
+                                                               int32_t* __restrict__ hist, int n_chunks) {
   __shared__ int shist[kMaxExperts];
   __shared__ float ssel[kGateWarps][kMaxExperts];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -105,7 +111,11 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int e = lane + 32 * i;
-      const float l = e < E ? lrow[e] : -CUDART_INF_F;
+      float l = -CUDART_INF_F;
+      if (e < E) {
+        l = lrow[e];
+        for (int s2 = 1; s2 < splits; ++s2) l += lrow[s2 * plane + e];
+      }
       if (grouped) {
         const float s = 1.0f / (1.0f + expf(-l));
         sv[i] = s;
@@ -237,12 +247,12 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
   }
   __syncthreads();
   if (hist)
-    for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(blockIdx.x) * E + e] = shist[e];
+    for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(e) * n_chunks + blockIdx.x] = shist[e];
 }
 
 // ------------------------------------------------------------ histogram only
 __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ idx, int n, int k, int E,
-                                                   int32_t* __restrict__ hist, uint32_t* status) {
+                                                   int32_t* __restrict__ hist, int n_chunks, uint32_t* status) {
   __shared__ int shist[kMaxExperts];
   for (int e = threadIdx.x; e < E; e += blockDim.x) shist[e] = 0;
   __syncthreads();
@@ -254,12 +264,13 @@ __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ i
     else record_status(status, ST_BAD_EXPERT_INDEX);
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(blockIdx.x) * E + e] = shist[e];
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(e) * n_chunks + blockIdx.x] = shist[e];
 }
 
 // ------------------------------------------------------------ scan
-// One CTA.  Warp w scans experts w, w+32, ... over the chunks (32 chunks per
-// step), giving each (chunk, expert) the number of earlier entries of that
+// One CTA.  hist and chunk_base are stored expert-major ([E][n_chunks]), so
+// warp w scans experts w, w+32, ... over 32 consecutive chunks per coalesced
+// load, giving each (expert, chunk) the number of earlier entries of that
 // expert; then counts, the exclusive offsets, and the absolute chunk bases.
 __global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ hist, int n_chunks, int E,
                                                     int32_t* __restrict__ counts,
@@ -269,17 +280,19 @@ __global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ 
   __shared__ int soff[kMaxExperts + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int e = warp; e < E; e += 32) {
+    const int32_t* hrow = hist + static_cast<long long>(e) * n_chunks;
+    int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
     int run = 0;
     for (int c0 = 0; c0 < n_chunks; c0 += 32) {
       const int c = c0 + lane;
-      const int v = c < n_chunks ? hist[static_cast<long long>(c) * E + e] : 0;
+      const int v = c < n_chunks ? hrow[c] : 0;
       int incl = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int u = __shfl_up_sync(kFull, incl, o);
         if (lane >= o) incl += u;
       }
-      if (c < n_chunks) chunk_base[static_cast<long long>(c) * E + e] = run + incl - v;
+      if (c < n_chunks) brow[c] = run + incl - v;
       run += __shfl_sync(kFull, incl, 31);
     }
     if (lane == 0) scount[e] = run;
@@ -315,8 +328,22 @@ __global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ 
     offsets[e] = soff[e];
   }
   if (threadIdx.x == 0) offsets[E] = soff[E];
-  const int total = n_chunks * E;
-  for (int i = threadIdx.x; i < total; i += blockDim.x) chunk_base[i] += soff[i % E];
+  for (int e = warp; e < E; e += 32) {
+    int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
+    const int base = soff[e];
+    for (int c = lane; c < n_chunks; c += 32) brow[c] += base;
+  }
+}
+
+// Sum of the K-slice planes of the router GEMM, added in slice order.
+__global__ void reduce_splits_kernel(const float* __restrict__ parts, int splits, long long plane,
+                                     float* __restrict__ out) {
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < plane;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    float v = parts[i];
+    for (int s2 = 1; s2 < splits; ++s2) v += parts[s2 * plane + i];
+    out[i] = v;
+  }
 }
 
 }  // namespace
@@ -329,17 +356,27 @@ cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int
   return cudaGetLastError();
 }
 
-cudaError_t launch_gate(const float* logits, int n, const GateParams& p, int32_t* idx, float* w,
+cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                         int32_t* hist, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  gate_kernel<<<ceil_div(n, kChunkTokens), kGateWarps * 32, 0, s>>>(logits, n, p, idx, w, hist);
+  const int chunks = ceil_div(n, kChunkTokens);
+  gate_kernel<<<chunks, kGateWarps * 32, 0, s>>>(logits, splits, static_cast<long long>(n) * p.n_experts, n, p,
+                                                  idx, w, hist, chunks);
   return cudaGetLastError();
 }
 
 cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
                         cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  hist_kernel<<<ceil_div(n, kChunkTokens), 256, 0, s>>>(idx, n, k, E, hist, status);
+  const int chunks = ceil_div(n, kChunkTokens);
+  hist_kernel<<<chunks, 256, 0, s>>>(idx, n, k, E, hist, chunks, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane, float* out, cudaStream_t s) {
+  if (plane <= 0) return cudaSuccess;
+  const int blocks = static_cast<int>(std::min<long long>((plane + 255) / 256, 4096));
+  reduce_splits_kernel<<<blocks, 256, 0, s>>>(parts, splits, plane, out);
   return cudaGetLastError();
 }
 

@@ -82,7 +82,7 @@ def test_router_logits_within_bound(cfg):
     c = Case.get(cfg)
     x = c.tokens(0)
     logits = torch.empty((x.shape[0], cfg.n_experts), dtype=torch.float32, device=DEV)
-    api.asap_moe_router_logits(c.h, x, logits)
+    api.asap_moe_router_logits(c.h, x, logits, c.ws(x.shape[0]))
     torch.cuda.synchronize()
     xf = bf16_to_f64(x)
     L = oracle.router_logits(xf, c.wf["router_w"])
@@ -288,6 +288,23 @@ def test_layer_matches_oracle(cfg):
     assert_clean(c)
 
 
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL, ST_SMALL], ids=lambda c: c.name)
+def test_route_equals_route_logits_of_router_logits(cfg):
+    """asap_moe_route == asap_moe_route_logits(asap_moe_router_logits(x))."""
+    c = Case.get(cfg)
+    x = c.tokens(0)
+    n, k, E = x.shape[0], cfg.top_k, cfg.n_experts
+    a = run_route(c, x)
+    logits = torch.empty((n, E), dtype=torch.float32, device=DEV)
+    api.asap_moe_router_logits(c.h, x, logits, c.ws(n))
+    b = (torch.empty((n, k), dtype=torch.int32, device=DEV), torch.empty((n, k), dtype=torch.float32, device=DEV),
+         torch.empty(E, dtype=torch.int32, device=DEV), torch.empty(E + 1, dtype=torch.int32, device=DEV))
+    api.asap_moe_route_logits(c.h, logits, *b, c.ws(n))
+    torch.cuda.synchronize()
+    for u, v in zip(a, b):
+        assert torch.equal(u, v)
+
+
 @pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
 def test_layer_equals_composed_calls_bit_for_bit(cfg):
     c = Case.get(cfg)
@@ -424,3 +441,30 @@ def test_ffn_halves_equal_expert_ffn_and_h_matches_oracle(cfg):
             ref = oracle.silu(X @ c.wf["w_gate"][e].T) * (X @ c.wf["w_up"][e].T)
             compare_rows(hg[a:b], ref, rel_norm=5e-3)
     assert_clean(c)
+
+
+def test_create_waits_for_weights_still_being_written():
+    """Weights produced by kernels still running on another stream are read
+    only after they are complete (create synchronises first)."""
+    cfg = inputs.small_variant(TINY, name="tiny_race")
+    w = inputs.make_weights(cfg, DEV)
+    ref = api.asap_moe_create(cfg, w, 160)
+    x = inputs.make_tokens(cfg, 160, 0, DEV)
+    out_ref = torch.empty_like(x)
+    api.asap_moe_layer(ref, x, out_ref, api.workspace(ref, 160))
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    w2 = {}
+    with torch.cuda.stream(side):
+        torch.cuda._sleep(50_000_000)                 # keep the side stream busy
+        for k_, v in w.items():
+            if v is not None:
+                w2[k_] = torch.zeros_like(v)
+                w2[k_].copy_(v)                      # the copy lands after the sleep
+    h2 = api.asap_moe_create(cfg, w2, 160)
+    out = torch.empty_like(x)
+    api.asap_moe_layer(h2, x, out, api.workspace(h2, 160))
+    torch.cuda.synchronize()
+    assert torch.equal(out.view(torch.int16), out_ref.view(torch.int16))
+    ref.close()
+    h2.close()

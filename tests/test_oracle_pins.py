@@ -306,6 +306,20 @@ def test_per_token_independence():
     assert np.allclose(tok, full[some], rtol=1e-12, atol=1e-12)
 
 
+def test_expert_major_sampling_equals_token_major():
+    rng = np.random.default_rng(34)
+    n, H, E, k, I = 12, 16, 6, 3, 8
+    x = rng.normal(0, 1, (n, H))
+    wg, wu = rng.normal(0, 0.3, (2, E, I, H))
+    wd = rng.normal(0, 0.3, (E, H, I))
+    sh = (rng.normal(0, 0.2, (I, H)), rng.normal(0, 0.2, (I, H)), rng.normal(0, 0.2, (H, I)))
+    idx = np.array([rng.permutation(E)[:k] for _ in range(n)])
+    w = rng.uniform(0, 1, (n, k))
+    a = layer.moe_layer_tokens(x, idx, w, wg, wu, wd, sh)
+    b = layer.moe_layer_tokens_by_expert(x, idx, w, lambda e: (wg[e], wu[e], wd[e]), sh)
+    assert np.allclose(a, b, rtol=1e-12, atol=1e-12)
+
+
 def test_shared_expert_enters_once():
     rng = np.random.default_rng(33)
     n, H, E, k, I = 10, 16, 4, 2, 8
