@@ -177,6 +177,18 @@ __device__ __forceinline__ void tmem_ld_wait() {
 // bytes stacked along M/N (stride byte offset 1024).  The leading byte offset
 // is unused for this layout.  Bits 46-48 hold the fixed value 0b001; bits
 // 61-63 select the 128-byte swizzle (2).
+// Same for 64-byte rows (32 bf16) written with 64-byte swizzle: 8-row atoms
+// of 512 bytes; bits 61-63 select the 64-byte swizzle (4).
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t addr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((addr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(512 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;
+  return d;
+}
+
 __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
   uint64_t d = 0;
   d |= static_cast<uint64_t>((addr & 0x3FFFFu) >> 4);

@@ -7,9 +7,11 @@
 // list is derived on the device from those offsets, so the host never reads
 // the per-expert counts back (the bubble-free principle of Section 3.4.2).
 //
-// Design (one CTA per SM, persistent, warp-specialised, 192 threads):
-//   warp 0   : TMA producer.  A box [128 rows, 64 K] and B box [256 rows, 64 K],
-//              128-byte swizzle, into a 4-stage shared-memory ring.
+// Design (one CTA per SM, persistent, warp-specialised, 224 threads):
+//   warps 0,6: TMA producers.  Weight boxes B [256 rows, 64 K] (warp 0) and
+//              activation boxes A [128 rows, 64 K] (warp 6) into separate
+//              shared-memory rings (4 + 4 stages, or 5 + 3 when the
+//              activations are L2-resident), 128-byte swizzle.
 //   warp 1   : TMEM allocator and MMA issuer (one thread): 4 x
 //              tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) per stage,
 //              fp32 accumulator in TMEM, two accumulators (2 x 256 columns) so
@@ -30,10 +32,24 @@ namespace asap {
 
 namespace {
 
-constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK, STAGES = 4;
+// Separate rings for the two operands.  The kernel streams HBM, and a k-step
+// can start only when both of its boxes have landed, so the useful pipeline
+// depth is that of the shallowest ring whose operand comes from HBM.  The
+// gate/up GEMM reads its activations (x_perm, just written by dispatch) from
+// HBM as well, so both rings get 4 stages; the down GEMM's activations (h)
+// are still in L2 from the gate/up launch, so its weight ring gets 5 stages
+// and its activation ring 3 (measured on GB300: 1.84 -> 1.73 ms per launch at
+// 4096 DeepSeek-V3 tokens, while 3 + 5 would slow the gate/up GEMM by 15 %).
+template <int EPI>
+struct Rings {
+  static constexpr int A = EPI == EPI_BF16 ? 3 : 4;
+  static constexpr int B = EPI == EPI_BF16 ? 5 : 4;
+};
+constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK;
+
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;  // warp 0 B producer, 1 MMA, 2-5 epilogue, 6 A producer
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
@@ -44,8 +60,11 @@ struct Sched {
   int mrows[kMaxExperts];
 };
 
-constexpr int kBarBytes = 256;  // 12 mbarriers + tmem slot + abort flag
-constexpr size_t kSmemBytes = 1024 + STAGES * (A_BYTES + B_BYTES) + kBarBytes + sizeof(Sched);
+constexpr int kBarBytes = 256;  // 2*SA + 2*SB + 5 mbarriers, tmem slot, abort flag
+template <int EPI>
+__host__ __device__ constexpr size_t smem_bytes() {
+  return 1024 + Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
+}
 
 struct Tile {
   int a_row, b_row, rows, n_tile, kb0, kb1, split;
@@ -169,21 +188,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const __grid_constant__ CUtensorMap tmB0,
                         const __grid_constant__ CUtensorMap tmA1,
                         const __grid_constant__ CUtensorMap tmB1, const GemmArgs args) {
+  constexpr int SA = Rings<EPI>::A, SB = Rings<EPI>::B;
+  static_assert(8 * (2 * SA + 2 * SB + 5) + 8 <= kBarBytes, "barrier area");
+  static_assert(smem_bytes<EPI>() <= 227 * 1024, "shared memory budget");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
   const uint32_t sA = base;
-  const uint32_t sB = base + STAGES * A_BYTES;
-  uint8_t* bar_area = gbase + STAGES * (A_BYTES + B_BYTES);
+  const uint32_t sB = base + SA * A_BYTES;
+  uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;
   const uint32_t bar0 = smem_u32(bar_area);
-  // mbarriers (8 bytes each): full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
-  auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
-  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
-  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * STAGES + 5));
+  // mbarriers (8 bytes each): fullA[SA], emptyA[SA], fullB[SB], emptyB[SB],
+  // tfull[2], tempty[2], drain
+  auto fullA = [&](int s) { return bar0 + 8u * s; };
+  auto emptyA = [&](int s) { return bar0 + 8u * (SA + s); };
+  auto fullB = [&](int s) { return bar0 + 8u * (2 * SA + s); };
+  auto emptyB = [&](int s) { return bar0 + 8u * (2 * SA + SB + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * SA + 2 * SB + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * SA + 2 * SB + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * SA + 2 * SB + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
 
@@ -193,9 +218,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      for (int s = 0; s < STAGES; ++s) {
-        mbar_init(full_bar(s), 1);
-        mbar_init(empty_bar(s), 1);
+      for (int s = 0; s < SA; ++s) {
+        mbar_init(fullA(s), 1);
+        mbar_init(emptyA(s), 1);
+      }
+      for (int s = 0; s < SB; ++s) {
+        mbar_init(fullB(s), 1);
+        mbar_init(emptyB(s), 1);
       }
       for (int a = 0; a < 2; ++a) {
         mbar_init(tfull_bar(a), 1);
@@ -265,10 +294,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int total0 = sch->tile_start[G];
   const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
 
-  if (warp == 0 && lane == 0) {
-    // ------------------------------------------------------------ producer
-    const uint64_t pol_a = l2_policy(args.hint_a);
-    const uint64_t pol_b = l2_policy(args.hint_b);
+  if ((warp == 0 || warp == 6) && lane == 0) {
+    // ------------------------------------------------------------ producers
+    // warp 0 streams the weight tiles (B) into its ring, warp 6 the
+    // activation tiles (A) into its own; the MMA issuer joins them per k-step.
+    const bool isB = warp == 0;
+    const int nst = isB ? SB : SA;
+    const uint32_t bytes = isB ? B_BYTES : A_BYTES;
+    const uint32_t ring = isB ? sB : sA;
+    const uint64_t pol = l2_policy(isB ? args.hint_b : args.hint_a);
     int stage = 0;
     uint32_t phase = 0;
     uint32_t pending = 0, issued_phase = 0;  // bit s: stage s has a load in flight
@@ -276,19 +310,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
-      const CUtensorMap* mA = T.p1 ? &tmA1 : &tmA0;
-      const CUtensorMap* mB = T.p1 ? &tmB1 : &tmB0;
+      const CUtensorMap* m = isB ? (T.p1 ? &tmB1 : &tmB0) : (T.p1 ? &tmA1 : &tmA0);
+      const int row = isB ? T.b_row : T.a_row;
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
-        if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag)) {
+        const uint32_t full = isB ? fullB(stage) : fullA(stage);
+        if (!mbar_wait(isB ? emptyB(stage) : emptyA(stage), phase ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(full_bar(stage), A_BYTES + B_BYTES);
-        tma_load_2d(sA + stage * A_BYTES, mA, full_bar(stage), kb * BK, T.a_row, pol_a);
-        tma_load_2d(sB + stage * B_BYTES, mB, full_bar(stage), kb * BK, T.b_row, pol_b);
+        mbar_arrive_expect_tx(full, bytes);
+        tma_load_2d(ring + stage * bytes, m, full, kb * BK, row, pol);
         pending |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-        if (++stage == STAGES) {
+        if (++stage == nst) {
           stage = 0;
           phase ^= 1u;
         }
@@ -299,13 +333,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       record_status(args.status, ST_WAIT_TIMEOUT);
       // let the copies already issued land before the CTA's memory goes away
       int dummy = 0;
-      for (int s = 0; s < STAGES; ++s)
-        if (pending & (1u << s)) mbar_wait(full_bar(s), (issued_phase >> s) & 1u, &dummy);
+      for (int s = 0; s < nst; ++s)
+        if (pending & (1u << s)) mbar_wait(isB ? fullB(s) : fullA(s), (issued_phase >> s) & 1u, &dummy);
     }
   } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    int stage = 0;
-    uint32_t phase = 0;
+    int sa = 0, sb = 0;
+    uint32_t pa = 0, pb = 0;
     bool ok = true, issued = false;
     int it = 0;
     for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
@@ -320,23 +354,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t d = tmem_base + acc * BN;
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
-        if (!mbar_wait(full_bar(stage), phase, abort_flag)) {
+        if (!mbar_wait(fullA(sa), pa, abort_flag) || !mbar_wait(fullB(sb), pb, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t a_addr = sA + stage * A_BYTES;
-        const uint32_t b_addr = sB + stage * B_BYTES;
+        const uint32_t a_addr = sA + sa * A_BYTES;
+        const uint32_t b_addr = sB + sb * B_BYTES;
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
-          tc_mma_bf16(d, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kIdesc,
-                      (kb > T.kb0 || kk > 0) ? 1u : 0u);
+          const uint64_t adesc = BK == 64 ? smem_desc_sw128(a_addr + kk * 32) : smem_desc_sw64(a_addr + kk * 32);
+          const uint64_t bdesc = BK == 64 ? smem_desc_sw128(b_addr + kk * 32) : smem_desc_sw64(b_addr + kk * 32);
+          tc_mma_bf16(d, adesc, bdesc, kIdesc, (kb > T.kb0 || kk > 0) ? 1u : 0u);
         }
         issued = true;
-        tc_commit(empty_bar(stage));
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1u;
+        tc_commit(emptyA(sa));
+        tc_commit(emptyB(sb));
+        if (++sa == SA) {
+          sa = 0;
+          pa ^= 1u;
+        }
+        if (++sb == SB) {
+          sb = 0;
+          pb ^= 1u;
         }
       }
       if (ok) tc_commit(tfull_bar(acc));
@@ -350,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(drain_bar, 0, &dummy);
       }
     }
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp <= 5) {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;
     const int row = q * 32 + lane;
@@ -387,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int EPI>
 cudaError_t set_attr() {
   return cudaFuncSetAttribute(grouped_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(kSmemBytes));
+                              static_cast<int>(smem_bytes<EPI>()));
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -411,7 +451,6 @@ EncodeFn get_encode_fn() {
 
 }  // namespace
 
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(sizeof(Sched) + 0 <= 8192, "schedule table");
 
 cudaError_t gemm_set_attributes() {
@@ -427,13 +466,13 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, 
   const dim3 g(grid), b(kThreads);
   switch (epi) {
     case EPI_SWIGLU:
-      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, smem_bytes<EPI_SWIGLU>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
       break;
     case EPI_BF16:
-      grouped_gemm_kernel<EPI_BF16><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_BF16><<<g, b, smem_bytes<EPI_BF16>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
       break;
     default:
-      grouped_gemm_kernel<EPI_F32><<<g, b, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_F32><<<g, b, smem_bytes<EPI_F32>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
       break;
   }
   return cudaGetLastError();
@@ -455,7 +494,8 @@ bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t
   const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
   const cuuint32_t estr[2] = {1, 1};
   const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
-                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        BK == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     if (err) *err = "cuTensorMapEncodeTiled failed with CUresult " + std::to_string(static_cast<int>(r));

@@ -41,7 +41,10 @@ struct GemmArgs {
 
 constexpr int kGemmBM = 128;
 constexpr int kGemmBN = 256;
-constexpr int kGemmBK = 64;
+#ifndef ASAP_GEMM_BK
+#define ASAP_GEMM_BK 64
+#endif
+constexpr int kGemmBK = ASAP_GEMM_BK;  // 64 (128-byte swizzle) or 32 (64-byte swizzle)
 
 cudaError_t gemm_set_attributes();
 // maps: A0, B0, A1, B1 (A1/B1 may repeat A0/B0 when m1 == 0)
