@@ -92,9 +92,12 @@ typedef enum {
 
 typedef enum {
   ASAP_BF16 = 0,              /* bf16 storage, fp32 accumulation */
-  ASAP_FP8_E4M3_BLOCK128 = 1  /* e4m3 weights with one fp32 scale per 128x128
-                                 block; activations e4m3 per token per 128
-                                 channels (reserved: ASAP_ERR_UNSUPPORTED) */
+  ASAP_FP8_E4M3_BLOCK128 = 1  /* e4m3 expert weights with one fp32 scale per
+                                 128 x 128 block; activations (x before the
+                                 gate/up GEMM, h before the down GEMM) e4m3 per
+                                 token per 128 channels with fp32 scales
+                                 s = amax / 448; fp32 accumulation; bf16 out.
+                                 The router stays bf16. */
 } asap_dtype;
 
 /* Shape and gating of one MoE layer.  Table 1 of the paper: E_total = 256,
@@ -118,13 +121,15 @@ typedef struct {
   int32_t max_tokens;    /* largest micro-batch a call may pass */
 } asap_moe_config;
 
-/* Device pointers to one layer's weights (bf16, row-major).  They are copied
- * (and re-packed) by asap_moe_create; the caller may free them afterwards.
- *   router_w  [E, H]
+/* Device pointers to one layer's weights (row-major).  They are copied (and
+ * re-packed) by asap_moe_create; the caller may free them afterwards.
+ *   router_w  [E, H] bf16
  *   router_bias [E] fp32 or NULL: selection-only correction bias
- *   w_gate, w_up [E][I, H];  w_down [E][H, I]
+ *   w_gate, w_up [E][I, H];  w_down [E][H, I]  (bf16, or e4m3 for FP8)
  *   sh_gate, sh_up [I_s, H]; sh_down [H, I_s]   (NULL when n_shared == 0)
- *   s_* : fp32 block scales of the FP8 configuration (NULL for bf16)        */
+ *   FP8 only, fp32 scales of 128 x 128 blocks (NULL for bf16):
+ *   s_gate, s_up [E][I/128][H/128]; s_down [E][H/128][I/128];
+ *   sh_s_gate, sh_s_up [I_s/128][H/128]; sh_s_down [H/128][I_s/128]      */
 typedef struct {
   const void* router_w;
   const float* router_bias;
@@ -188,7 +193,10 @@ int asap_moe_route_logits(asap_moe_t h, const float* logits, int32_t n, int32_t*
 /* Dispatch (Section 3.2.1 token payload): from idx, build perm_src/perm_dst
  * and copy every token row into its k expert segments of x_perm.  idx values
  * outside [0, E) are recorded in the status word and the entry is skipped.
- * x_perm_scales is reserved for the FP8 configuration (pass NULL). */
+ * FP8 configuration: x_perm is e4m3 [n*k, H] and x_perm_scales fp32
+ * [n*k, H/128] (one scale per row per 128 channels, s = amax / 448); each
+ * token row is quantised once and written k times.  bf16: x_perm_scales is
+ * ignored (pass NULL). */
 int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx,
                       void* x_perm, float* x_perm_scales, int32_t* perm_src,
                       int32_t* perm_dst, void* ws, size_t ws_bytes, void* stream);
@@ -196,7 +204,10 @@ int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx
 /* Expert FFN (Section 3.4.2 GMM): y_perm rows of expert e's segment
  * [offsets[e], offsets[e+1]) = SwiGLU_e(x_perm rows); y_shared = shared
  * SwiGLU of x (ignored when n_shared == 0).  The grouped GEMMs find their
- * tiles on the device from offsets (offsets[E] must equal n*k). */
+ * tiles on the device from offsets (offsets[E] must equal n*k).  FP8
+ * configuration: x_perm / x_perm_scales as produced by asap_moe_dispatch; x
+ * stays bf16 (quantised here for the shared expert); h is quantised to e4m3
+ * per row per 128 channels between the two GEMMs; y_perm, y_shared bf16. */
 int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
                         const int32_t* offsets, const void* x, int32_t n, void* y_perm,
                         void* y_shared, void* ws, size_t ws_bytes, void* stream);
@@ -207,7 +218,9 @@ int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_sc
  *   gate_up: h_perm [n*k, I] = silu(X_e Wg_e^T) * (X_e Wu_e^T) per segment,
  *            h_shared [n, I_s] likewise for the shared expert on x;
  *   down   : y_perm = h_perm Wd_e^T per segment, y_shared = h_shared Ws_d^T.
- * No workspace.  *_scales are reserved for the FP8 configuration (NULL). */
+ * No workspace.  bf16 configuration only (the FP8 configuration returns
+ * ASAP_ERR_UNSUPPORTED; its h is e4m3 with scales, use asap_moe_expert_ffn);
+ * *_scales are ignored (pass NULL). */
 int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
                             const int32_t* offsets, const void* x, int32_t n, void* h_perm,
                             void* h_shared, void* stream);

@@ -46,8 +46,8 @@ def bf16_bits_to_f64(bits):
     return _BF16_TABLE[np.asarray(bits, dtype=np.uint16)]
 
 
-def e4m3_bits_to_f64(bits):
-    """OCP e4m3fn bit patterns (uint8) -> float64, exactly.
+def _e4m3_fields_to_f64(bits):
+    """OCP e4m3fn bit patterns (uint8) -> float64, exactly, from the fields.
 
     Layout: 1 sign bit, 4 exponent bits (bias 7), 3 fraction bits.
     exponent 0     : subnormal, value = (-1)^s * 2^-6 * f/8
@@ -63,6 +63,18 @@ def e4m3_bits_to_f64(bits):
     mag = np.where(e == 0, sub, normal)
     mag = np.where((e == 15) & (f == 7), np.nan, mag)
     return sign * mag
+
+
+_E4M3_TABLE = None
+
+
+def e4m3_bits_to_f64(bits):
+    """OCP e4m3fn bit patterns (uint8) -> float64, exactly: a lookup in the
+    table of all 256 patterns decoded by ``_e4m3_fields_to_f64``."""
+    global _E4M3_TABLE
+    if _E4M3_TABLE is None:
+        _E4M3_TABLE = _e4m3_fields_to_f64(np.arange(256, dtype=np.uint8))
+    return _E4M3_TABLE[np.asarray(bits, dtype=np.uint8)]
 
 
 E4M3_MAX = 448.0

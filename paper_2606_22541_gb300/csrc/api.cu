@@ -24,6 +24,12 @@ struct asap_moe_s {
   void* sh_down = nullptr;       // [H, Is]
   uint32_t* status = nullptr;    // device status word
   bool tc_router = false;        // router GEMM on the tensor core (E == 256)
+  bool fp8 = false;              // e4m3 experts with fp32 128 x 128 block scales
+  // FP8 only: block scales, gate/up rows interleaved like the weights
+  float* gu_scales = nullptr;     // [E][2I/128][H/128]
+  float* d_scales = nullptr;      // [E][H/128][I/128]
+  float* sh_gu_scales = nullptr;  // [2Is/128][H/128]
+  float* sh_d_scales = nullptr;   // [H/128][Is/128]
   CUtensorMap tm_router, tm_gate_up, tm_down, tm_sh_gate_up, tm_sh_down;
 };
 
@@ -49,7 +55,11 @@ int cuda_fail(cudaError_t e, const char* what) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Layout {
-  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst, x_perm, h, h_sh, y_sh;
+  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst;
+  // bf16: x_perm (also y_perm in asap_moe_layer), h, h_sh, y_sh
+  size_t x_perm, h, h_sh, y_sh;
+  // fp8: quantised rows and their per-128-channel scales, bf16 expert outputs
+  size_t xq, xs, xq_sh, xs_sh, hq, hs, hq_sh, hs_sh, y_perm;
   size_t total;
 };
 
@@ -61,21 +71,36 @@ Layout layout(const asap_moe_config& c, long long n) {
     off = (off + bytes + 255) & ~static_cast<size_t>(255);
     return o;
   };
-  const long long nk = n * c.top_k;
-  const long long chunks = (n + asap::kChunkTokens - 1) / asap::kChunkTokens;
-  L.logits = take(static_cast<size_t>(asap::kMaxRouterSplits) * n * c.n_experts * 4);  // K-slice planes
-  L.idx = take(static_cast<size_t>(nk) * 4);
-  L.w = take(static_cast<size_t>(nk) * 4);
-  L.hist = take(static_cast<size_t>(chunks) * c.n_experts * 4);
-  L.chunk_base = take(static_cast<size_t>(chunks) * c.n_experts * 4);
-  L.counts = take(static_cast<size_t>(c.n_experts) * 4);
-  L.offsets = take(static_cast<size_t>(c.n_experts + 1) * 4);
-  L.perm_src = take(static_cast<size_t>(nk) * 4);
-  L.perm_dst = take(static_cast<size_t>(nk) * 4);
-  L.x_perm = take(static_cast<size_t>(nk) * c.hidden * 2);  // also holds y_perm in asap_moe_layer
-  L.h = take(static_cast<size_t>(nk) * c.inter * 2);
-  L.h_sh = take(c.n_shared ? static_cast<size_t>(n) * c.shared_inter * 2 : 0);
-  L.y_sh = take(c.n_shared ? static_cast<size_t>(n) * c.hidden * 2 : 0);
+  const size_t nk = static_cast<size_t>(n) * c.top_k;
+  const size_t N = static_cast<size_t>(n);
+  const size_t chunks = (N + asap::kChunkTokens - 1) / asap::kChunkTokens;
+  const size_t H = c.hidden, I = c.inter, Is = c.n_shared ? c.shared_inter : 0, E = c.n_experts;
+  L.logits = take(asap::kMaxRouterSplits * N * E * 4);  // K-slice planes
+  L.idx = take(nk * 4);
+  L.w = take(nk * 4);
+  L.hist = take(chunks * E * 4);
+  L.chunk_base = take(chunks * E * 4);
+  L.counts = take(E * 4);
+  L.offsets = take((E + 1) * 4);
+  L.perm_src = take(nk * 4);
+  L.perm_dst = take(nk * 4);
+  if (c.dtype == ASAP_FP8_E4M3_BLOCK128) {
+    L.xq = take(nk * H);
+    L.xs = take(nk * (H / 128) * 4);
+    L.xq_sh = take(N * H * (Is ? 1 : 0));
+    L.xs_sh = take(N * (H / 128) * 4 * (Is ? 1 : 0));
+    L.hq = take(nk * I);
+    L.hs = take(nk * (I / 128) * 4);
+    L.hq_sh = take(N * Is);
+    L.hs_sh = take(N * (Is / 128) * 4);
+    L.y_perm = take(nk * H * 2);
+    L.y_sh = take(N * H * 2 * (Is ? 1 : 0));
+  } else {
+    L.x_perm = take(nk * H * 2);  // also holds y_perm in asap_moe_layer
+    L.h = take(nk * I * 2);
+    L.h_sh = take(N * Is * 2);
+    L.y_sh = take(N * H * 2 * (Is ? 1 : 0));
+  }
   L.total = off;
   return L;
 }
@@ -279,6 +304,115 @@ int run_expert_ffn(asap_moe_t h, const void* x_perm, const int32_t* offsets, con
   return run_down(h, hbuf, offsets, hsh, n, y_perm, y_sh, st);
 }
 
+// FP8 GEMM1: hq = e4m3(silu(Xq Wg^T) * (Xq Wu^T)) with its row scales, routed
+// segments plus the shared expert on the quantised x.
+int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t* offsets, const void* xq_sh,
+                    const float* xs_sh, int n, void* hq, float* hs, void* hq_sh, float* hs_sh, cudaStream_t st) {
+  const asap_moe_config& c = h->cfg;
+  const long long nk = static_cast<long long>(n) * c.top_k;
+  const bool sh = c.n_shared != 0;
+  std::string err;
+  CUtensorMap maps[4];
+  if (!asap::encode_tmap_u8(&maps[0], xq, nk, c.hidden, asap::kGemmBM, &err)) return fail(ASAP_ERR_INVALID, "x_perm: " + err);
+  maps[1] = h->tm_gate_up;
+  if (sh) {
+    if (!asap::encode_tmap_u8(&maps[2], xq_sh, n, c.hidden, asap::kGemmBM, &err))
+      return fail(ASAP_ERR_INVALID, "quantised x: " + err);
+    maps[3] = h->tm_sh_gate_up;
+  } else {
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+  }
+  asap::Fp8Args f{};
+  asap::GemmArgs& a = f.g;
+  a.offsets = offsets;
+  a.groups = c.n_experts;
+  a.m0 = static_cast<int>(nk);
+  a.b_stride0 = 2 * c.inter;
+  a.n_tiles0 = c.inter / 128;
+  a.k_iters0 = c.hidden / asap::kFp8BK;
+  a.out0 = hq;
+  a.ldo0 = c.inter;
+  a.m1 = sh ? n : 0;
+  a.n_tiles1 = sh ? c.shared_inter / 128 : 0;
+  a.k_iters1 = c.hidden / asap::kFp8BK;
+  a.out1 = hq_sh;
+  a.ldo1 = c.shared_inter;
+  a.status = h->status;
+  a.hint_a = 2;
+  a.hint_b = 1;
+  a.k_splits = 1;
+  f.a_scale0 = xs;
+  f.a_sld0 = c.hidden / 128;
+  f.a_scale1 = xs_sh;
+  f.a_sld1 = c.hidden / 128;
+  f.b_scale0 = h->gu_scales;
+  f.b_nblk0 = 2 * c.inter / 128;
+  f.b_scale1 = h->sh_gu_scales;
+  f.b_nblk1 = sh ? 2 * c.shared_inter / 128 : 0;
+  f.out_scale0 = hs;
+  f.o_sld0 = c.inter / 128;
+  f.out_scale1 = hs_sh;
+  f.o_sld1 = sh ? c.shared_inter / 128 : 0;
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
+  CU_TRY(asap::fp8_gemm_launch(asap::EPI_SWIGLU, maps, f, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+         "fp8 gate/up GEMM launch");
+  return ASAP_OK;
+}
+
+// FP8 GEMM2: y = (hq * hs) (Wd * sd)^T, bf16 out.
+int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* offsets, const void* hq_sh,
+                 const float* hs_sh, int n, void* y_perm, void* y_sh, cudaStream_t st) {
+  const asap_moe_config& c = h->cfg;
+  const long long nk = static_cast<long long>(n) * c.top_k;
+  const bool sh = c.n_shared != 0;
+  std::string err;
+  CUtensorMap maps[4];
+  if (!asap::encode_tmap_u8(&maps[0], hq, nk, c.inter, asap::kGemmBM, &err)) return fail(ASAP_ERR_INVALID, "h: " + err);
+  maps[1] = h->tm_down;
+  if (sh) {
+    if (!asap::encode_tmap_u8(&maps[2], hq_sh, n, c.shared_inter, asap::kGemmBM, &err))
+      return fail(ASAP_ERR_INVALID, "h_shared: " + err);
+    maps[3] = h->tm_sh_down;
+  } else {
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+  }
+  asap::Fp8Args f{};
+  asap::GemmArgs& a = f.g;
+  a.offsets = offsets;
+  a.groups = c.n_experts;
+  a.m0 = static_cast<int>(nk);
+  a.b_stride0 = c.hidden;
+  a.n_tiles0 = c.hidden / asap::kGemmBN;
+  a.k_iters0 = c.inter / asap::kFp8BK;
+  a.out0 = y_perm;
+  a.ldo0 = c.hidden;
+  a.m1 = sh ? n : 0;
+  a.n_tiles1 = sh ? c.hidden / asap::kGemmBN : 0;
+  a.k_iters1 = sh ? c.shared_inter / asap::kFp8BK : 0;
+  a.out1 = y_sh;
+  a.ldo1 = c.hidden;
+  a.status = h->status;
+  a.hint_a = 2;
+  a.hint_b = 1;
+  a.k_splits = 1;
+  f.a_scale0 = hs;
+  f.a_sld0 = c.inter / 128;
+  f.a_scale1 = hs_sh;
+  f.a_sld1 = sh ? c.shared_inter / 128 : 0;
+  f.b_scale0 = h->d_scales;
+  f.b_nblk0 = c.hidden / 128;
+  f.b_scale1 = h->sh_d_scales;
+  f.b_nblk1 = c.hidden / 128;
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
+  CU_TRY(asap::fp8_gemm_launch(asap::EPI_BF16, maps, f, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+         "fp8 down GEMM launch");
+  return ASAP_OK;
+}
+
 }  // namespace
 
 // ============================================================ public API
@@ -307,9 +441,7 @@ ASAP_API int asap_moe_check_config(const asap_moe_config* c) {
     if (c->top_k > c->topk_groups * gsz) return fail(ASAP_ERR_INVALID, "top_k exceeds the experts of the kept groups");
     if (!(c->route_scale > 0.0f)) return fail(ASAP_ERR_INVALID, "route_scale must be positive");
   }
-  if (c->dtype == ASAP_FP8_E4M3_BLOCK128)
-    return fail(ASAP_ERR_UNSUPPORTED, "the FP8 configuration is not built yet");
-  if (c->dtype != ASAP_BF16) return fail(ASAP_ERR_INVALID, "unknown dtype");
+  if (c->dtype != ASAP_BF16 && c->dtype != ASAP_FP8_E4M3_BLOCK128) return fail(ASAP_ERR_INVALID, "unknown dtype");
   if (c->max_tokens < 1 || static_cast<long long>(c->max_tokens) * c->top_k >= (1ll << 31))
     return fail(ASAP_ERR_INVALID, "max_tokens * top_k must be in [1, 2^31)");
   return ASAP_OK;
@@ -337,6 +469,10 @@ ASAP_API int asap_moe_destroy(asap_moe_t h) {
   cudaFree(h->sh_gate_up);
   cudaFree(h->sh_down);
   cudaFree(h->status);
+  cudaFree(h->gu_scales);
+  cudaFree(h->d_scales);
+  cudaFree(h->sh_gu_scales);
+  cudaFree(h->sh_d_scales);
   cudaSetDevice(prev);
   delete h;
   return ASAP_OK;
@@ -351,6 +487,10 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
     return fail(ASAP_ERR_INVALID, "router and expert weights are required");
   if (cfg->n_shared && (!wts->sh_gate || !wts->sh_up || !wts->sh_down))
     return fail(ASAP_ERR_INVALID, "shared-expert weights are required when n_shared == 1");
+  if (cfg->dtype == ASAP_FP8_E4M3_BLOCK128 &&
+      (!wts->s_gate || !wts->s_up || !wts->s_down ||
+       (cfg->n_shared && (!wts->sh_s_gate || !wts->sh_s_up || !wts->sh_s_down))))
+    return fail(ASAP_ERR_INVALID, "the FP8 configuration needs the fp32 block scales of every expert matrix");
   const asap_moe_config& c = *cfg;
   asap_moe_s* h = new asap_moe_s();
   h->cfg = c;
@@ -375,12 +515,15 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
     return bail(fail(ASAP_ERR_UNSUPPORTED, "libasap_moe is built for sm_103a (GB300) only; device is sm_" +
                                                std::to_string(cc_major) + std::to_string(cc_minor)));
   e = asap::gemm_set_attributes();
+  if (e == cudaSuccess) e = asap::fp8_gemm_set_attributes();
   if (e != cudaSuccess) return bail(cuda_fail(e, "GEMM attributes"));
+  h->fp8 = c.dtype == ASAP_FP8_E4M3_BLOCK128;
   e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking);
   if (e != cudaSuccess) return bail(cuda_fail(e, "stream"));
 
   const size_t H = c.hidden, E = c.n_experts, I = c.inter, Is = c.shared_inter;
-  const size_t router_bytes = E * H * 2, gu_bytes = E * 2 * I * H * 2, down_bytes = E * H * I * 2;
+  const size_t wb = h->fp8 ? 1 : 2;  // bytes per expert-weight element
+  const size_t router_bytes = E * H * 2, gu_bytes = E * 2 * I * H * wb, down_bytes = E * H * I * wb;
   if ((e = cudaMalloc(&h->status, 256)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc status"));
   if ((e = cudaMemsetAsync(h->status, 0, 256, st)) != cudaSuccess) return bail(cuda_fail(e, "memset"));
   if ((e = cudaMalloc(&h->router_w, router_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc router"));
@@ -393,19 +536,45 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
   }
   if ((e = cudaMalloc(&h->gate_up, gu_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc gate/up"));
   if ((e = asap::launch_pack_gate_up(wts->w_gate, wts->w_up, static_cast<int>(E), static_cast<int>(I),
-                                     static_cast<int>(H), h->gate_up, st)) != cudaSuccess)
+                                     static_cast<long long>(H * wb), h->gate_up, st)) != cudaSuccess)
     return bail(cuda_fail(e, "pack gate/up"));
   if ((e = cudaMalloc(&h->down, down_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc down"));
   if ((e = cudaMemcpyAsync(h->down, wts->w_down, down_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
     return bail(cuda_fail(e, "copy down"));
   if (c.n_shared) {
-    if ((e = cudaMalloc(&h->sh_gate_up, 2 * Is * H * 2)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared"));
-    if ((e = asap::launch_pack_gate_up(wts->sh_gate, wts->sh_up, 1, static_cast<int>(Is), static_cast<int>(H),
+    if ((e = cudaMalloc(&h->sh_gate_up, 2 * Is * H * wb)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared"));
+    if ((e = asap::launch_pack_gate_up(wts->sh_gate, wts->sh_up, 1, static_cast<int>(Is), static_cast<long long>(H * wb),
                                        h->sh_gate_up, st)) != cudaSuccess)
       return bail(cuda_fail(e, "pack shared"));
-    if ((e = cudaMalloc(&h->sh_down, H * Is * 2)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared down"));
-    if ((e = cudaMemcpyAsync(h->sh_down, wts->sh_down, H * Is * 2, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+    if ((e = cudaMalloc(&h->sh_down, H * Is * wb)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared down"));
+    if ((e = cudaMemcpyAsync(h->sh_down, wts->sh_down, H * Is * wb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
       return bail(cuda_fail(e, "copy shared down"));
+  }
+  if (h->fp8) {
+    // scale rows interleaved like the weight rows: gate block b -> 2b, up block b -> 2b+1
+    const size_t kb = H / 128, rowb = kb * 4;
+    auto interleave = [&](float** dst, const float* g, const float* u, size_t blocks) -> cudaError_t {
+      cudaError_t r = cudaMalloc(dst, 2 * blocks * rowb);
+      if (r == cudaSuccess) r = cudaMemcpy2DAsync(*dst, 2 * rowb, g, rowb, rowb, blocks, cudaMemcpyDeviceToDevice, st);
+      if (r == cudaSuccess)
+        r = cudaMemcpy2DAsync(reinterpret_cast<char*>(*dst) + rowb, 2 * rowb, u, rowb, rowb, blocks,
+                              cudaMemcpyDeviceToDevice, st);
+      return r;
+    };
+    if ((e = interleave(&h->gu_scales, wts->s_gate, wts->s_up, E * (I / 128))) != cudaSuccess)
+      return bail(cuda_fail(e, "gate/up scales"));
+    const size_t dsb = E * (H / 128) * (I / 128) * 4;
+    if ((e = cudaMalloc(&h->d_scales, dsb)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(h->d_scales, wts->s_down, dsb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+      return bail(cuda_fail(e, "down scales"));
+    if (c.n_shared) {
+      if ((e = interleave(&h->sh_gu_scales, wts->sh_s_gate, wts->sh_s_up, Is / 128)) != cudaSuccess)
+        return bail(cuda_fail(e, "shared gate/up scales"));
+      const size_t sdb = (H / 128) * (Is / 128) * 4;
+      if ((e = cudaMalloc(&h->sh_d_scales, sdb)) != cudaSuccess ||
+          (e = cudaMemcpyAsync(h->sh_d_scales, wts->sh_s_down, sdb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+        return bail(cuda_fail(e, "shared down scales"));
+    }
   }
   if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return bail(cuda_fail(e, "create sync"));
   cudaStreamDestroy(st);
@@ -415,15 +584,16 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
   h->tc_router = (c.n_experts == asap::kGemmBN);
   if (h->tc_router && !asap::encode_tmap_bf16(&h->tm_router, h->router_w, E, H, asap::kGemmBN, &err))
     return bail(fail(ASAP_ERR_CUDA, "router map: " + err));
-  if (!asap::encode_tmap_bf16(&h->tm_gate_up, h->gate_up, E * 2 * I, H, asap::kGemmBN, &err))
-    return bail(fail(ASAP_ERR_CUDA, "gate/up map: " + err));
-  if (!asap::encode_tmap_bf16(&h->tm_down, h->down, E * H, I, asap::kGemmBN, &err))
-    return bail(fail(ASAP_ERR_CUDA, "down map: " + err));
+  auto enc = [&](CUtensorMap* m, const void* p, uint64_t rows, uint64_t cols) {
+    return h->fp8 ? asap::encode_tmap_u8(m, p, rows, cols, asap::kGemmBN, &err)
+                  : asap::encode_tmap_bf16(m, p, rows, cols, asap::kGemmBN, &err);
+  };
+  if (!enc(&h->tm_gate_up, h->gate_up, E * 2 * I, H)) return bail(fail(ASAP_ERR_CUDA, "gate/up map: " + err));
+  if (!enc(&h->tm_down, h->down, E * H, I)) return bail(fail(ASAP_ERR_CUDA, "down map: " + err));
   if (c.n_shared) {
-    if (!asap::encode_tmap_bf16(&h->tm_sh_gate_up, h->sh_gate_up, 2 * Is, H, asap::kGemmBN, &err))
+    if (!enc(&h->tm_sh_gate_up, h->sh_gate_up, 2 * Is, H))
       return bail(fail(ASAP_ERR_CUDA, "shared gate/up map: " + err));
-    if (!asap::encode_tmap_bf16(&h->tm_sh_down, h->sh_down, H, Is, asap::kGemmBN, &err))
-      return bail(fail(ASAP_ERR_CUDA, "shared down map: " + err));
+    if (!enc(&h->tm_sh_down, h->sh_down, H, Is)) return bail(fail(ASAP_ERR_CUDA, "shared down map: " + err));
   }
   *out = h;
   return ASAP_OK;
@@ -468,11 +638,11 @@ ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx
 ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx, void* x_perm,
                                float* x_perm_scales, int32_t* perm_src, int32_t* perm_dst, void* ws,
                                size_t ws_bytes, void* stream) {
-  (void)x_perm_scales;
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !idx || !x_perm || !perm_src || !perm_dst || !aligned16(x) || !aligned16(x_perm))
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+  if (h->fp8 && !x_perm_scales) return fail(ASAP_ERR_INVALID, "the FP8 configuration needs x_perm_scales");
   const asap_moe_config& c = h->cfg;
   const Layout L = layout(c, n);
   const int chunks = asap::ceil_div(n, asap::kChunkTokens);
@@ -482,16 +652,20 @@ ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int
   CU_TRY(asap::launch_hist(idx, n, c.top_k, c.n_experts, hist, h->status, st), "hist launch");
   CU_TRY(asap::launch_scan(hist, chunks, c.n_experts, at<int32_t>(ws, L.counts), at<int32_t>(ws, L.offsets), base, st),
          "scan launch");
-  CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, base, x_perm, perm_src, perm_dst, h->status,
-                               st),
-         "dispatch launch");
+  if (h->fp8)
+    CU_TRY(asap::launch_dispatch_fp8(x, n, c.hidden, c.top_k, c.n_experts, idx, base, x_perm, x_perm_scales, nullptr,
+                                     nullptr, perm_src, perm_dst, h->status, st),
+           "dispatch launch");
+  else
+    CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, base, x_perm, perm_src, perm_dst,
+                                 h->status, st),
+           "dispatch launch");
   return ASAP_OK;
 }
 
 ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
                                  const int32_t* offsets, const void* x, int32_t n, void* y_perm, void* y_shared,
                                  void* ws, size_t ws_bytes, void* stream) {
-  (void)x_perm_scales;
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x_perm || !offsets || !y_perm || !aligned16(x_perm) || !aligned16(y_perm))
@@ -499,8 +673,20 @@ ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* 
   if (h->cfg.n_shared && (!x || !y_shared || !aligned16(x) || !aligned16(y_shared)))
     return fail(ASAP_ERR_INVALID, "x and y_shared are required for the shared expert");
   const Layout L = layout(h->cfg, n);
-  return run_expert_ffn(h, x_perm, offsets, x, n, y_perm, y_shared, at<void>(ws, L.h), at<void>(ws, L.h_sh),
-                        S(stream));
+  cudaStream_t st = S(stream);
+  if (h->fp8) {
+    if (!x_perm_scales) return fail(ASAP_ERR_INVALID, "the FP8 configuration needs x_perm_scales");
+    const asap_moe_config& c = h->cfg;
+    void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
+    float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
+    if (c.n_shared) CU_TRY(asap::launch_quantize_rows(x, n, c.hidden, xq_sh, xs_sh, st), "quantise launch");
+    if ((r = run_gate_up_fp8(h, x_perm, x_perm_scales, offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), st)) != ASAP_OK)
+      return r;
+    return run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
+                        at<float>(ws, L.hs_sh), n, y_perm, y_shared, st);
+  }
+  return run_expert_ffn(h, x_perm, offsets, x, n, y_perm, y_shared, at<void>(ws, L.h), at<void>(ws, L.h_sh), st);
 }
 
 ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
@@ -509,6 +695,7 @@ ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const flo
   (void)x_perm_scales;
   int r = check_call(h, n, nullptr, 0, false);
   if (r != ASAP_OK || n == 0) return r;
+  if (h->fp8) return fail(ASAP_ERR_UNSUPPORTED, "the FP8 configuration runs the FFN through asap_moe_expert_ffn");
   if (!x_perm || !offsets || !h_perm || !aligned16(x_perm) || !aligned16(h_perm))
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!x || !h_shared || !aligned16(x) || !aligned16(h_shared)))
@@ -522,6 +709,7 @@ ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float*
   (void)h_perm_scales;
   int r = check_call(h, n, nullptr, 0, false);
   if (r != ASAP_OK || n == 0) return r;
+  if (h->fp8) return fail(ASAP_ERR_UNSUPPORTED, "the FP8 configuration runs the FFN through asap_moe_expert_ffn");
   if (!h_perm || !offsets || !y_perm || !aligned16(h_perm) || !aligned16(y_perm))
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!h_shared || !y_shared || !aligned16(h_shared) || !aligned16(y_shared)))
@@ -557,11 +745,29 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
   int32_t* offsets = at<int32_t>(ws, L.offsets);
   int32_t* perm_src = at<int32_t>(ws, L.perm_src);
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
-  void* x_perm = at<void>(ws, L.x_perm);
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
   const int splits = router_splits(h, n);
   if ((r = run_router_logits(h, x, n, logits, splits, st)) != ASAP_OK) return r;
   if ((r = run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, st)) != ASAP_OK) return r;
+  if (h->fp8) {
+    void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
+    float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
+    CU_TRY(asap::launch_dispatch_fp8(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base),
+                                     at<void>(ws, L.xq), at<float>(ws, L.xs), xq_sh, xs_sh, perm_src, perm_dst,
+                                     h->status, st),
+           "dispatch launch");
+    if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), st)) != ASAP_OK)
+      return r;
+    void* y_perm = at<void>(ws, L.y_perm);
+    if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
+                          at<float>(ws, L.hs_sh), n, y_perm, y_sh, st)) != ASAP_OK)
+      return r;
+    CU_TRY(asap::launch_combine(y_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
+           "combine launch");
+    return ASAP_OK;
+  }
+  void* x_perm = at<void>(ws, L.x_perm);
   CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base), x_perm,
                                perm_src, perm_dst, h->status, st),
          "dispatch launch");

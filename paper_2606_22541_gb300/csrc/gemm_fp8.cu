@@ -1,0 +1,415 @@
+// Grouped GEMM with e4m3 operands and fp32 block scales on the sm_103a
+// tensor core (tcgen05.mma kind::f8f6f4), fed by TMA.
+//
+// The FP8 configuration of the MoE layer stores expert weights as e4m3 with
+// one fp32 scale per 128 x 128 block and quantises activations per token per
+// 128 channels.  The scales are arbitrary fp32 values, so they cannot ride
+// in the tensor core's power-of-two block-scale path; instead every 128-wide
+// K block is multiplied into one of two TMEM partial buffers (ping-pong) and
+// eight epilogue warps add it, times (row scale x block scale), into fp32
+// register accumulators while the tensor core already works on the next
+// block.
+//
+// Roles (one CTA per SM, persistent, 352 threads):
+//   warp 0    : weight producer, boxes [256 rows, 128 B], 4-stage ring
+//   warp 10   : activation producer, boxes [128 rows, 128 B], 4-stage ring
+//   warp 1    : TMEM allocator (512 columns) and MMA issuer: per K block
+//               4 x tcgen05.mma.cta_group::1.kind::f8f6f4 M=128 N=256 K=32
+//   warps 2-9 : epilogue; warp w owns TMEM lanes 32*(w%4).. and, with
+//               h = (w-2)/4, one half of the 256 columns of a tile
+// Tile schedule, masking and bounded waits as in the bf16 kernel.
+#include "common.cuh"
+#include "gemm_sched.cuh"
+#include "internal.h"
+
+#include <cuda_fp8.h>
+
+#include <mutex>
+
+namespace asap {
+
+namespace {
+
+constexpr int BM = kGemmBM, BN = kGemmBN, BK = kFp8BK;
+constexpr int SA = 4, SB = 4;
+constexpr int A_BYTES = BM * BK;  // 16 KB
+constexpr int B_BYTES = BN * BK;  // 32 KB
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 32 * (3 + kEpiWarps);  // 352
+constexpr int kAProdWarp = 2 + kEpiWarps;      // 10
+constexpr uint32_t kTmemCols = 2 * BN;          // two partial buffers
+// kind::f8f6f4: fp32 accumulator (bits 4-5 = 1), A and B e4m3 (format 0),
+// both K-major, N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+constexpr uint32_t kIdescF8 = (1u << 4) | (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
+
+constexpr int kBarBytes = 256;
+constexpr size_t kSmemBytes = 1024 + SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 2 * BM * sizeof(float);
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(8 * (2 * SA + 2 * SB + 7) + 8 <= kBarBytes, "barrier area");
+
+__device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(kIdescF8), "r"(accumulate)
+      : "memory");
+}
+
+// acc[j] += s * partial[j] for 16 consecutive TMEM columns
+__device__ __forceinline__ void promote16(float* acc, uint32_t taddr, float s) {
+  uint32_t v[16];
+  tmem_ld16(taddr, v);
+  tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 16; ++j) acc[j] = fmaf(s, __uint_as_float(v[j]), acc[j]);
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    grouped_gemm_fp8_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+                            const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+                            const Fp8Args fa) {
+  const GemmArgs& args = fa.g;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sA = base;
+  const uint32_t sB = base + SA * A_BYTES;
+  uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;
+  const uint32_t bar0 = smem_u32(bar_area);
+  auto fullA = [&](int s) { return bar0 + 8u * s; };
+  auto emptyA = [&](int s) { return bar0 + 8u * (SA + s); };
+  auto fullB = [&](int s) { return bar0 + 8u * (2 * SA + s); };
+  auto emptyB = [&](int s) { return bar0 + 8u * (2 * SA + SB + s); };
+  auto pfull = [&](int b) { return bar0 + 8u * (2 * SA + 2 * SB + b); };
+  auto pempty = [&](int b) { return bar0 + 8u * (2 * SA + 2 * SB + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * SA + 2 * SB + 4);
+  // amax exchange between the two epilogue halves of a row (per tile parity)
+  auto xchg = [&](int b) { return bar0 + 8u * (2 * SA + 2 * SB + 5 + b); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 7));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
+  float* amax_x = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sch) + sizeof(Sched));  // [2][2][BM]
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int G = args.offsets ? args.groups : 1;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int s = 0; s < SA; ++s) {
+        mbar_init(fullA(s), 1);
+        mbar_init(emptyA(s), 1);
+      }
+      for (int s = 0; s < SB; ++s) {
+        mbar_init(fullB(s), 1);
+        mbar_init(emptyB(s), 1);
+      }
+      for (int b = 0; b < 2; ++b) {
+        mbar_init(pfull(b), 1);
+        mbar_init(pempty(b), kEpiWarps * 32);
+      }
+      mbar_init(drain_bar, 1);
+      mbar_init(xchg(0), kEpiWarps * 32);
+      mbar_init(xchg(1), kEpiWarps * 32);
+      *abort_flag = 0;
+      fence_barrier_init();
+      tma_prefetch_desc(&tmA0);
+      tma_prefetch_desc(&tmB0);
+      if (args.m1 > 0) {
+        tma_prefetch_desc(&tmA1);
+        tma_prefetch_desc(&tmB1);
+      }
+    }
+    build_schedule(args, sch, G, lane);
+  } else if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total0 = sch->tile_start[G];
+  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+
+  if ((warp == 0 || warp == kAProdWarp) && lane == 0) {
+    // ------------------------------------------------------------ producers
+    const bool isB = warp == 0;
+    const uint32_t bytes = isB ? B_BYTES : A_BYTES;
+    const uint32_t ring = isB ? sB : sA;
+    const int nst = isB ? SB : SA;
+    const uint64_t pol = l2_policy(isB ? args.hint_b : args.hint_a);
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t pending = 0, issued_phase = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      const CUtensorMap* m = isB ? (T.p1 ? &tmB1 : &tmB0) : (T.p1 ? &tmA1 : &tmA0);
+      const int row = isB ? T.b_row : T.a_row;
+      for (int kb = T.kb0; kb < T.kb1; ++kb) {
+        const uint32_t full = isB ? fullB(stage) : fullA(stage);
+        if (!mbar_wait(isB ? emptyB(stage) : emptyA(stage), phase ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(full, bytes);
+        tma_load_2d(ring + stage * bytes, m, full, kb * BK, row, pol);
+        pending |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == nst) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      record_status(args.status, ST_WAIT_TIMEOUT);
+      int dummy = 0;
+      for (int s = 0; s < nst; ++s)
+        if (pending & (1u << s)) mbar_wait(isB ? fullB(s) : fullA(s), (issued_phase >> s) & 1u, &dummy);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    int sa = 0, sb = 0;
+    uint32_t pa = 0, pb = 0;
+    uint32_t kc = 0;  // K blocks issued by this CTA (partial-buffer ping-pong)
+    bool ok = true, issued = false;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      for (int kb = T.kb0; kb < T.kb1; ++kb, ++kc) {
+        const int buf = kc & 1;
+        if (!mbar_wait(pempty(buf), ((kc >> 1) & 1) ^ 1u, abort_flag) || !mbar_wait(fullA(sa), pa, abort_flag) ||
+            !mbar_wait(fullB(sb), pb, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_addr = sA + sa * A_BYTES;
+        const uint32_t b_addr = sB + sb * B_BYTES;
+        const uint32_t d = tmem_base + buf * BN;
+#pragma unroll
+        for (int kk = 0; kk < BK / 32; ++kk)
+          tc_mma_f8(d, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kk > 0 ? 1u : 0u);
+        issued = true;
+        tc_commit(emptyA(sa));
+        tc_commit(emptyB(sb));
+        tc_commit(pfull(buf));
+        if (++sa == SA) {
+          sa = 0;
+          pa ^= 1u;
+        }
+        if (++sb == SB) {
+          sb = 0;
+          pb ^= 1u;
+        }
+      }
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      record_status(args.status, ST_WAIT_TIMEOUT);
+      if (issued) {
+        int dummy = 0;
+        tc_commit(drain_bar);
+        mbar_wait(drain_bar, 0, &dummy);
+      }
+    }
+  } else if (warp >= 2 && warp < 2 + kEpiWarps) {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int r = q * 32 + lane;
+    const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    uint32_t kc = 0;
+    int it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+      Tile T;
+      decode_tile(t, sch, G, total0, args, T);
+      const int mrows = T.p1 ? args.m1 : args.m0;
+      const long long row = static_cast<long long>(T.a_row) + r;
+      const long long srow = row < mrows ? row : mrows - 1;  // in-bounds scale row for masked rows
+      const float* as = T.p1 ? fa.a_scale1 : fa.a_scale0;
+      const int asld = T.p1 ? fa.a_sld1 : fa.a_sld0;
+      const float* arow = as + srow * asld;
+      const int g = T.group;
+      const int nblk = T.p1 ? fa.b_nblk1 : fa.b_nblk0;
+      const float* bs = (T.p1 ? fa.b_scale1 : fa.b_scale0) + static_cast<long long>(g) * nblk * asld;
+      // scale rows of this thread's columns: SwiGLU tiles hold gate block nt
+      // (scale row 2nt) and up block nt (2nt+1); plain tiles hold blocks 2nt, 2nt+1
+      const float* bs_lo = bs + static_cast<long long>(2 * T.n_tile + (EPI == EPI_SWIGLU ? 0 : half)) * asld;
+      const float* bs_hi = bs + static_cast<long long>(2 * T.n_tile + 1) * asld;
+
+      float acc[128];
+#pragma unroll
+      for (int j = 0; j < 128; ++j) acc[j] = 0.f;
+      for (int kb = T.kb0; kb < T.kb1; ++kb, ++kc) {
+        const int buf = kc & 1;
+        const float sa = __ldg(arow + kb);
+        const float s_lo = sa * __ldg(bs_lo + kb);
+        const float s_hi = EPI == EPI_SWIGLU ? sa * __ldg(bs_hi + kb) : s_lo;
+        if (!__all_sync(0xffffffffu, mbar_wait(pfull(buf), (kc >> 1) & 1, abort_flag))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t pb = lane_addr + buf * BN;
+        if constexpr (EPI == EPI_SWIGLU) {
+          // columns [64h, 64h+64) of the gate half and of the up half
+#pragma unroll
+          for (int c = 0; c < 64; c += 16) promote16(acc + c, pb + half * 64 + c, s_lo);
+#pragma unroll
+          for (int c = 0; c < 64; c += 16) promote16(acc + 64 + c, pb + 128 + half * 64 + c, s_hi);
+        } else {
+#pragma unroll
+          for (int c = 0; c < 128; c += 16) promote16(acc + c, pb + half * 128 + c, s_lo);
+        }
+        tc_fence_before();
+        mbar_arrive(pempty(buf));
+      }
+      if (!ok) break;
+      const bool valid = r < T.rows;
+      if constexpr (EPI == EPI_SWIGLU) {
+        // h = silu(gate) * up for 64 channels, then e4m3 with one scale per
+        // row per 128 channels (this tile's 128 h columns): the two halves of
+        // a row exchange their partial amax through shared memory
+        float amax = 0.f;
+#pragma unroll
+        for (int j = 0; j < 64; ++j) {
+          const float gv = acc[j];
+          const float hv = gv / (1.0f + __expf(-gv)) * acc[64 + j];
+          acc[j] = hv;
+          amax = fmaxf(amax, fabsf(hv));
+        }
+        float* xs = amax_x + (it & 1) * 2 * BM;
+        xs[half * BM + r] = amax;
+        mbar_arrive(xchg(it & 1));
+        if (!__all_sync(0xffffffffu, mbar_wait(xchg(it & 1), (it >> 1) & 1, abort_flag))) {
+          ok = false;
+          break;
+        }
+        amax = fmaxf(amax, xs[(1 - half) * BM + r]);
+        const float scale = amax > 0.f ? amax / 448.0f : 1.0f;
+        if (valid) {
+          uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
+          const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
+          uint8_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * (BN / 2) + half * 64;
+#pragma unroll
+          for (int j = 0; j < 64; j += 16) {
+            uint32_t w4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const __nv_fp8x2_storage_t lo = __nv_cvt_float2_to_fp8x2(
+                  make_float2(acc[j + 4 * u] / scale, acc[j + 4 * u + 1] / scale), __NV_SATFINITE, __NV_E4M3);
+              const __nv_fp8x2_storage_t hi = __nv_cvt_float2_to_fp8x2(
+                  make_float2(acc[j + 4 * u + 2] / scale, acc[j + 4 * u + 3] / scale), __NV_SATFINITE, __NV_E4M3);
+              w4[u] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+            }
+            *reinterpret_cast<uint4*>(dst + j) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          }
+          if (half == 0) {
+            float* os = T.p1 ? fa.out_scale1 : fa.out_scale0;
+            const int osld = T.p1 ? fa.o_sld1 : fa.o_sld0;
+            os[row * osld + T.n_tile] = scale;
+          }
+        }
+      } else {
+        if (valid) {
+          uint16_t* out = static_cast<uint16_t*>(T.p1 ? args.out1 : args.out0);
+          const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
+          uint16_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * BN + half * 128;
+#pragma unroll
+          for (int j = 0; j < 128; j += 8) {
+            *reinterpret_cast<uint4*>(dst + j) =
+                make_uint4(pack_bf16x2(acc[j], acc[j + 1]), pack_bf16x2(acc[j + 2], acc[j + 3]),
+                           pack_bf16x2(acc[j + 4], acc[j + 5]), pack_bf16x2(acc[j + 6], acc[j + 7]));
+          }
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      record_status(args.status, ST_WAIT_TIMEOUT);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn encode_fn() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(p);
+  });
+  return fn;
+}
+
+}  // namespace
+
+cudaError_t fp8_gemm_set_attributes() {
+  cudaError_t e = cudaFuncSetAttribute(grouped_gemm_fp8_kernel<EPI_SWIGLU>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemBytes));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(grouped_gemm_fp8_kernel<EPI_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kSmemBytes));
+  return e;
+}
+
+cudaError_t fp8_gemm_launch(int epi, const CUtensorMap* maps, const Fp8Args& args, int grid, cudaStream_t stream) {
+  if (grid <= 0) return cudaSuccess;
+  if (epi == EPI_SWIGLU)
+    grouped_gemm_fp8_kernel<EPI_SWIGLU><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3],
+                                                                                 args);
+  else
+    grouped_gemm_fp8_kernel<EPI_BF16><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3],
+                                                                               args);
+  return cudaGetLastError();
+}
+
+bool encode_tmap_u8(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                    std::string* err) {
+  EncodeFn fn = encode_fn();
+  if (!fn) {
+    if (err) *err = "cuTensorMapEncodeTiled is not available from the driver";
+    return false;
+  }
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15u) != 0 || cols % 16 != 0 || rows == 0) {
+    if (err) *err = "tensor for TMA must be 16-byte aligned with 16-byte row stride and >= 1 row";
+    return false;
+  }
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    if (err) *err = "cuTensorMapEncodeTiled failed with CUresult " + std::to_string(static_cast<int>(r));
+    return false;
+  }
+  return true;
+}
+
+}  // namespace asap

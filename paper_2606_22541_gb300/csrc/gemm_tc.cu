@@ -24,6 +24,7 @@
 // Rows of a tile past the segment end belong to the next expert (or are
 // zero-filled by TMA past the tensor end) and are masked at the store.
 #include "common.cuh"
+#include "gemm_sched.cuh"
 #include "internal.h"
 
 #include <mutex>
@@ -53,12 +54,6 @@ constexpr int kThreads = 224;  // warp 0 B producer, 1 MMA, 2-5 epilogue, 6 A pr
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
-struct Sched {
-  int tile_start[kMaxExperts + 1];
-  int mtiles[kMaxExperts];
-  int row_base[kMaxExperts];
-  int mrows[kMaxExperts];
-};
 
 constexpr int kBarBytes = 256;  // 2*SA + 2*SB + 5 mbarriers, tmem slot, abort flag
 template <int EPI>
@@ -66,50 +61,7 @@ __host__ __device__ constexpr size_t smem_bytes() {
   return 1024 + Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
 }
 
-struct Tile {
-  int a_row, b_row, rows, n_tile, kb0, kb1, split;
-  bool p1;
-};
 
-__device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int total0,
-                                            const GemmArgs& a, Tile& T) {
-  if (t < total0) {
-    int lo = 0, hi = G;  // largest g with tile_start[g] <= t
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (s->tile_start[mid] <= t) lo = mid; else hi = mid;
-    }
-    const int g = lo;
-    int local = t - s->tile_start[g];
-    const int mt = s->mtiles[g];
-    const int per_split = mt * a.n_tiles0;
-    const int split = local / per_split;   // K slice (split-K of problem 0)
-    local -= split * per_split;
-    const int nt = local / mt;
-    const int mi = local - nt * mt;
-    T.a_row = s->row_base[g] + mi * BM;
-    T.rows = min(BM, s->mrows[g] - mi * BM);
-    T.b_row = g * a.b_stride0 + nt * BN;
-    T.n_tile = nt;
-    T.split = split;
-    T.kb0 = static_cast<int>(static_cast<long long>(a.k_iters0) * split / a.k_splits);
-    T.kb1 = static_cast<int>(static_cast<long long>(a.k_iters0) * (split + 1) / a.k_splits);
-    T.p1 = false;
-  } else {
-    const int u = t - total0;
-    const int mt = (a.m1 + BM - 1) / BM;
-    const int nt = u / mt;
-    const int mi = u - nt * mt;
-    T.a_row = mi * BM;
-    T.rows = min(BM, a.m1 - mi * BM);
-    T.b_row = nt * BN;
-    T.n_tile = nt;
-    T.split = 0;
-    T.kb0 = 0;
-    T.kb1 = a.k_iters1;
-    T.p1 = true;
-  }
-}
 
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr,
@@ -240,49 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(&tmB1);
       }
     }
-    // Per-group m-tile counts and their exclusive prefix (warp scan; each
-    // lane owns up to 8 consecutive groups).  Bad offsets -> empty group.
-    int local = 0;
-    int cnt[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int g = lane * 8 + i;
-      cnt[i] = 0;
-      if (g < G) {
-        int lo = 0, m = args.m0;
-        if (args.offsets) {
-          lo = __ldg(args.offsets + g);
-          const int hi = __ldg(args.offsets + g + 1);
-          m = hi - lo;
-          if (lo < 0 || m < 0 || hi > args.m0) {
-            record_status(args.status, ST_BAD_OFFSETS);
-            lo = 0;
-            m = 0;
-          }
-        }
-        sch->row_base[g] = lo;
-        sch->mrows[g] = m;
-        cnt[i] = (m + BM - 1) / BM;
-        sch->mtiles[g] = cnt[i];
-        local += cnt[i] * args.n_tiles0 * args.k_splits;
-      }
-    }
-    int incl = local;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    int run = incl - local;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int g = lane * 8 + i;
-      if (g < G) {
-        sch->tile_start[g] = run;
-        run += cnt[i] * args.n_tiles0 * args.k_splits;
-      }
-    }
-    if (lane == 31) sch->tile_start[G] = incl;
+    build_schedule(args, sch, G, lane);
   } else if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();

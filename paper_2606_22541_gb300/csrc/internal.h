@@ -55,6 +55,40 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, 
 bool encode_tmap_bf16(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols,
                       uint32_t box_rows, std::string* err);
 
+// ------------------------------------------------------------ FP8 grouped GEMM
+// e4m3 A and B with fp32 block scales: A scales per row per 128-wide K block
+// ([rows][K/128]), B scales per 128 x 128 block ([groups][N/128][K/128]).
+// Per 128-wide K block the tensor core accumulates into one of two TMEM
+// partial buffers; the epilogue warps add each partial, times the row and
+// block scales, into fp32 registers.
+//  EPI_SWIGLU: out = e4m3 h [rows][N/2] (B rows interleaved 128 gate / 128 up
+//              per 256-row tile, B scale rows interleaved gate / up) and
+//              out_scale = per row per 128 channels of h ([rows][N/256]).
+//  EPI_BF16:   out = bf16 [rows][N].
+struct Fp8Args {
+  GemmArgs g;
+  const float* a_scale0;  // [m0][a_sld0]
+  const float* a_scale1;  // [m1][a_sld1]
+  int a_sld0, a_sld1;     // K/128
+  const float* b_scale0;  // [groups][b_nblk0][a_sld0]
+  const float* b_scale1;  // [b_nblk1][a_sld1]
+  int b_nblk0, b_nblk1;   // N/128
+  float* out_scale0;      // EPI_SWIGLU only: [m0][o_sld0]
+  float* out_scale1;
+  int o_sld0, o_sld1;
+};
+constexpr int kFp8BK = 128;  // K elements (bytes) per stage and per scale block
+
+cudaError_t fp8_gemm_set_attributes();
+cudaError_t fp8_gemm_launch(int epi, const CUtensorMap* maps, const Fp8Args& args, int grid, cudaStream_t stream);
+// 2-D row-major byte tensor [rows, cols] for 128-byte-swizzled boxes of [box_rows, 128].
+bool encode_tmap_u8(CUtensorMap* map, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                    std::string* err);
+
+// Rows of bf16 -> e4m3 with one fp32 scale per row per 128 channels
+// (s = amax / 448, q = round-to-nearest-even of v / s, saturated).
+cudaError_t launch_quantize_rows(const void* x, int rows, int cols, void* q, float* s, cudaStream_t st);
+
 // ------------------------------------------------------------ routing
 struct GateParams {
   int n_experts, top_k, gating, n_groups, topk_groups;
@@ -77,11 +111,18 @@ cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* count
 cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
                             const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+// FP8 dispatch: every token row is quantised once (e4m3, fp32 scale per 128
+// channels) and written to its k positions of xq / xs, and to row t of
+// xq_sh / xs_sh when those are non-null (shared expert input).
+cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s);
 cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float* w,
                            const int32_t* perm_dst, int n, int H, int k, void* out,
                            uint32_t* status, cudaStream_t s);
 // packed[e][b*256 + r] = gate[e][b*128 + r] (r < 128), up[...] for r >= 128
-cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, int H, void* packed,
+// Rows are row_bytes wide (H * element size).
+cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, long long row_bytes, void* packed,
                                 cudaStream_t s);
 
 inline int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }

@@ -10,6 +10,8 @@
 #include "common.cuh"
 #include "internal.h"
 
+#include <cuda_fp8.h>
+
 namespace asap {
 
 namespace {
@@ -25,10 +27,36 @@ constexpr int kRankWarps = kChunkTokens * kMaxTopK / 32;  // warps that rank the
 // positions increase with (t, j) inside every segment.  chunk_base is
 // expert-major: chunk_base[e * n_chunks + chunk].  Then one warp per token
 // reads its row once and writes it to its k positions.
+// Quantise 8 consecutive values of a 128-channel block held by 16 lanes
+// (lanes 0-15 one block, 16-31 the next): scale = amax / 448 over the block,
+// q = e4m3(v / scale) with round-to-nearest-even and saturation.
+__device__ __forceinline__ uint2 quantize8(uint4 v, float& scale) {
+  float f[8] = {bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y),
+                bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w)};
+  float am = 0.f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(f[i]));
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, o));
+  scale = am > 0.f ? am / 448.0f : 1.0f;
+  uint32_t w[2];
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const __nv_fp8x2_storage_t lo =
+        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u] / scale, f[4 * u + 1] / scale), __NV_SATFINITE, __NV_E4M3);
+    const __nv_fp8x2_storage_t hi =
+        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u + 2] / scale, f[4 * u + 3] / scale), __NV_SATFINITE, __NV_E4M3);
+    w[u] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+  }
+  return make_uint2(w[0], w[1]);
+}
+
+template <bool FP8>
 __global__ void __launch_bounds__(kDispatchWarps * 32)
     dispatch_kernel(const uint4* __restrict__ x, int n, int V, int k, int E,
                     const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
-                    uint4* __restrict__ x_perm, int32_t* __restrict__ perm_src,
+                    void* __restrict__ x_perm_v, float* __restrict__ xs, uint2* __restrict__ xq_sh,
+                    float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
                     int32_t* __restrict__ perm_dst, uint32_t* status) {
   __shared__ int wcnt[kRankWarps][kMaxExperts];
   __shared__ int spos[kChunkTokens * kMaxTopK];
@@ -86,24 +114,64 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
     int p[kMaxTopK];
 #pragma unroll
     for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[warp * k + j] : -1;
-    int v = lane;
-    for (; v + 32 < V; v += 64) {
-      const uint4 a = __ldg(src + v);
-      const uint4 b = __ldg(src + v + 32);
+    if constexpr (!FP8) {
+      uint4* x_perm = static_cast<uint4*>(x_perm_v);
+      int v = lane;
+      for (; v + 32 < V; v += 64) {
+        const uint4 a = __ldg(src + v);
+        const uint4 b = __ldg(src + v + 32);
 #pragma unroll
-      for (int j = 0; j < kMaxTopK; ++j)
-        if (p[j] >= 0) {
-          uint4* d = x_perm + static_cast<long long>(p[j]) * V;
-          d[v] = a;
-          d[v + 32] = b;
+        for (int j = 0; j < kMaxTopK; ++j)
+          if (p[j] >= 0) {
+            uint4* d = x_perm + static_cast<long long>(p[j]) * V;
+            d[v] = a;
+            d[v + 32] = b;
+          }
+      }
+      for (; v < V; v += 32) {
+        const uint4 a = __ldg(src + v);
+#pragma unroll
+        for (int j = 0; j < kMaxTopK; ++j)
+          if (p[j] >= 0) x_perm[static_cast<long long>(p[j]) * V + v] = a;
+      }
+    } else {
+      // e4m3 rows: V vectors of 8 values -> V 8-byte words; one scale per 16
+      // vectors (128 channels); a warp covers two blocks per step
+      uint2* xq = static_cast<uint2*>(x_perm_v);
+      const int nb = V / 16;
+      const long long t = t0 + warp;
+      for (int v = lane; v < V; v += 32) {
+        float scale;
+        const uint2 q = quantize8(__ldg(src + v), scale);
+        const int blk = v >> 4;
+        const bool head = (lane & 15) == 0;
+#pragma unroll
+        for (int j = 0; j < kMaxTopK; ++j)
+          if (p[j] >= 0) {
+            xq[static_cast<long long>(p[j]) * V + v] = q;
+            if (head) xs[static_cast<long long>(p[j]) * nb + blk] = scale;
+          }
+        if (xq_sh) {
+          xq_sh[t * V + v] = q;
+          if (head) xs_sh[t * nb + blk] = scale;
         }
+      }
     }
-    for (; v < V; v += 32) {
-      const uint4 a = __ldg(src + v);
-#pragma unroll
-      for (int j = 0; j < kMaxTopK; ++j)
-        if (p[j] >= 0) x_perm[static_cast<long long>(p[j]) * V + v] = a;
-    }
+  }
+}
+
+// Rows of bf16 to e4m3 with a scale per 128 channels; one warp per row.
+__global__ void __launch_bounds__(256) quantize_rows_kernel(const uint4* __restrict__ x, int rows, int V,
+                                                            uint2* __restrict__ q, float* __restrict__ s) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long r = static_cast<long long>(blockIdx.x) * 8 + warp;
+  if (r >= rows) return;
+  const int nb = V / 16;
+  for (int v = lane; v < V; v += 32) {
+    float scale;
+    const uint2 w = quantize8(__ldg(x + r * V + v), scale);
+    q[r * V + v] = w;
+    if ((lane & 15) == 0) s[r * nb + (v >> 4)] = scale;
   }
 }
 
@@ -200,9 +268,27 @@ cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
-  dispatch_kernel<<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
-                                                         chunk_base, chunks, static_cast<uint4*>(x_perm), perm_src,
-                                                         perm_dst, status);
+  dispatch_kernel<false><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
+                                                                chunk_base, chunks, x_perm, nullptr, nullptr, nullptr,
+                                                                perm_src, perm_dst, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int chunks = ceil_div(n, kChunkTokens);
+  dispatch_kernel<true><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
+                                                               chunk_base, chunks, xq, xs, static_cast<uint2*>(xq_sh),
+                                                               xs_sh, perm_src, perm_dst, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_rows(const void* x, int rows, int cols, void* q, float* s, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  quantize_rows_kernel<<<ceil_div(rows, 8), 256, 0, st>>>(static_cast<const uint4*>(x), rows, cols / 8,
+                                                          static_cast<uint2*>(q), s);
   return cudaGetLastError();
 }
 
@@ -216,10 +302,10 @@ cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, int H, void* packed,
+cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, long long row_bytes, void* packed,
                                 cudaStream_t s) {
   pack_gate_up_kernel<<<4096, 256, 0, s>>>(static_cast<const uint4*>(gate), static_cast<const uint4*>(up), E, I,
-                                           H / 8, static_cast<uint4*>(packed));
+                                           static_cast<int>(row_bytes / 16), static_cast<uint4*>(packed));
   return cudaGetLastError();
 }
 

@@ -43,10 +43,7 @@ def test_library_exports_every_declared_symbol(L):
 def test_check_config(L):
     for c in CONFIGS.values():
         code = api.asap_moe_check_config(c, 4096)
-        if c.dtype == "bf16":
-            assert code == _native.ASAP_OK, api.asap_moe_last_error()
-        else:
-            assert code == _native.ASAP_ERR_UNSUPPORTED
+        assert code == _native.ASAP_OK, api.asap_moe_last_error()
     from dataclasses import replace
     bad = [replace(TINY, hidden=200), replace(TINY, top_k=9), replace(TINY, inter=100),
            replace(DSV3, n_groups=7), replace(DSV3, topk_groups=0), replace(TINY, n_experts=300),
@@ -54,6 +51,15 @@ def test_check_config(L):
     for b in bad:
         assert api.asap_moe_check_config(b, 16) == _native.ASAP_ERR_INVALID
     assert api.asap_moe_check_config(TINY, 0) == _native.ASAP_ERR_INVALID
+
+
+def test_workspace_size_fp8(L):
+    from paper_2606_22541_gb300.configs import DSV3_FP8
+    a = api.asap_moe_workspace_size(DSV3_FP8, 4096)
+    b = api.asap_moe_workspace_size(DSV3, 4096)
+    # e4m3 rows of x and h plus bf16 expert outputs
+    assert a > 4096 * 8 * (7168 + 2048 + 7168 * 2)
+    assert a != b
 
 
 def test_workspace_size(L):

@@ -1,0 +1,197 @@
+"""FP8 configuration (e4m3 expert weights with fp32 128 x 128 block scales,
+e4m3 activations per token per 128 channels) through the C ABI against the
+float64 oracle, which emulates the activation quantisation."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_22541_gb300 import api, inputs
+from paper_2606_22541_gb300.configs import DSV3_FP8
+
+from _helpers import bf16_to_f64, routing_check
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+REL_NORM_FP8 = 3e-2
+F8_SMALL = inputs.small_variant(DSV3_FP8, name="fp8_small", hidden=512, inter=256, shared_inter=256,
+                                microbatches=[300, 77])
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def e4m3_to_f64(t):
+    return oracle.e4m3_bits_to_f64(t.detach().contiguous().view(torch.uint8).cpu().numpy())
+
+
+def dequant_expert(w, e):
+    """Float64 weights of routed expert e, decoded by the oracle."""
+    return (oracle.dequant_blocks(e4m3_to_f64(w["w_gate"][e]), w["s_gate"][e].cpu().numpy()),
+            oracle.dequant_blocks(e4m3_to_f64(w["w_up"][e]), w["s_up"][e].cpu().numpy()),
+            oracle.dequant_blocks(e4m3_to_f64(w["w_down"][e]), w["s_down"][e].cpu().numpy()))
+
+
+def shared_expert(w):
+    return (oracle.dequant_blocks(e4m3_to_f64(w["sh_gate"]), w["sh_s_gate"].cpu().numpy()),
+            oracle.dequant_blocks(e4m3_to_f64(w["sh_up"]), w["sh_s_up"].cpu().numpy()),
+            oracle.dequant_blocks(e4m3_to_f64(w["sh_down"]), w["sh_s_down"].cpu().numpy()))
+
+
+def compare_fp8(g, r):
+    g = np.asarray(g, np.float64)
+    r = np.asarray(r, np.float64)
+    norm = float(np.linalg.norm(g - r) / np.linalg.norm(r))
+    rms = np.sqrt(np.mean(r * r, axis=-1, keepdims=True))
+    worst = float((np.abs(g - r) / np.maximum(np.abs(r), rms)).max())
+    assert norm <= REL_NORM_FP8, f"normwise {norm:.3e}"
+    assert worst <= 0.5, f"elementwise {worst:.3e}"   # gross-error guard; the fp8 bound is normwise
+    return norm, worst
+
+
+@pytest.fixture(scope="module")
+def small():
+    w = inputs.make_weights(F8_SMALL, DEV)
+    h = api.asap_moe_create(F8_SMALL, w, max(F8_SMALL.microbatches))
+    yield w, h
+    h.close()
+
+
+def test_dispatch_quantises_like_the_oracle(small):
+    w, h = small
+    cfg = F8_SMALL
+    n, k, E, H = 300, cfg.top_k, cfg.n_experts, cfg.hidden
+    x = inputs.make_tokens(cfg, n, 0, DEV)
+    rng = np.random.default_rng(3)
+    idx_np = np.array([rng.permutation(E)[:k] for _ in range(n)], np.int64)
+    xq = torch.empty((n * k, H), dtype=torch.uint8, device=DEV)
+    xs = torch.empty((n * k, H // 128), dtype=torch.float32, device=DEV)
+    ps = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    pd = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(h, x, torch.tensor(idx_np, dtype=torch.int32, device=DEV), xq, ps, pd,
+                          api.workspace(h, n), x_perm_scales=xs)
+    torch.cuda.synchronize()
+    src, dst = oracle.permutation(idx_np, E)
+    assert np.array_equal(ps.cpu().numpy(), src)
+    q_ref, s_ref = oracle.quantize_rows_e4m3(oracle.dispatch(bf16_to_f64(x), src))
+    q = e4m3_to_f64(xq)
+    s = xs.cpu().numpy().astype(np.float64)
+    assert np.allclose(s, s_ref, rtol=1e-6, atol=0)
+    diff = q != q_ref
+    assert diff.mean() < 1e-3, diff.mean()
+    # where the float32 and float64 quotients straddle a rounding boundary,
+    # the two picks are neighbouring e4m3 values
+    assert np.all(np.abs(q[diff] - q_ref[diff]) <= np.abs(q_ref[diff]) * 2.0 ** -3 + 2.0 ** -9)
+
+
+def test_fp8_layer_matches_oracle(small):
+    w, h = small
+    cfg = F8_SMALL
+    ocfg = cfg.oracle_cfg()
+    wr = bf16_to_f64(w["router_w"])
+    shared = shared_expert(w)
+    cache = {}
+
+    def get_expert(e):
+        if e not in cache:
+            cache[e] = dequant_expert(w, e)
+        return cache[e]
+
+    for i, n in enumerate(cfg.microbatches):
+        x = inputs.make_tokens(cfg, n, i, DEV)
+        out = torch.empty_like(x)
+        api.asap_moe_layer(h, x, out, api.workspace(h, n))
+        torch.cuda.synchronize()
+        xf = bf16_to_f64(x)
+        L = oracle.router_logits(xf, wr)
+        idx_ref, w_ref = oracle.route(L, ocfg)
+        eps = oracle.logit_error_bound(xf, wr)
+        dec = np.array([oracle.token_decided(L[t], eps[t], ocfg) for t in range(n)])
+        ref = np.zeros((n, cfg.hidden))
+        for t in np.nonzero(dec)[0]:
+            wg, wu, wd = zip(*[get_expert(int(e)) for e in idx_ref[t]])
+            ref[t] = oracle.moe_layer_tokens_fp8(xf[t:t + 1], np.arange(cfg.top_k)[None], w_ref[t:t + 1],
+                                                 list(wg), list(wu), list(wd), shared)[0]
+        compare_fp8(bf16_to_f64(out)[dec], ref[dec])
+    code, word = api.asap_moe_status(h)
+    assert code == 0 and word == 0
+
+
+def test_fp8_expert_ffn_equals_layer_bits(small):
+    w, h = small
+    cfg = F8_SMALL
+    n, k, E, H = 300, cfg.top_k, cfg.n_experts, cfg.hidden
+    x = inputs.make_tokens(cfg, n, 0, DEV)
+    ws = api.workspace(h, n)
+    out = torch.empty_like(x)
+    api.asap_moe_layer(h, x, out, ws)
+    idx = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    wt = torch.empty((n, k), dtype=torch.float32, device=DEV)
+    counts = torch.empty(E, dtype=torch.int32, device=DEV)
+    offs = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+    api.asap_moe_route(h, x, idx, wt, counts, offs, ws)
+    xq = torch.empty((n * k, H), dtype=torch.uint8, device=DEV)
+    xs = torch.empty((n * k, H // 128), dtype=torch.float32, device=DEV)
+    ps = torch.empty(n * k, dtype=torch.int32, device=DEV)
+    pd = torch.empty((n, k), dtype=torch.int32, device=DEV)
+    api.asap_moe_dispatch(h, x, idx, xq, ps, pd, ws, x_perm_scales=xs)
+    y = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+    ysh = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+    api.asap_moe_expert_ffn(h, xq, offs, x, y, ysh, ws, x_perm_scales=xs)
+    out2 = torch.empty_like(x)
+    api.asap_moe_combine(h, y, ysh, wt, pd, out2)
+    torch.cuda.synchronize()
+    assert torch.equal(out.view(torch.int16), out2.view(torch.int16))
+
+
+def test_fp8_full_size_streams_against_oracle():
+    cfg = DSV3_FP8
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
+    xs = inputs.make_microbatches(cfg, DEV)
+    wss = [api.workspace(h, x.shape[0]) for x in xs]
+    streams = [torch.cuda.Stream() for _ in xs]
+    outs = [torch.empty_like(x) for x in xs]
+    torch.cuda.synchronize()
+    for x, o, ws, s in zip(xs, outs, wss, streams):
+        api.asap_moe_layer(h, x, o, ws, stream=s)
+    torch.cuda.synchronize()
+    ocfg = cfg.oracle_cfg()
+    wr = bf16_to_f64(w["router_w"])
+    shared = shared_expert(w)
+    rng = np.random.default_rng(cfg.seed)
+    xs_s, idx_s, w_s, g_s = [], [], [], []
+    for i, x in enumerate(xs[:4]):
+        n, k, E = x.shape[0], cfg.top_k, cfg.n_experts
+        idx = torch.empty((n, k), dtype=torch.int32, device=DEV)
+        wt = torch.empty((n, k), dtype=torch.float32, device=DEV)
+        counts = torch.empty(E, dtype=torch.int32, device=DEV)
+        offs = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+        api.asap_moe_route(h, x, idx, wt, counts, offs, wss[i])
+        torch.cuda.synchronize()
+        xf = bf16_to_f64(x)
+        L = oracle.router_logits(xf, wr)
+        eps = oracle.logit_error_bound(xf, wr)
+        idx_ref, w_ref = oracle.route(L, ocfg)
+        dec = routing_check(L, eps, ocfg, idx.cpu().numpy().astype(np.int64),
+                            wt.cpu().numpy().astype(np.float64), w_ref, idx_ref)
+        pick = rng.choice(np.nonzero(dec)[0], 2, replace=False)
+        xs_s.append(xf[pick]); idx_s.append(idx_ref[pick]); w_s.append(w_ref[pick])
+        g_s.append(bf16_to_f64(outs[i])[pick])
+    x_s, idx_a, w_a, g = map(np.concatenate, (xs_s, idx_s, w_s, g_s))
+    ref = np.zeros_like(x_s)
+    for e in np.unique(idx_a):
+        rows, slots = np.nonzero(idx_a == e)
+        wg, wu, wd = dequant_expert(w, int(e))
+        for r_, s_ in zip(rows, slots):
+            ref[r_] += w_a[r_, s_] * oracle.swiglu_fp8(x_s[r_:r_ + 1], wg, wu, wd)[0]
+    for r_ in range(len(ref)):
+        ref[r_] += oracle.swiglu_fp8(x_s[r_:r_ + 1], *shared)[0]
+    compare_fp8(g, ref)
+    code, word = api.asap_moe_status(h)
+    assert code == 0 and word == 0
+    h.close()
