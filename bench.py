@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--cpu-sample-tokens", type=int, default=6)
     ap.add_argument("--microbatches", default=None,
                     help="comma-separated micro-batch sizes overriding the workload's")
+    ap.add_argument("--measure-fp8-peak", action="store_true",
+                    help="print the dense e4m3 matmul peak (torch._scaled_mm 8192^3, best of 10) and exit")
     return ap.parse_args()
 
 
@@ -233,7 +235,8 @@ GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb30
 
 
 def weight_gb(cfg):
-    return (cfg.n_experts * 3 * cfg.hidden * cfg.inter + cfg.n_shared * 3 * cfg.hidden * cfg.shared_inter) * 2 / 1e9
+    eb = 2 if cfg.dtype == "bf16" else 1
+    return (cfg.n_experts * 3 * cfg.hidden * cfg.inter + cfg.n_shared * 3 * cfg.hidden * cfg.shared_inter) * eb / 1e9
 
 
 def load_peaks():
@@ -332,7 +335,12 @@ def run_ours(args, dist):
     kern = kernel_pass(args, h, cfg, xs, dev)
     peaks, peaks_src = load_peaks()
     result["kernels"] = kern["table"]
-    result["roofline"] = roofline(kern, peaks, peaks_src)
+    tensor_peak = None
+    if cfg.dtype != "bf16":
+        # e4m3 tensor peak: the measured bf16 figure times the nominal fp8/bf16 ratio (4.5 / 2.25)
+        tensor_peak = 2.0 * peaks["bf16_tflops_sustained"]
+        result["dtype"] = "e4m3 (fp32 accumulate, bf16 out)"
+    result["roofline"] = roofline(kern, peaks, peaks_src, tensor_peak)
     gemm_flops = kern["gemm_flops"]
     gemm_ms = kern["gemm_ms"]
     result["grouped_gemm_tensor_frac"] = {
@@ -379,30 +387,42 @@ def kernel_pass(args, h, cfg, xs, dev):
     y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
     out = torch.empty((n, H), dtype=torch.bfloat16, device=dev)
     ws = api.workspace(h, n, dev)
+    fp8 = cfg.dtype != "bf16"
     names = ["router_gemm", "gate_scan", "dispatch", "gemm_gate_up_swiglu", "gemm_down", "combine"]
+    if fp8:
+        names = ["router_gemm", "gate_scan", "dispatch", "expert_ffn_fp8", "combine"]
+        x_perm = torch.empty((n * k, H), dtype=torch.uint8, device=dev)
+        xsc = torch.empty((n * k, H // 128), dtype=torch.float32, device=dev)
     times = {nm: [] for nm in names}
     active = []   # experts with tokens, per micro-batch (for the weight bytes)
     for it in range(args.kernel_steps + 1):
         rec = []
         for x in xs:
             m = x.shape[0]
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
             ev[0].record(s)
             api.asap_moe_router_logits(h, x, logits[:m], ws, stream=s)
             ev[1].record(s)
             api.asap_moe_route_logits(h, logits[:m], idx[:m], w[:m], counts, offsets, ws, stream=s)
             ev[2].record(s)
-            api.asap_moe_dispatch(h, x, idx[:m], x_perm[:m * k], perm_src[:m * k], perm_dst[:m], ws, stream=s)
+            api.asap_moe_dispatch(h, x, idx[:m], x_perm[:m * k], perm_src[:m * k], perm_dst[:m], ws, stream=s,
+                                  x_perm_scales=xsc[:m * k] if fp8 else None)
             ev[3].record(s)
-            api.asap_moe_expert_gate_up(h, x_perm[:m * k], offsets, x, hbuf[:m * k],
-                                        hsh[:m] if hsh is not None else None, stream=s)
-            ev[4].record(s)
-            api.asap_moe_expert_down(h, hbuf[:m * k], offsets, hsh[:m] if hsh is not None else None, m,
-                                     y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s)
-            ev[5].record(s)
+            if fp8:
+                api.asap_moe_expert_ffn(h, x_perm[:m * k], offsets, x, y_perm[:m * k],
+                                        y_sh[:m] if y_sh is not None else None, ws, stream=s,
+                                        x_perm_scales=xsc[:m * k])
+                ev[4].record(s)
+            else:
+                api.asap_moe_expert_gate_up(h, x_perm[:m * k], offsets, x, hbuf[:m * k],
+                                            hsh[:m] if hsh is not None else None, stream=s)
+                ev[4].record(s)
+                api.asap_moe_expert_down(h, hbuf[:m * k], offsets, hsh[:m] if hsh is not None else None, m,
+                                         y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s)
+                ev[5].record(s)
             api.asap_moe_combine(h, y_perm[:m * k], y_sh[:m] if y_sh is not None else None, w[:m], perm_dst[:m],
                                  out[:m], stream=s)
-            ev[6].record(s)
+            ev[len(names)].record(s)
             rec.append(ev)
             if it == 0:
                 torch.cuda.synchronize()
@@ -419,21 +439,31 @@ def kernel_pass(args, h, cfg, xs, dev):
     nk = m * k
     mean_active = sum(active) / len(active)
     # algorithmic bytes / FLOPs per launch (one micro-batch of m tokens)
-    wb = 2  # bf16
+    wb = 2  # bf16 activations
+    eb = 1 if fp8 else 2  # expert-weight element bytes
     alg = {
         "router_gemm": dict(bytes=m * H * wb + E * H * wb + m * E * 4, flops=2.0 * m * H * E),
         "gate_scan": dict(bytes=m * E * 4 + nk * 8, flops=0.0),
         "dispatch": dict(bytes=m * H * wb + nk * H * wb + nk * 12, flops=0.0),
         "gemm_gate_up_swiglu": dict(
-            bytes=mean_active * 2 * I * H * wb + (2 * Is * H * wb if cfg.n_shared else 0)
+            bytes=mean_active * 2 * I * H * eb + (2 * Is * H * eb if cfg.n_shared else 0)
             + nk * H * wb + (m * H * wb if cfg.n_shared else 0) + nk * I * wb + (m * Is * wb if cfg.n_shared else 0),
             flops=2.0 * nk * H * 2 * I + (2.0 * m * H * 2 * Is if cfg.n_shared else 0.0)),
         "gemm_down": dict(
-            bytes=mean_active * H * I * wb + (H * Is * wb if cfg.n_shared else 0)
+            bytes=mean_active * H * I * eb + (H * Is * eb if cfg.n_shared else 0)
             + nk * I * wb + (m * Is * wb if cfg.n_shared else 0) + nk * H * wb + (m * H * wb if cfg.n_shared else 0),
             flops=2.0 * nk * I * H + (2.0 * m * Is * H if cfg.n_shared else 0.0)),
         "combine": dict(bytes=nk * H * wb + (m * H * wb if cfg.n_shared else 0) + m * H * wb + nk * 8, flops=0.0),
     }
+    if fp8:
+        # e4m3 activations (x_perm, h) and bf16 outputs
+        alg["dispatch"] = dict(bytes=m * H * wb + nk * H + nk * (H // 128) * 4 + nk * 12, flops=0.0)
+        g1 = alg["gemm_gate_up_swiglu"]
+        g2 = alg["gemm_down"]
+        alg["expert_ffn_fp8"] = dict(
+            bytes=mean_active * 3 * I * H + (3 * Is * H if cfg.n_shared else 0) + nk * H + 2 * nk * I
+            + (m * H * 2 + m * H + 2 * m * Is if cfg.n_shared else 0) + nk * H * 2 + (m * H * 2 if cfg.n_shared else 0),
+            flops=g1["flops"] + g2["flops"])
     table = {}
     for nm in names:
         sec = avg[nm] / 1e3
@@ -443,21 +473,22 @@ def kernel_pass(args, h, cfg, xs, dev):
     for nm in names:
         table[nm]["share"] = avg[nm] / total_ms
     gemm_flops = alg["gemm_gate_up_swiglu"]["flops"] + alg["gemm_down"]["flops"]
-    gemm_ms = avg["gemm_gate_up_swiglu"] + avg["gemm_down"]
+    gemm_ms = avg["expert_ffn_fp8"] if fp8 else avg["gemm_gate_up_swiglu"] + avg["gemm_down"]
     return {"table": table, "avg": avg, "alg": alg, "gemm_flops": gemm_flops, "gemm_ms": gemm_ms,
             "active_experts": mean_active, "serial_ms_per_microbatch": total_ms}
 
 
-def roofline(kern, peaks, peaks_src):
+def roofline(kern, peaks, peaks_src, tensor_peak=None):
     nm = max(kern["avg"], key=kern["avg"].get)
     a = kern["alg"][nm]
     sec = kern["avg"][nm] / 1e3
+    tpk = tensor_peak or peaks["bf16_tflops_sustained"]
     t_hbm = a["bytes"] / (peaks["hbm_gbs"] * 1e9)
-    t_tc = a["flops"] / (peaks["bf16_tflops_sustained"] * 1e12) if a["flops"] else 0.0
+    t_tc = a["flops"] / (tpk * 1e12) if a["flops"] else 0.0
     traffic, src = profile_traffic("gemm_gate_up_swiglu_dsv3.md", GEMM_SOURCES) if nm.startswith("gemm") else (None, None)
     if t_tc >= t_hbm:
         achieved = a["flops"] / sec / 1e12
-        peak = peaks["bf16_tflops_sustained"]
+        peak = tpk
         r = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak}
     else:
         achieved = a["bytes"] / sec / 1e9
@@ -467,8 +498,7 @@ def roofline(kern, peaks, peaks_src):
               "alg_flops_per_launch": a["flops"], "avg_launch_ms": kern["avg"][nm],
               "peak_source": f"{peaks_src} ({'sustained bf16 tensor' if r['bound'] == 'tensor' else 'HBM copy'})",
               "hbm_frac_of_measured": a["bytes"] / sec / 1e9 / peaks["hbm_gbs"],
-              "tensor_frac_of_sustained_measured": (a["flops"] / sec / 1e12 / peaks["bf16_tflops_sustained"])
-              if a["flops"] else None,
+              "tensor_frac_of_sustained_measured": (a["flops"] / sec / 1e12 / tpk) if a["flops"] else None,
               "traffic_source": src})
     return r
 
@@ -547,8 +577,33 @@ def run_reference(args, dist):
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def measure_fp8_peak():
+    """Dense e4m3 matmul throughput: torch._scaled_mm at 8192^3, best of 10."""
+    import torch
+    n = 8192
+    a = torch.randn(n, n, device="cuda").to(torch.float8_e4m3fn)
+    b = torch.randn(n, n, device="cuda").to(torch.float8_e4m3fn).t()
+    one = torch.ones((), device="cuda")
+    for _ in range(3):
+        torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+    best = 1e9
+    for _ in range(10):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+        e1.record()
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    return {"fp8_e4m3_tflops": 2.0 * n ** 3 / (best / 1e3) / 1e12, "ms": best, "n": n,
+            "how": "torch._scaled_mm e4m3 x e4m3 -> bf16, 8192^3, best of 10, CUDA events"}
+
+
 def main():
     args = parse_args()
+    if args.measure_fp8_peak:
+        print(json.dumps(measure_fp8_peak()), flush=True)
+        return
     dist = Dist()
     if args.impl == "reference":
         if dist.rank == 0:

@@ -95,4 +95,8 @@ DSV3_E32 = LayerConfig("dsv3_e32_profile", hidden=7168, n_experts=32, top_k=8, i
                        shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
                        route_scale=2.5, microbatches=[512], seed=1002)
 
-CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32)}
+DSV3_FP8_E32 = LayerConfig("dsv3_fp8_e32_profile", hidden=7168, n_experts=32, top_k=8, inter=2048, n_shared=1,
+                           shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                           route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[512], seed=1004)
+
+CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32, DSV3_FP8_E32)}

@@ -6,17 +6,18 @@
 // 128 channels.  The scales are arbitrary fp32 values, so they cannot ride
 // in the tensor core's power-of-two block-scale path; instead every 128-wide
 // K block is multiplied into one of two TMEM partial buffers (ping-pong) and
-// eight epilogue warps add it, times (row scale x block scale), into fp32
+// the epilogue warps add it, times (row scale x block scale), into fp32
 // register accumulators while the tensor core already works on the next
-// block.
+// block.  The per-row and per-block scales of the next two K blocks are
+// loaded ahead, so their L2 latency stays off the promotion path.
 //
 // Roles (one CTA per SM, persistent, 352 threads):
 //   warp 0    : weight producer, boxes [256 rows, 128 B], 4-stage ring
-//   warp 10   : activation producer, boxes [128 rows, 128 B], 4-stage ring
+//   last warp : activation producer, boxes [128 rows, 128 B], 4-stage ring
 //   warp 1    : TMEM allocator (512 columns) and MMA issuer: per K block
 //               4 x tcgen05.mma.cta_group::1.kind::f8f6f4 M=128 N=256 K=32
-//   warps 2-9 : epilogue; warp w owns TMEM lanes 32*(w%4).. and, with
-//               h = (w-2)/4, one half of the 256 columns of a tile
+//   epilogue  : 8 warps; warp w owns TMEM lanes 32*(w%4).. and, with
+//               cq = (w-2)/4, one half of the 256 columns of a tile
 // Tile schedule, masking and bounded waits as in the bf16 kernel.
 #include "common.cuh"
 #include "gemm_sched.cuh"
@@ -34,16 +35,21 @@ constexpr int BM = kGemmBM, BN = kGemmBN, BK = kFp8BK;
 constexpr int SA = 4, SB = 4;
 constexpr int A_BYTES = BM * BK;  // 16 KB
 constexpr int B_BYTES = BN * BK;  // 32 KB
-constexpr int kEpiWarps = 8;
-constexpr int kThreads = 32 * (3 + kEpiWarps);  // 352
-constexpr int kAProdWarp = 2 + kEpiWarps;      // 10
+#ifndef ASAP_FP8_EPI_WARPS
+#define ASAP_FP8_EPI_WARPS 8
+#endif
+constexpr int kEpiWarps = ASAP_FP8_EPI_WARPS;   // 8 or 16: 2 or 4 per TMEM lane quarter
+constexpr int kColGroups = kEpiWarps / 4;       // column groups per row
+constexpr int kCols = BN / kColGroups;          // accumulator columns per thread
+constexpr int kThreads = 32 * (3 + kEpiWarps);
+constexpr int kAProdWarp = 2 + kEpiWarps;
 constexpr uint32_t kTmemCols = 2 * BN;          // two partial buffers
 // kind::f8f6f4: fp32 accumulator (bits 4-5 = 1), A and B e4m3 (format 0),
 // both K-major, N >> 3 in bits 17-22, M >> 4 in bits 24-28.
 constexpr uint32_t kIdescF8 = (1u << 4) | (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
 
 constexpr int kBarBytes = 256;
-constexpr size_t kSmemBytes = 1024 + SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 2 * BM * sizeof(float);
+constexpr size_t kSmemBytes = 1024 + SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 4 * BM * sizeof(float);
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(8 * (2 * SA + 2 * SB + 7) + 8 <= kBarBytes, "barrier area");
 
@@ -56,13 +62,27 @@ __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t adesc, uint6
       : "memory");
 }
 
-// acc[j] += s * partial[j] for 16 consecutive TMEM columns
-__device__ __forceinline__ void promote16(float* acc, uint32_t taddr, float s) {
-  uint32_t v[16];
-  tmem_ld16(taddr, v);
-  tmem_ld_wait();
+#ifndef ASAP_FP8_PROMOTE
+#define ASAP_FP8_PROMOTE 16
+#endif
+// acc[j] += s * partial[j] for 32 consecutive TMEM columns
+__device__ __forceinline__ void promote32(float* acc, uint32_t taddr, float s) {
+  if constexpr (ASAP_FP8_PROMOTE == 32) {
+    uint32_t v[32];
+    tmem_ld32(taddr, v);
+    tmem_ld_wait();
 #pragma unroll
-  for (int j = 0; j < 16; ++j) acc[j] = fmaf(s, __uint_as_float(v[j]), acc[j]);
+    for (int j = 0; j < 32; ++j) acc[j] = fmaf(s, __uint_as_float(v[j]), acc[j]);
+  } else {
+#pragma unroll
+    for (int c = 0; c < 32; c += 16) {
+      uint32_t v[16];
+      tmem_ld16(taddr + c, v);
+      tmem_ld_wait();
+#pragma unroll
+      for (int j = 0; j < 16; ++j) acc[c + j] = fmaf(s, __uint_as_float(v[j]), acc[c + j]);
+    }
+  }
 }
 
 template <int EPI>
@@ -91,7 +111,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 7));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
-  float* amax_x = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sch) + sizeof(Sched));  // [2][2][BM]
+  float* amax_x = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sch) + sizeof(Sched));  // [2][4][BM]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -222,8 +242,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 2 && warp < 2 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
+    // warp w reads TMEM lanes 32*(w%4).. (rows) and column quarter cq:
+    // SwiGLU tiles: gate columns [32cq, 32cq+32) and the matching up columns
+    // 128 + [32cq, 32cq+32), i.e. h channels [32cq, 32cq+32) of the tile;
+    // plain tiles: columns [64cq, 64cq+64).
     const int q = warp & 3;
-    const int half = (warp - 2) >> 2;
+    const int cq = (warp - 2) >> 2;  // column group
     const int r = q * 32 + lane;
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
     uint32_t kc = 0;
@@ -235,25 +259,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int mrows = T.p1 ? args.m1 : args.m0;
       const long long row = static_cast<long long>(T.a_row) + r;
       const long long srow = row < mrows ? row : mrows - 1;  // in-bounds scale row for masked rows
-      const float* as = T.p1 ? fa.a_scale1 : fa.a_scale0;
       const int asld = T.p1 ? fa.a_sld1 : fa.a_sld0;
-      const float* arow = as + srow * asld;
-      const int g = T.group;
+      const float* arow = (T.p1 ? fa.a_scale1 : fa.a_scale0) + srow * asld;
       const int nblk = T.p1 ? fa.b_nblk1 : fa.b_nblk0;
-      const float* bs = (T.p1 ? fa.b_scale1 : fa.b_scale0) + static_cast<long long>(g) * nblk * asld;
-      // scale rows of this thread's columns: SwiGLU tiles hold gate block nt
-      // (scale row 2nt) and up block nt (2nt+1); plain tiles hold blocks 2nt, 2nt+1
-      const float* bs_lo = bs + static_cast<long long>(2 * T.n_tile + (EPI == EPI_SWIGLU ? 0 : half)) * asld;
+      const float* bs = (T.p1 ? fa.b_scale1 : fa.b_scale0) + static_cast<long long>(T.group) * nblk * asld;
+      // scale rows of this warp's columns: SwiGLU tiles hold gate block nt
+      // (scale row 2nt) and up block nt (2nt+1); plain tiles blocks 2nt, 2nt+1
+      const int lo_blk = EPI == EPI_SWIGLU ? 0 : (cq * kCols) / 128;
+      const float* bs_lo = bs + static_cast<long long>(2 * T.n_tile + lo_blk) * asld;
       const float* bs_hi = bs + static_cast<long long>(2 * T.n_tile + 1) * asld;
+      // scales of the next two K blocks are loaded ahead (L2 latency)
+      auto ld_scales = [&](int kb, float& a, float& bl, float& bh) {
+        if (kb < T.kb1) {
+          a = __ldg(arow + kb);
+          bl = __ldg(bs_lo + kb);
+          bh = EPI == EPI_SWIGLU ? __ldg(bs_hi + kb) : 0.f;
+        }
+      };
+      float a0 = 0.f, l0 = 0.f, h0 = 0.f, a1 = 0.f, l1 = 0.f, h1 = 0.f;
+      ld_scales(T.kb0, a0, l0, h0);
+      ld_scales(T.kb0 + 1, a1, l1, h1);
 
-      float acc[128];
+      float acc[kCols];
 #pragma unroll
-      for (int j = 0; j < 128; ++j) acc[j] = 0.f;
+      for (int j = 0; j < kCols; ++j) acc[j] = 0.f;
       for (int kb = T.kb0; kb < T.kb1; ++kb, ++kc) {
         const int buf = kc & 1;
-        const float sa = __ldg(arow + kb);
-        const float s_lo = sa * __ldg(bs_lo + kb);
-        const float s_hi = EPI == EPI_SWIGLU ? sa * __ldg(bs_hi + kb) : s_lo;
+        const float s_lo = a0 * l0;
+        const float s_hi = a0 * h0;
+        a0 = a1;
+        l0 = l1;
+        h0 = h1;
+        ld_scales(kb + 2, a1, l1, h1);
         if (!__all_sync(0xffffffffu, mbar_wait(pfull(buf), (kc >> 1) & 1, abort_flag))) {
           ok = false;
           break;
@@ -261,14 +298,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t pb = lane_addr + buf * BN;
         if constexpr (EPI == EPI_SWIGLU) {
-          // columns [64h, 64h+64) of the gate half and of the up half
+          // h channels [cq*kCols/2, +kCols/2): gate columns, then the matching up columns
 #pragma unroll
-          for (int c = 0; c < 64; c += 16) promote16(acc + c, pb + half * 64 + c, s_lo);
+          for (int c = 0; c < kCols / 2; c += 32) promote32(acc + c, pb + cq * (kCols / 2) + c, s_lo);
 #pragma unroll
-          for (int c = 0; c < 64; c += 16) promote16(acc + 64 + c, pb + 128 + half * 64 + c, s_hi);
+          for (int c = 0; c < kCols / 2; c += 32)
+            promote32(acc + kCols / 2 + c, pb + 128 + cq * (kCols / 2) + c, s_hi);
         } else {
 #pragma unroll
-          for (int c = 0; c < 128; c += 16) promote16(acc + c, pb + half * 128 + c, s_lo);
+          for (int c = 0; c < kCols; c += 32) promote32(acc + c, pb + cq * kCols + c, s_lo);
         }
         tc_fence_before();
         mbar_arrive(pempty(buf));
@@ -276,32 +314,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       const bool valid = r < T.rows;
       if constexpr (EPI == EPI_SWIGLU) {
-        // h = silu(gate) * up for 64 channels, then e4m3 with one scale per
-        // row per 128 channels (this tile's 128 h columns): the two halves of
-        // a row exchange their partial amax through shared memory
+        // h = silu(gate) * up for 32 channels, then e4m3 with one scale per
+        // row per 128 channels (this tile's 128 h columns): the four column
+        // quarters of a row exchange their partial amax through shared memory
+        constexpr int kH = kCols / 2;  // h channels per thread
         float amax = 0.f;
 #pragma unroll
-        for (int j = 0; j < 64; ++j) {
+        for (int j = 0; j < kH; ++j) {
           const float gv = acc[j];
-          const float hv = gv / (1.0f + __expf(-gv)) * acc[64 + j];
+          const float hv = gv / (1.0f + __expf(-gv)) * acc[kH + j];
           acc[j] = hv;
           amax = fmaxf(amax, fabsf(hv));
         }
-        float* xs = amax_x + (it & 1) * 2 * BM;
-        xs[half * BM + r] = amax;
+        float* xs = amax_x + (it & 1) * 4 * BM;
+        xs[cq * BM + r] = amax;
         mbar_arrive(xchg(it & 1));
         if (!__all_sync(0xffffffffu, mbar_wait(xchg(it & 1), (it >> 1) & 1, abort_flag))) {
           ok = false;
           break;
         }
-        amax = fmaxf(amax, xs[(1 - half) * BM + r]);
+#pragma unroll
+        for (int u = 0; u < kColGroups; ++u) amax = fmaxf(amax, xs[u * BM + r]);
         const float scale = amax > 0.f ? amax / 448.0f : 1.0f;
         if (valid) {
           uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
           const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
-          uint8_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * (BN / 2) + half * 64;
+          uint8_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * (BN / 2) + cq * kH;
 #pragma unroll
-          for (int j = 0; j < 64; j += 16) {
+          for (int j = 0; j < kH; j += 16) {
             uint32_t w4[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
@@ -313,7 +353,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             *reinterpret_cast<uint4*>(dst + j) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
-          if (half == 0) {
+          if (cq == 0) {
             float* os = T.p1 ? fa.out_scale1 : fa.out_scale0;
             const int osld = T.p1 ? fa.o_sld1 : fa.o_sld0;
             os[row * osld + T.n_tile] = scale;
@@ -323,9 +363,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (valid) {
           uint16_t* out = static_cast<uint16_t*>(T.p1 ? args.out1 : args.out0);
           const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
-          uint16_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * BN + half * 128;
+          uint16_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * BN + cq * kCols;
 #pragma unroll
-          for (int j = 0; j < 128; j += 8) {
+          for (int j = 0; j < kCols; j += 8) {
             *reinterpret_cast<uint4*>(dst + j) =
                 make_uint4(pack_bf16x2(acc[j], acc[j + 1]), pack_bf16x2(acc[j + 2], acc[j + 3]),
                            pack_bf16x2(acc[j + 4], acc[j + 5]), pack_bf16x2(acc[j + 6], acc[j + 7]));
