@@ -267,7 +267,7 @@ def run_ours(args, dist):
     mbs = cfg.microbatches
     n_max = max(mbs)
     weights = inputs.make_weights(cfg, dev)
-    h = api.asap_moe_create(cfg, weights, n_max)
+    h = api.asap_moe_create(cfg, weights, sum(mbs))   # sum: the batched call serves all at once
     del weights
     torch.cuda.empty_cache()
     xs = inputs.make_microbatches(cfg, dev)
@@ -349,6 +349,9 @@ def run_ours(args, dist):
         "of_sustained_measured": gemm_flops / (gemm_ms / 1e3) / 1e12 / peaks["bf16_tflops_sustained"],
         "peaks": peaks_src,
         "note": "algorithmic FLOPs of both grouped GEMMs (routed + shared) over their event-timed durations"}
+
+    # ---------------- all micro-batches in one pass (one grouped GEMM per weight matrix)
+    result["aggregated"] = aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist)
 
     # ---------------- end to end through host buffers
     result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
@@ -501,6 +504,76 @@ def roofline(kern, peaks, peaks_src, tensor_peak=None):
               "tensor_frac_of_sustained_measured": (a["flops"] / sec / 1e12 / tpk) if a["flops"] else None,
               "traffic_source": src})
     return r
+
+
+def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
+    """The same micro-batches through asap_moe_layer_batched: each expert's
+    weights stream once per step instead of once per micro-batch.  Also times
+    the two grouped GEMMs on the combined segments (route + dispatch of the
+    concatenated tokens, then the gate/up and down calls, events between)."""
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    n_all = sum(x.shape[0] for x in xs)
+    ws = api.workspace(h, n_all, dev)
+    outs = [torch.empty_like(x) for x in xs]
+    s = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        api.asap_moe_layer_batched(h, xs, outs, ws)
+    torch.cuda.synchronize()
+    dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    for _ in range(args.steps):
+        api.asap_moe_layer_batched(h, xs, outs, ws)
+    b.record(s)
+    torch.cuda.synchronize()
+    ms = dist.max(a.elapsed_time(b)) / args.steps
+    res = {"value": dist.world * n_all / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+           "note": "asap_moe_layer_batched over the step's micro-batches on one stream; outputs are bit-identical "
+                   "to the per-micro-batch calls"}
+    if cfg.dtype != "bf16":
+        return res
+    k, E, H, I, Is = cfg.top_k, cfg.n_experts, cfg.hidden, cfg.inter, cfg.shared_inter
+    x = torch.cat(xs)
+    idx = torch.empty((n_all, k), dtype=torch.int32, device=dev)
+    w = torch.empty((n_all, k), dtype=torch.float32, device=dev)
+    counts = torch.empty(E, dtype=torch.int32, device=dev)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    api.asap_moe_route(h, x, idx, w, counts, offsets, ws)
+    x_perm = torch.empty((n_all * k, H), dtype=torch.bfloat16, device=dev)
+    ps = torch.empty(n_all * k, dtype=torch.int32, device=dev)
+    pd = torch.empty((n_all, k), dtype=torch.int32, device=dev)
+    api.asap_moe_dispatch(h, x, idx, x_perm, ps, pd, ws)
+    del ws
+    hb = torch.empty((n_all * k, I), dtype=torch.bfloat16, device=dev)
+    hsh = torch.empty((n_all, Is), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
+    y = torch.empty_like(x_perm)
+    ysh = torch.empty((n_all, H), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
+    t1, t2 = [], []
+    for it in range(args.kernel_steps + 1):
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e[0].record(s)
+        api.asap_moe_expert_gate_up(h, x_perm, offsets, x, hb, hsh)
+        e[1].record(s)
+        api.asap_moe_expert_down(h, hb, offsets, hsh, n_all, y, ysh)
+        e[2].record(s)
+        torch.cuda.synchronize()
+        if it:
+            t1.append(e[0].elapsed_time(e[1]))
+            t2.append(e[1].elapsed_time(e[2]))
+    g1, g2 = sum(t1) / len(t1), sum(t2) / len(t2)
+    nk = n_all * k
+    flops = 2.0 * nk * H * 2 * I + 2.0 * nk * I * H + (6.0 * n_all * H * Is if cfg.n_shared else 0.0)
+    tf = flops / ((g1 + g2) / 1e3) / 1e12
+    active = int((counts > 0).sum().item())
+    wbytes = active * 3 * H * I * 2 + (3 * H * Is * 2 if cfg.n_shared else 0)
+    res.update({"gemm_gate_up_ms": g1, "gemm_down_ms": g2, "grouped_gemm_tflops": tf,
+                "grouped_gemm_frac_of_burst_measured": tf / peaks["bf16_tflops"],
+                "grouped_gemm_frac_of_sustained_measured": tf / peaks["bf16_tflops_sustained"],
+                "weight_gb_per_step": wbytes / 1e9})
+    return res
 
 
 def e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist):

@@ -265,6 +265,22 @@ int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
 int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
                            int32_t* counts, int32_t* offsets, void* stream);
 
+/* Several micro-batches that are ready at the same time, served in one pass:
+ * each is routed exactly as asap_moe_layer would route it alone, then the
+ * rows of all of them share the expert segments, so each expert's weights
+ * stream from HBM once for the whole set (one grouped GEMM per weight
+ * matrix) instead of once per micro-batch.  The paper serves DP groups one at
+ * a time and names the lower token density per MoE invocation as the cost of
+ * that (Section 3.3); this call trades the independence of the groups for
+ * that density when several are ready together.  out for micro-batch i is
+ * bit-identical to asap_moe_layer on xs[i] alone.
+ *   count      1..64; xs, ns, outs: host arrays of count device pointers /
+ *              sizes (ns[i] may be 0)
+ *   sum(ns) <= max_tokens; the workspace is asap_moe_workspace_size for
+ *   sum(ns) tokens. */
+int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,
+                           void* const* outs, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise the device, return ASAP_OK or ASAP_ERR_DEVICE_STATUS, write the
  * raw status word (0 = clean) to *word if non-NULL, then clear it. */
 int asap_moe_status(asap_moe_t h, uint32_t* word);

@@ -52,6 +52,7 @@ SIGNATURES = {
     "asap_moe_combine": [_P, _P, _P, _P, _P, _I, _P, _P],
     "asap_moe_layer": [_P, _P, _I, _P, _P, _SZ, _P],
     "asap_moe_route_noalloc": [_P, _P, _I, _P, _P, _P, _P, _P],
+    "asap_moe_layer_batched": [_P, _I, ctypes.POINTER(_P), ctypes.POINTER(_I), ctypes.POINTER(_P), _P, _SZ, _P],
     "asap_moe_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "asap_moe_last_error": [],
 }

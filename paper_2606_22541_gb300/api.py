@@ -148,6 +148,18 @@ def asap_moe_layer(h, x, out, ws, stream=None):
     check("asap_moe_layer", lib().asap_moe_layer(h.ptr, _ptr(x), x.shape[0], _ptr(out), p, n, _stream(stream)))
 
 
+def asap_moe_layer_batched(h, xs, outs, ws, stream=None):
+    """Serve several ready micro-batches in one pass (one grouped GEMM per
+    weight matrix); outs[i] equals asap_moe_layer on xs[i] bit for bit."""
+    cnt = len(xs)
+    xa = (ctypes.c_void_p * cnt)(*[x.data_ptr() for x in xs])
+    na = (ctypes.c_int32 * cnt)(*[x.shape[0] for x in xs])
+    oa = (ctypes.c_void_p * cnt)(*[o.data_ptr() for o in outs])
+    p, n = _ws(ws)
+    check("asap_moe_layer_batched",
+          lib().asap_moe_layer_batched(h.ptr, cnt, xa, na, oa, p, n, _stream(stream)))
+
+
 def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
     """asap_moe_route with its scratch in the library's static device array
     (at most 4096 tokens; calls overlapping on the GPU race)."""

@@ -54,6 +54,8 @@ int cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+constexpr int kMaxBatch = 64;  // micro-batches one asap_moe_layer_batched call may serve
+
 struct Layout {
   size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst;
   // bf16: x_perm (also y_perm in asap_moe_layer), h, h_sh, y_sh
@@ -73,7 +75,8 @@ Layout layout(const asap_moe_config& c, long long n) {
   };
   const size_t nk = static_cast<size_t>(n) * c.top_k;
   const size_t N = static_cast<size_t>(n);
-  const size_t chunks = (N + asap::kChunkTokens - 1) / asap::kChunkTokens;
+  // one extra chunk per micro-batch a batched call may serve
+  const size_t chunks = (N + asap::kChunkTokens - 1) / asap::kChunkTokens + kMaxBatch;
   const size_t H = c.hidden, I = c.inter, Is = c.n_shared ? c.shared_inter : 0, E = c.n_experts;
   L.logits = take(asap::kMaxRouterSplits * N * E * 4);  // K-slice planes
   L.idx = take(nk * 4);
@@ -777,6 +780,123 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
     return r;
   CU_TRY(asap::launch_combine(x_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
          "combine launch");
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,
+                                    void* const* outs, void* ws, size_t ws_bytes, void* stream) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  if (count < 1 || count > kMaxBatch || !xs || !ns || !outs)
+    return fail(ASAP_ERR_INVALID, "count must be in [1, 64] with host arrays xs, ns, outs");
+  long long N = 0;
+  for (int i = 0; i < count; ++i) {
+    if (ns[i] < 0) return fail(ASAP_ERR_INVALID, "negative micro-batch size");
+    if (ns[i] > 0 && (!xs[i] || !outs[i] || !aligned16(xs[i]) || !aligned16(outs[i])))
+      return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+    N += ns[i];
+  }
+  if (N > h->cfg.max_tokens)
+    return fail(ASAP_ERR_INVALID, "the micro-batches hold " + std::to_string(N) + " tokens, more than max_tokens");
+  int r = check_call(h, static_cast<int32_t>(N), ws, ws_bytes, true);
+  if (r != ASAP_OK || N == 0) return r;
+  const asap_moe_config& c = h->cfg;
+  const int n_all = static_cast<int>(N);
+  const Layout L = layout(c, n_all);
+  cudaStream_t st = S(stream);
+  const int k = c.top_k, E = c.n_experts;
+  const long long nk = N * k;
+  float* logits = at<float>(ws, L.logits);
+  int32_t* idx = at<int32_t>(ws, L.idx);
+  float* w = at<float>(ws, L.w);
+  int32_t* hist = at<int32_t>(ws, L.hist);
+  int32_t* base = at<int32_t>(ws, L.chunk_base);
+  int32_t* offsets = at<int32_t>(ws, L.offsets);
+  int32_t* perm_src = at<int32_t>(ws, L.perm_src);
+  int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
+  int chunks_total = 0;
+  for (int i = 0; i < count; ++i) chunks_total += asap::ceil_div(ns[i], asap::kChunkTokens);
+  // routing: each micro-batch exactly as asap_moe_route would route it alone
+  int tok0 = 0, chunk0 = 0;
+  for (int i = 0; i < count; ++i) {
+    const int n = ns[i];
+    if (n > 0) {
+      const int splits = router_splits(h, n);
+      float* lg = logits + static_cast<long long>(asap::kMaxRouterSplits) * tok0 * E;
+      if ((r = run_router_logits(h, xs[i], n, lg, splits, st)) != ASAP_OK) return r;
+      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h), idx + static_cast<long long>(tok0) * k,
+                                   w + static_cast<long long>(tok0) * k, hist, chunk0, chunks_total, st),
+             "gate launch");
+    }
+    tok0 += n;
+    chunk0 += asap::ceil_div(n, asap::kChunkTokens);
+  }
+  // one histogram scan over every chunk: expert segments hold the rows of all
+  // micro-batches, in (micro-batch, token, slot) order
+  CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, st), "scan launch");
+  void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
+  tok0 = 0;
+  chunk0 = 0;
+  for (int i = 0; i < count; ++i) {
+    const int n = ns[i];
+    if (n > 0) {
+      asap::DispatchSeg seg{};
+      seg.chunk0 = chunk0;
+      seg.n_chunks_total = chunks_total;
+      seg.tok0 = tok0;
+      seg.rows_total = nk;
+      const int32_t* idx_i = idx + static_cast<long long>(tok0) * k;
+      int32_t* pd_i = perm_dst + static_cast<long long>(tok0) * k;
+      if (h->fp8) {
+        void* xq_sh = c.n_shared ? static_cast<uint8_t*>(at<void>(ws, L.xq_sh)) + static_cast<long long>(tok0) * c.hidden
+                                 : nullptr;
+        float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) + static_cast<long long>(tok0) * (c.hidden / 128) : nullptr;
+        CU_TRY(asap::launch_dispatch_fp8_seg(xs[i], n, c.hidden, k, E, idx_i, base, at<void>(ws, L.xq),
+                                             at<float>(ws, L.xs), xq_sh, xs_sh, perm_src, pd_i, h->status, seg, st),
+               "dispatch launch");
+      } else {
+        // the shared expert reads the gathered rows from y_sh's region, which
+        // its own output overwrites only after the gate/up GEMM
+        seg.x_sh = y_sh ? static_cast<uint16_t*>(y_sh) + static_cast<long long>(tok0) * c.hidden : nullptr;
+        CU_TRY(asap::launch_dispatch_seg(xs[i], n, c.hidden, k, E, idx_i, base, at<void>(ws, L.x_perm), perm_src, pd_i,
+                                         h->status, seg, st),
+               "dispatch launch");
+      }
+    }
+    tok0 += n;
+    chunk0 += asap::ceil_div(n, asap::kChunkTokens);
+  }
+  // one grouped GEMM per weight matrix over every micro-batch's rows
+  void* y_perm;
+  if (h->fp8) {
+    void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
+    float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
+    if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n_all,
+                             at<void>(ws, L.hq), at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh),
+                             st)) != ASAP_OK)
+      return r;
+    y_perm = at<void>(ws, L.y_perm);
+    if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
+                          at<float>(ws, L.hs_sh), n_all, y_perm, y_sh, st)) != ASAP_OK)
+      return r;
+  } else {
+    y_perm = at<void>(ws, L.x_perm);
+    if ((r = run_gate_up(h, y_perm, offsets, y_sh, n_all, at<void>(ws, L.h), at<void>(ws, L.h_sh), st)) != ASAP_OK)
+      return r;
+    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), n_all, y_perm, y_sh, st)) != ASAP_OK)
+      return r;
+  }
+  tok0 = 0;
+  for (int i = 0; i < count; ++i) {
+    const int n = ns[i];
+    if (n > 0) {
+      const void* ysh_i = y_sh ? static_cast<const uint16_t*>(y_sh) + static_cast<long long>(tok0) * c.hidden : nullptr;
+      CU_TRY(asap::launch_combine(y_perm, ysh_i, w + static_cast<long long>(tok0) * k,
+                                  perm_dst + static_cast<long long>(tok0) * k, n, c.hidden, k, outs[i], h->status, st,
+                                  nk),
+             "combine launch");
+    }
+    tok0 += n;
+  }
   return ASAP_OK;
 }
 

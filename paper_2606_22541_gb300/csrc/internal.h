@@ -102,12 +102,29 @@ cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int
 cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                         int32_t* hist, cudaStream_t s);
 cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane, float* out, cudaStream_t s);
+// Gating of one micro-batch among several served together: its chunks are
+// columns [chunk0, chunk0 + ceil(n/32)) of the expert-major histogram with
+// n_chunks_total columns.
+cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
+                            int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s);
 cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
                         cudaStream_t s);
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
                         int32_t* chunk_base, cudaStream_t s);
 
 // ------------------------------------------------------------ permute
+// Place of one micro-batch among several served by one call: its chunks start
+// at column chunk0 of chunk_base (n_chunks_total columns), its tokens at
+// global index tok0, positions run over rows_total rows; x_sh (bf16 only,
+// nullable) receives its rows for the shared expert (pointer already offset
+// to the micro-batch's first token).
+struct DispatchSeg {
+  int chunk0;
+  int n_chunks_total;
+  int tok0;
+  long long rows_total;
+  void* x_sh;
+};
 cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
                             const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s);
@@ -117,9 +134,17 @@ cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int
 cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
                                 const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
                                 int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+// rows_total: rows of y_perm the positions may address (0 = n * k).
 cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float* w,
                            const int32_t* perm_dst, int n, int H, int k, void* out,
-                           uint32_t* status, cudaStream_t s);
+                           uint32_t* status, cudaStream_t s, long long rows_total = 0);
+cudaError_t launch_dispatch_seg(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                const int32_t* chunk_base, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
+                                uint32_t* status, const DispatchSeg& seg, cudaStream_t s);
+cudaError_t launch_dispatch_fp8_seg(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                    const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                    int32_t* perm_src, int32_t* perm_dst, uint32_t* status, const DispatchSeg& seg,
+                                    cudaStream_t s);
 // packed[e][b*256 + r] = gate[e][b*128 + r] (r < 128), up[...] for r >= 128
 // Rows are row_bytes wide (H * element size).
 cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, long long row_bytes, void* packed,

@@ -57,14 +57,14 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
                     const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
                     void* __restrict__ x_perm_v, float* __restrict__ xs, uint2* __restrict__ xq_sh,
                     float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
-                    int32_t* __restrict__ perm_dst, uint32_t* status) {
+                    int32_t* __restrict__ perm_dst, uint32_t* status, const DispatchSeg seg) {
   __shared__ int wcnt[kRankWarps][kMaxExperts];
   __shared__ int spos[kChunkTokens * kMaxTopK];
   const int c = blockIdx.x;
   const int t0 = c * kChunkTokens;
   const int nt = min(kChunkTokens, n - t0);
   const int ne = nt * k;
-  const int nk = n * k;
+  const long long nk = seg.rows_total;  // positions of every micro-batch of the call
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kRankWarps * E; i += blockDim.x) wcnt[i / E][i % E] = 0;
   __syncthreads();
@@ -85,7 +85,7 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
   }
   __syncthreads();
   for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
-    int run = chunk_base[static_cast<long long>(ee) * n_chunks + c];
+    int run = chunk_base[static_cast<long long>(ee) * n_chunks + seg.chunk0 + c];
 #pragma unroll
     for (int w = 0; w < kRankWarps; ++w) {
       const int v = wcnt[w][ee];
@@ -105,7 +105,7 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
     }
     spos[i] = pos;
     perm_dst[static_cast<long long>(t0) * k + i] = pos;
-    if (pos >= 0) perm_src[pos] = t0 + i / k;
+    if (pos >= 0) perm_src[pos] = seg.tok0 + t0 + i / k;
   }
   __syncthreads();
   // row copies: one warp per token, read once, write k times
@@ -116,6 +116,9 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
     for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[warp * k + j] : -1;
     if constexpr (!FP8) {
       uint4* x_perm = static_cast<uint4*>(x_perm_v);
+      // optional copy of the row for the shared expert (calls that serve
+      // several micro-batches gather their tokens into one matrix)
+      uint4* sh = seg.x_sh ? static_cast<uint4*>(seg.x_sh) + static_cast<long long>(t0 + warp) * V : nullptr;
       int v = lane;
       for (; v + 32 < V; v += 64) {
         const uint4 a = __ldg(src + v);
@@ -127,12 +130,17 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
             d[v] = a;
             d[v + 32] = b;
           }
+        if (sh) {
+          sh[v] = a;
+          sh[v + 32] = b;
+        }
       }
       for (; v < V; v += 32) {
         const uint4 a = __ldg(src + v);
 #pragma unroll
         for (int j = 0; j < kMaxTopK; ++j)
           if (p[j] >= 0) x_perm[static_cast<long long>(p[j]) * V + v] = a;
+        if (sh) sh[v] = a;
       }
     } else {
       // e4m3 rows: V vectors of 8 values -> V 8-byte words; one scale per 16
@@ -182,11 +190,10 @@ constexpr int kCombineWarps = 8;
 __global__ void __launch_bounds__(kCombineWarps * 32)
     combine_kernel(const uint4* __restrict__ y_perm, const uint4* __restrict__ y_sh,
                    const float* __restrict__ w, const int32_t* __restrict__ perm_dst, int n, int V,
-                   int k, uint4* __restrict__ out, uint32_t* status) {
+                   int k, uint4* __restrict__ out, uint32_t* status, long long nk) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = blockIdx.x * kCombineWarps + warp;
   if (t >= n) return;
-  const long long nk = static_cast<long long>(n) * k;
   int p[kMaxTopK];
   float wj[kMaxTopK];
 #pragma unroll
@@ -266,22 +273,43 @@ __global__ void pack_gate_up_kernel(const uint4* __restrict__ gate, const uint4*
 cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
                             const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+  DispatchSeg seg{};
+  seg.n_chunks_total = ceil_div(n, kChunkTokens);
+  seg.rows_total = static_cast<long long>(n) * k;
+  return launch_dispatch_seg(x, n, H, k, E, idx, chunk_base, x_perm, perm_src, perm_dst, status, seg, s);
+}
+
+cudaError_t launch_dispatch_seg(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                const int32_t* chunk_base, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
+                                uint32_t* status, const DispatchSeg& seg, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
   dispatch_kernel<false><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
-                                                                chunk_base, chunks, x_perm, nullptr, nullptr, nullptr,
-                                                                perm_src, perm_dst, status);
+                                                                chunk_base, seg.n_chunks_total, x_perm, nullptr,
+                                                                nullptr, nullptr, perm_src, perm_dst, status, seg);
   return cudaGetLastError();
 }
 
 cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
                                 const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
                                 int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+  DispatchSeg seg{};
+  seg.n_chunks_total = ceil_div(n, kChunkTokens);
+  seg.rows_total = static_cast<long long>(n) * k;
+  return launch_dispatch_fp8_seg(x, n, H, k, E, idx, chunk_base, xq, xs, xq_sh, xs_sh, perm_src, perm_dst, status,
+                                 seg, s);
+}
+
+cudaError_t launch_dispatch_fp8_seg(const void* x, int n, int H, int k, int E, const int32_t* idx,
+                                    const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                    int32_t* perm_src, int32_t* perm_dst, uint32_t* status, const DispatchSeg& seg,
+                                    cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
   dispatch_kernel<true><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
-                                                               chunk_base, chunks, xq, xs, static_cast<uint2*>(xq_sh),
-                                                               xs_sh, perm_src, perm_dst, status);
+                                                               chunk_base, seg.n_chunks_total, xq, xs,
+                                                               static_cast<uint2*>(xq_sh), xs_sh, perm_src, perm_dst,
+                                                               status, seg);
   return cudaGetLastError();
 }
 
@@ -294,11 +322,11 @@ cudaError_t launch_quantize_rows(const void* x, int rows, int cols, void* q, flo
 
 cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float* w,
                            const int32_t* perm_dst, int n, int H, int k, void* out, uint32_t* status,
-                           cudaStream_t s) {
+                           cudaStream_t s, long long rows_total) {
   if (n <= 0) return cudaSuccess;
   combine_kernel<<<ceil_div(n, kCombineWarps), kCombineWarps * 32, 0, s>>>(
       static_cast<const uint4*>(y_perm), static_cast<const uint4*>(y_shared), w, perm_dst, n, H / 8, k,
-      static_cast<uint4*>(out), status);
+      static_cast<uint4*>(out), status, rows_total > 0 ? rows_total : static_cast<long long>(n) * k);
   return cudaGetLastError();
 }
 

@@ -92,7 +92,8 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
                                                                long long plane, int n, GateParams p,
                                                                int32_t* __restrict__ idx,
                                                                float* __restrict__ wout,
-                                                               int32_t* __restrict__ hist, int n_chunks) {
+                                                               int32_t* __restrict__ hist, int n_chunks,
+                                                               int chunk0) {
   __shared__ int shist[kMaxExperts];
   __shared__ float ssel[kGateWarps][kMaxExperts];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -247,7 +248,8 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
   }
   __syncthreads();
   if (hist)
-    for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(e) * n_chunks + blockIdx.x] = shist[e];
+    for (int e = threadIdx.x; e < E; e += blockDim.x)
+      hist[static_cast<long long>(e) * n_chunks + chunk0 + blockIdx.x] = shist[e];
 }
 
 // ------------------------------------------------------------ histogram only
@@ -358,10 +360,15 @@ cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int
 
 cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                         int32_t* hist, cudaStream_t s) {
+  return launch_gate_seg(logits, splits, n, p, idx, w, hist, 0, ceil_div(n, kChunkTokens), s);
+}
+
+cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
+                            int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
   gate_kernel<<<chunks, kGateWarps * 32, 0, s>>>(logits, splits, static_cast<long long>(n) * p.n_experts, n, p,
-                                                  idx, w, hist, chunks);
+                                                  idx, w, hist, n_chunks_total, chunk0);
   return cudaGetLastError();
 }
 
