@@ -231,7 +231,8 @@ def sources_sha256(files):
     return d.hexdigest()
 
 
-GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb300/csrc/common.cuh"]
+GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb300/csrc/common.cuh",
+                "paper_2606_22541_gb300/csrc/gemm_sched.cuh", "paper_2606_22541_gb300/csrc/internal.h"]
 
 
 def weight_gb(cfg):

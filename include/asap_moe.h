@@ -158,6 +158,26 @@ typedef struct asap_moe_s* asap_moe_t;
 int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* weights,
                     asap_moe_t* out);
 
+/* One handle over n_layers MoE layers of the same shape: the layer-oblivious
+ * MoE Super Kernel of Section 3.4.2 (Section 4.1 describes it as a layer-ID
+ * input plus a pre-computed list of weight addresses).
+ *  - weights points to n_layers structs; layer l is copied and packed as
+ *    asap_moe_create does, and occupies that much HBM (all layers stay
+ *    resident).
+ *  - A device table receives, per layer, the TMA descriptors of its packed
+ *    weights and its router, bias and scale pointers.  Every kernel of this
+ *    library that reads weights finds them in that table at a layer id it
+ *    loads from device memory when it starts.
+ *  - Calls without a layer_id argument use layer 0.  asap_moe_create(c, w, o)
+ *    is asap_moe_create_layers(c, w, 1, o).
+ *  - 1 <= n_layers <= 4096, else ASAP_ERR_INVALID.  Synchronous, like
+ *    asap_moe_create.                                                      */
+int asap_moe_create_layers(const asap_moe_config* cfg, const asap_moe_weights* weights,
+                           int32_t n_layers, asap_moe_t* out);
+
+/* Number of layers of the handle (1 for asap_moe_create). */
+int asap_moe_n_layers(asap_moe_t h, int32_t* n_layers);
+
 /* Free everything create allocated.  Synchronises the device first.  NULL is
  * accepted. */
 int asap_moe_destroy(asap_moe_t h);
@@ -241,6 +261,22 @@ int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared,
 int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
                    size_t ws_bytes, void* stream);
 
+/* asap_moe_layer for the layer whose id is the int32 at layer_id (a device
+ * pointer).  The kernels load the id when they run, so what is enqueued does
+ * not depend on the layer: a sequence of these calls can be enqueued, or
+ * captured once in a CUDA graph and replayed, before the layer of each
+ * micro-batch is known (bubble-free kernel dispatching, Section 3.4.2).
+ *  - *layer_id must not change from the start of the call's first kernel to
+ *    the end of its last: write it on the same stream before the call, or
+ *    order the writer with an event.
+ *  - An id outside [0, n_layers) sets status bit 16 (asap_moe_status) and
+ *    the kernels use layer 0; nothing outside the table is read.
+ *  - NULL or unaligned layer_id returns ASAP_ERR_INVALID.
+ *  - out for layer l is bit-identical to asap_moe_layer on a handle created
+ *    from layer l's weights alone. */
+int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int32_t n,
+                       void* out, void* ws, size_t ws_bytes, void* stream);
+
 /* asap_moe_route without any device allocation (no counterpart in the
  * paper; this entry point exists for callers that cannot allocate).
  *
@@ -281,8 +317,17 @@ int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx,
 int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,
                            void* const* outs, void* ws, size_t ws_bytes, void* stream);
 
+/* asap_moe_layer_batched for micro-batches that all belong to the layer whose
+ * id is at layer_id (device int32), with the rules of asap_moe_layer_dyn. */
+int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t count,
+                               const void* const* xs, const int32_t* ns, void* const* outs,
+                               void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise the device, return ASAP_OK or ASAP_ERR_DEVICE_STATUS, write the
- * raw status word (0 = clean) to *word if non-NULL, then clear it. */
+ * raw status word (0 = clean) to *word if non-NULL, then clear it.  Bits:
+ * 1 expert index outside [0, E); 2 permutation position out of range;
+ * 4 a wait passed its time limit; 8 offsets not monotone or past the rows;
+ * 16 layer id outside [0, n_layers). */
 int asap_moe_status(asap_moe_t h, uint32_t* word);
 
 /* Thread-local text of this thread's last failure ("" if none). */

@@ -39,6 +39,9 @@ _SZ = ctypes.c_size_t
 
 SIGNATURES = {
     "asap_moe_create": [ctypes.POINTER(AsapMoeConfig), ctypes.POINTER(AsapMoeWeights), ctypes.POINTER(_P)],
+    "asap_moe_create_layers": [ctypes.POINTER(AsapMoeConfig), ctypes.POINTER(AsapMoeWeights), _I,
+                               ctypes.POINTER(_P)],
+    "asap_moe_n_layers": [_P, ctypes.POINTER(_I)],
     "asap_moe_destroy": [_P],
     "asap_moe_workspace_size": [ctypes.POINTER(AsapMoeConfig), _I, ctypes.POINTER(_SZ)],
     "asap_moe_check_config": [ctypes.POINTER(AsapMoeConfig)],
@@ -53,6 +56,9 @@ SIGNATURES = {
     "asap_moe_layer": [_P, _P, _I, _P, _P, _SZ, _P],
     "asap_moe_route_noalloc": [_P, _P, _I, _P, _P, _P, _P, _P],
     "asap_moe_layer_batched": [_P, _I, ctypes.POINTER(_P), ctypes.POINTER(_I), ctypes.POINTER(_P), _P, _SZ, _P],
+    "asap_moe_layer_dyn": [_P, _P, _P, _I, _P, _P, _SZ, _P],
+    "asap_moe_layer_batched_dyn": [_P, _P, _I, ctypes.POINTER(_P), ctypes.POINTER(_I), ctypes.POINTER(_P), _P, _SZ,
+                                   _P],
     "asap_moe_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "asap_moe_last_error": [],
 }

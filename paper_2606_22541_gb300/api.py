@@ -60,16 +60,38 @@ def asap_moe_check_config(cfg, max_tokens=1):
     return lib().asap_moe_check_config(ctypes.byref(c))
 
 
+def _weights_struct(weights, w):
+    for name, _ in AsapMoeWeights._fields_:
+        t = weights.get(name)
+        setattr(w, name, None if t is None else t.data_ptr())
+
+
 def asap_moe_create(cfg, weights, max_tokens):
     """weights: dict of CUDA tensors named like asap_moe_weights' fields."""
     c = make_config(cfg, max_tokens)
     w = AsapMoeWeights()
-    for name, _ in AsapMoeWeights._fields_:
-        t = weights.get(name)
-        setattr(w, name, None if t is None else t.data_ptr())
+    _weights_struct(weights, w)
     out = ctypes.c_void_p()
     check("asap_moe_create", lib().asap_moe_create(ctypes.byref(c), ctypes.byref(w), ctypes.byref(out)))
     return Handle(out, cfg, c)
+
+
+def asap_moe_create_layers(cfg, layers, max_tokens):
+    """One handle over several layers of the same shape; layers: a list of
+    weight dicts, one per layer (layer l = layers[l])."""
+    c = make_config(cfg, max_tokens)
+    ws = (AsapMoeWeights * len(layers))()
+    for i, weights in enumerate(layers):
+        _weights_struct(weights, ws[i])
+    out = ctypes.c_void_p()
+    check("asap_moe_create_layers", lib().asap_moe_create_layers(ctypes.byref(c), ws, len(layers), ctypes.byref(out)))
+    return Handle(out, cfg, c)
+
+
+def asap_moe_n_layers(h):
+    out = ctypes.c_int32()
+    check("asap_moe_n_layers", lib().asap_moe_n_layers(h.ptr, ctypes.byref(out)))
+    return out.value
 
 
 def asap_moe_destroy(h):
@@ -158,6 +180,25 @@ def asap_moe_layer_batched(h, xs, outs, ws, stream=None):
     p, n = _ws(ws)
     check("asap_moe_layer_batched",
           lib().asap_moe_layer_batched(h.ptr, cnt, xa, na, oa, p, n, _stream(stream)))
+
+
+def asap_moe_layer_dyn(h, layer_id, x, out, ws, stream=None):
+    """asap_moe_layer for the layer whose id the kernels read from layer_id
+    (a one-element int32 CUDA tensor) when they run."""
+    p, n = _ws(ws)
+    check("asap_moe_layer_dyn", lib().asap_moe_layer_dyn(h.ptr, _ptr(layer_id), _ptr(x), x.shape[0], _ptr(out), p, n,
+                                                         _stream(stream)))
+
+
+def asap_moe_layer_batched_dyn(h, layer_id, xs, outs, ws, stream=None):
+    """asap_moe_layer_batched for micro-batches of the layer at layer_id."""
+    cnt = len(xs)
+    xa = (ctypes.c_void_p * cnt)(*[x.data_ptr() for x in xs])
+    na = (ctypes.c_int32 * cnt)(*[x.shape[0] for x in xs])
+    oa = (ctypes.c_void_p * cnt)(*[o.data_ptr() for o in outs])
+    p, n = _ws(ws)
+    check("asap_moe_layer_batched_dyn",
+          lib().asap_moe_layer_batched_dyn(h.ptr, _ptr(layer_id), cnt, xa, na, oa, p, n, _stream(stream)))
 
 
 def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):

@@ -9,28 +9,35 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #define ASAP_API extern "C" __attribute__((visibility("default")))
 
-struct asap_moe_s {
-  asap_moe_config cfg;
-  int device = 0;
-  int num_sms = 0;
+// Device copies of one layer's weights.
+struct LayerWeights {
   void* router_w = nullptr;      // [E, H] bf16
   float* router_bias = nullptr;  // [E] fp32 or nullptr
-  void* gate_up = nullptr;       // [E][2I, H] bf16, gate/up interleaved per 128 rows
-  void* down = nullptr;          // [E][H, I] bf16
+  void* gate_up = nullptr;       // [E][2I, H], gate/up interleaved per 128 rows
+  void* down = nullptr;          // [E][H, I]
   void* sh_gate_up = nullptr;    // [2Is, H]
   void* sh_down = nullptr;       // [H, Is]
-  uint32_t* status = nullptr;    // device status word
-  bool tc_router = false;        // router GEMM on the tensor core (E == 256)
-  bool fp8 = false;              // e4m3 experts with fp32 128 x 128 block scales
   // FP8 only: block scales, gate/up rows interleaved like the weights
   float* gu_scales = nullptr;     // [E][2I/128][H/128]
   float* d_scales = nullptr;      // [E][H/128][I/128]
   float* sh_gu_scales = nullptr;  // [2Is/128][H/128]
   float* sh_d_scales = nullptr;   // [H/128][Is/128]
-  CUtensorMap tm_router, tm_gate_up, tm_down, tm_sh_gate_up, tm_sh_down;
+};
+
+struct asap_moe_s {
+  asap_moe_config cfg;
+  int device = 0;
+  int num_sms = 0;
+  std::vector<LayerWeights> layers;
+  asap::LayerEntry* table = nullptr;  // device [n_layers]: descriptors and pointers per layer
+  int32_t* layer_ids = nullptr;       // device [n_layers] = 0, 1, ...: fixed layer ids
+  uint32_t* status = nullptr;         // device status word
+  bool tc_router = false;             // router GEMM on the tensor core (E == 256)
+  bool fp8 = false;                   // e4m3 experts with fp32 128 x 128 block scales
 };
 
 namespace {
@@ -57,7 +64,7 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 constexpr int kMaxBatch = 64;  // micro-batches one asap_moe_layer_batched call may serve
 
 struct Layout {
-  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst;
+  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst, tile_counters;
   // bf16: x_perm (also y_perm in asap_moe_layer), h, h_sh, y_sh
   size_t x_perm, h, h_sh, y_sh;
   // fp8: quantised rows and their per-128-channel scales, bf16 expert outputs
@@ -87,6 +94,7 @@ Layout layout(const asap_moe_config& c, long long n) {
   L.offsets = take((E + 1) * 4);
   L.perm_src = take(nk * 4);
   L.perm_dst = take(nk * 4);
+  L.tile_counters = take(asap::kTileCounters * 4);
   if (c.dtype == ASAP_FP8_E4M3_BLOCK128) {
     L.xq = take(nk * H);
     L.xs = take(nk * (H / 128) * 4);
@@ -114,6 +122,11 @@ T* at(void* ws, size_t off) {
 }
 
 cudaStream_t S(void* s) { return static_cast<cudaStream_t>(s); }
+
+// The layer-table entry a launch reads: *layer, resolved on the device.
+asap::LayerRef lref(asap_moe_t h, const int32_t* layer) {
+  return asap::LayerRef{h->table, layer, static_cast<int>(h->layers.size())};
+}
 
 int check_call(asap_moe_t h, int32_t n, void* ws, size_t ws_bytes, bool needs_ws) {
   if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
@@ -149,17 +162,18 @@ int router_splits(asap_moe_t h, int n) {
 
 // Router logits as ``splits`` planes of partial sums [splits][n][E] (planes
 // are added in order by the consumer); splits == 1 writes the logits.
-int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int splits, cudaStream_t st) {
+int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int splits, const int32_t* layer,
+                      cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   if (h->tc_router) {
-    CUtensorMap maps[4];
+    CUtensorMap maps[2];
     std::string err;
     if (!asap::encode_tmap_bf16(&maps[0], x, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
-    maps[1] = h->tm_router;
-    maps[2] = maps[0];
-    maps[3] = maps[1];
+    maps[1] = maps[0];
     asap::GemmArgs a{};
+    a.lref = lref(h, layer);
+    a.bmap0 = a.bmap1 = asap::MAP_ROUTER;
     a.offsets = nullptr;
     a.groups = 1;
     a.m0 = n;
@@ -177,12 +191,13 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
     const int tiles = asap::ceil_div(n, asap::kGemmBM) * splits;
     CU_TRY(asap::gemm_launch(asap::EPI_F32, maps, a, std::min(tiles, h->num_sms), st), "router GEMM launch");
   } else {
-    CU_TRY(asap::launch_router_small(x, h->router_w, n, c.hidden, c.n_experts, logits, st), "router launch");
+    CU_TRY(asap::launch_router_small(x, lref(h, layer), n, c.hidden, c.n_experts, logits, h->status, st),
+           "router launch");
   }
   return ASAP_OK;
 }
 
-asap::GateParams gate_params(asap_moe_t h) {
+asap::GateParams gate_params(asap_moe_t h, const int32_t* layer) {
   const asap_moe_config& c = h->cfg;
   asap::GateParams p{};
   p.n_experts = c.n_experts;
@@ -191,18 +206,19 @@ asap::GateParams gate_params(asap_moe_t h) {
   p.n_groups = c.gating == ASAP_GATE_SIGMOID_GROUPED ? c.n_groups : 1;
   p.topk_groups = c.gating == ASAP_GATE_SIGMOID_GROUPED ? c.topk_groups : 1;
   p.route_scale = c.route_scale;
-  p.bias = h->router_bias;
+  p.lref = lref(h, layer);
+  p.status = h->status;
   return p;
 }
 
 int run_gate_scan(asap_moe_t h, const float* logits, int splits, int n, int32_t* idx, float* w, int32_t* counts,
-                  int32_t* offsets, void* ws, cudaStream_t st) {
+                  int32_t* offsets, void* ws, const int32_t* layer, cudaStream_t st) {
   const Layout L = layout(h->cfg, n);
   int32_t* hist = at<int32_t>(ws, L.hist);
   int32_t* base = at<int32_t>(ws, L.chunk_base);
-  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h), idx, w, hist, st), "gate launch");
+  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h, layer), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
-                           st),
+                           st, at<int32_t>(ws, L.tile_counters)),
          "scan launch");
   return ASAP_OK;
 }
@@ -213,25 +229,26 @@ int ub_mtiles(const asap_moe_config& c, long long nk) {
 
 // GEMM1: h = silu(X Wg^T) * (X Wu^T) on the routed segments, plus the shared
 // expert on x (problem 1 of the same launch).
+// counter: a zeroed int the launch claims its tiles from (nullptr: static order).
 int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n, void* hbuf,
-                void* hsh, cudaStream_t st) {
+                void* hsh, const int32_t* layer, int32_t* counter, cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
   std::string err;
-  CUtensorMap maps[4];
+  CUtensorMap maps[2];
   if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "x_perm: " + err);
-  maps[1] = h->tm_gate_up;
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[2], x, n, c.hidden, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
-    maps[3] = h->tm_sh_gate_up;
   } else {
-    maps[2] = maps[0];
-    maps[3] = maps[1];
+    maps[1] = maps[0];
   }
   asap::GemmArgs a{};
+  a.lref = lref(h, layer);
+  a.bmap0 = asap::MAP_GATE_UP;
+  a.bmap1 = sh ? asap::MAP_SH_GATE_UP : asap::MAP_GATE_UP;
   a.offsets = offsets;
   a.groups = c.n_experts;
   a.m0 = static_cast<int>(nk);
@@ -249,6 +266,7 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   a.hint_a = 2;
   a.hint_b = 1;
   a.k_splits = 1;
+  a.tile_counter = counter;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -258,24 +276,24 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
 
 // GEMM2: y = h Wd^T on the routed segments, plus the shared expert.
 int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void* hsh, int n, void* y_perm,
-             void* y_sh, cudaStream_t st) {
+             void* y_sh, const int32_t* layer, int32_t* counter, cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
   std::string err;
-  CUtensorMap maps[4];
+  CUtensorMap maps[2];
   if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "h: " + err);
-  maps[1] = h->tm_down;
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[2], hsh, n, c.shared_inter, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "h_shared: " + err);
-    maps[3] = h->tm_sh_down;
   } else {
-    maps[2] = maps[0];
-    maps[3] = maps[1];
+    maps[1] = maps[0];
   }
   asap::GemmArgs a{};
+  a.lref = lref(h, layer);
+  a.bmap0 = asap::MAP_DOWN;
+  a.bmap1 = sh ? asap::MAP_SH_DOWN : asap::MAP_DOWN;
   a.offsets = offsets;
   a.groups = c.n_experts;
   a.m0 = static_cast<int>(nk);
@@ -293,6 +311,7 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.hint_a = 2;
   a.hint_b = 1;
   a.k_splits = 1;
+  a.tile_counter = counter;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -300,34 +319,37 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   return ASAP_OK;
 }
 
+// counters: kTileCounters zeroed ints (or nullptr)
 int run_expert_ffn(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n,
-                   void* y_perm, void* y_sh, void* hbuf, void* hsh, cudaStream_t st) {
-  int r = run_gate_up(h, x_perm, offsets, x, n, hbuf, hsh, st);
+                   void* y_perm, void* y_sh, void* hbuf, void* hsh, const int32_t* layer, int32_t* counters,
+                   cudaStream_t st) {
+  int r = run_gate_up(h, x_perm, offsets, x, n, hbuf, hsh, layer, counters, st);
   if (r != ASAP_OK) return r;
-  return run_down(h, hbuf, offsets, hsh, n, y_perm, y_sh, st);
+  return run_down(h, hbuf, offsets, hsh, n, y_perm, y_sh, layer, counters ? counters + 1 : nullptr, st);
 }
 
 // FP8 GEMM1: hq = e4m3(silu(Xq Wg^T) * (Xq Wu^T)) with its row scales, routed
 // segments plus the shared expert on the quantised x.
 int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t* offsets, const void* xq_sh,
-                    const float* xs_sh, int n, void* hq, float* hs, void* hq_sh, float* hs_sh, cudaStream_t st) {
+                    const float* xs_sh, int n, void* hq, float* hs, void* hq_sh, float* hs_sh, const int32_t* layer,
+                    int32_t* counter, cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
   std::string err;
-  CUtensorMap maps[4];
+  CUtensorMap maps[2];
   if (!asap::encode_tmap_u8(&maps[0], xq, nk, c.hidden, asap::kGemmBM, &err)) return fail(ASAP_ERR_INVALID, "x_perm: " + err);
-  maps[1] = h->tm_gate_up;
   if (sh) {
-    if (!asap::encode_tmap_u8(&maps[2], xq_sh, n, c.hidden, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_u8(&maps[1], xq_sh, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "quantised x: " + err);
-    maps[3] = h->tm_sh_gate_up;
   } else {
-    maps[2] = maps[0];
-    maps[3] = maps[1];
+    maps[1] = maps[0];
   }
   asap::Fp8Args f{};
   asap::GemmArgs& a = f.g;
+  a.lref = lref(h, layer);
+  a.bmap0 = asap::MAP_GATE_UP;
+  a.bmap1 = sh ? asap::MAP_SH_GATE_UP : asap::MAP_GATE_UP;
   a.offsets = offsets;
   a.groups = c.n_experts;
   a.m0 = static_cast<int>(nk);
@@ -345,13 +367,12 @@ int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t
   a.hint_a = 2;
   a.hint_b = 1;
   a.k_splits = 1;
+  a.tile_counter = counter;
   f.a_scale0 = xs;
   f.a_sld0 = c.hidden / 128;
   f.a_scale1 = xs_sh;
   f.a_sld1 = c.hidden / 128;
-  f.b_scale0 = h->gu_scales;
   f.b_nblk0 = 2 * c.inter / 128;
-  f.b_scale1 = h->sh_gu_scales;
   f.b_nblk1 = sh ? 2 * c.shared_inter / 128 : 0;
   f.out_scale0 = hs;
   f.o_sld0 = c.inter / 128;
@@ -366,24 +387,25 @@ int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t
 
 // FP8 GEMM2: y = (hq * hs) (Wd * sd)^T, bf16 out.
 int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* offsets, const void* hq_sh,
-                 const float* hs_sh, int n, void* y_perm, void* y_sh, cudaStream_t st) {
+                 const float* hs_sh, int n, void* y_perm, void* y_sh, const int32_t* layer, int32_t* counter,
+                 cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
   std::string err;
-  CUtensorMap maps[4];
+  CUtensorMap maps[2];
   if (!asap::encode_tmap_u8(&maps[0], hq, nk, c.inter, asap::kGemmBM, &err)) return fail(ASAP_ERR_INVALID, "h: " + err);
-  maps[1] = h->tm_down;
   if (sh) {
-    if (!asap::encode_tmap_u8(&maps[2], hq_sh, n, c.shared_inter, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_u8(&maps[1], hq_sh, n, c.shared_inter, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "h_shared: " + err);
-    maps[3] = h->tm_sh_down;
   } else {
-    maps[2] = maps[0];
-    maps[3] = maps[1];
+    maps[1] = maps[0];
   }
   asap::Fp8Args f{};
   asap::GemmArgs& a = f.g;
+  a.lref = lref(h, layer);
+  a.bmap0 = asap::MAP_DOWN;
+  a.bmap1 = sh ? asap::MAP_SH_DOWN : asap::MAP_DOWN;
   a.offsets = offsets;
   a.groups = c.n_experts;
   a.m0 = static_cast<int>(nk);
@@ -401,13 +423,12 @@ int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* o
   a.hint_a = 2;
   a.hint_b = 1;
   a.k_splits = 1;
+  a.tile_counter = counter;
   f.a_scale0 = hs;
   f.a_sld0 = c.inter / 128;
   f.a_scale1 = hs_sh;
   f.a_sld1 = sh ? c.shared_inter / 128 : 0;
-  f.b_scale0 = h->d_scales;
   f.b_nblk0 = c.hidden / 128;
-  f.b_scale1 = h->sh_d_scales;
   f.b_nblk1 = c.hidden / 128;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
@@ -465,38 +486,147 @@ ASAP_API int asap_moe_destroy(asap_moe_t h) {
   cudaGetDevice(&prev);
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
-  cudaFree(h->router_w);
-  cudaFree(h->router_bias);
-  cudaFree(h->gate_up);
-  cudaFree(h->down);
-  cudaFree(h->sh_gate_up);
-  cudaFree(h->sh_down);
+  for (LayerWeights& L : h->layers) {
+    cudaFree(L.router_w);
+    cudaFree(L.router_bias);
+    cudaFree(L.gate_up);
+    cudaFree(L.down);
+    cudaFree(L.sh_gate_up);
+    cudaFree(L.sh_down);
+    cudaFree(L.gu_scales);
+    cudaFree(L.d_scales);
+    cudaFree(L.sh_gu_scales);
+    cudaFree(L.sh_d_scales);
+  }
+  cudaFree(h->table);
+  cudaFree(h->layer_ids);
   cudaFree(h->status);
-  cudaFree(h->gu_scales);
-  cudaFree(h->d_scales);
-  cudaFree(h->sh_gu_scales);
-  cudaFree(h->sh_d_scales);
   cudaSetDevice(prev);
   delete h;
   return ASAP_OK;
 }
 
-ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* wts, asap_moe_t* out) {
+namespace {
+
+constexpr int kMaxLayers = 4096;
+
+int check_weights(const asap_moe_config& c, const asap_moe_weights* wts) {
+  if (!wts || !wts->router_w || !wts->w_gate || !wts->w_up || !wts->w_down)
+    return fail(ASAP_ERR_INVALID, "router and expert weights are required");
+  if (c.n_shared && (!wts->sh_gate || !wts->sh_up || !wts->sh_down))
+    return fail(ASAP_ERR_INVALID, "shared-expert weights are required when n_shared == 1");
+  if (c.dtype == ASAP_FP8_E4M3_BLOCK128 &&
+      (!wts->s_gate || !wts->s_up || !wts->s_down ||
+       (c.n_shared && (!wts->sh_s_gate || !wts->sh_s_up || !wts->sh_s_down))))
+    return fail(ASAP_ERR_INVALID, "the FP8 configuration needs the fp32 block scales of every expert matrix");
+  return ASAP_OK;
+}
+
+// Allocate one layer's device copies and enqueue the copies / packing on st.
+int pack_layer(asap_moe_t h, const asap_moe_weights* wts, LayerWeights& L, cudaStream_t st) {
+  const asap_moe_config& c = h->cfg;
+  const size_t H = c.hidden, E = c.n_experts, I = c.inter, Is = c.shared_inter;
+  const size_t wb = h->fp8 ? 1 : 2;  // bytes per expert-weight element
+  const size_t router_bytes = E * H * 2, gu_bytes = E * 2 * I * H * wb, down_bytes = E * H * I * wb;
+  cudaError_t e;
+  if ((e = cudaMalloc(&L.router_w, router_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc router");
+  if ((e = cudaMemcpyAsync(L.router_w, wts->router_w, router_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+    return cuda_fail(e, "copy router");
+  if (wts->router_bias) {
+    if ((e = cudaMalloc(&L.router_bias, E * 4)) != cudaSuccess) return cuda_fail(e, "cudaMalloc bias");
+    if ((e = cudaMemcpyAsync(L.router_bias, wts->router_bias, E * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+      return cuda_fail(e, "copy bias");
+  }
+  if ((e = cudaMalloc(&L.gate_up, gu_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc gate/up");
+  if ((e = asap::launch_pack_gate_up(wts->w_gate, wts->w_up, static_cast<int>(E), static_cast<int>(I),
+                                     static_cast<long long>(H * wb), L.gate_up, st)) != cudaSuccess)
+    return cuda_fail(e, "pack gate/up");
+  if ((e = cudaMalloc(&L.down, down_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc down");
+  if ((e = cudaMemcpyAsync(L.down, wts->w_down, down_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+    return cuda_fail(e, "copy down");
+  if (c.n_shared) {
+    if ((e = cudaMalloc(&L.sh_gate_up, 2 * Is * H * wb)) != cudaSuccess) return cuda_fail(e, "cudaMalloc shared");
+    if ((e = asap::launch_pack_gate_up(wts->sh_gate, wts->sh_up, 1, static_cast<int>(Is),
+                                       static_cast<long long>(H * wb), L.sh_gate_up, st)) != cudaSuccess)
+      return cuda_fail(e, "pack shared");
+    if ((e = cudaMalloc(&L.sh_down, H * Is * wb)) != cudaSuccess) return cuda_fail(e, "cudaMalloc shared down");
+    if ((e = cudaMemcpyAsync(L.sh_down, wts->sh_down, H * Is * wb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+      return cuda_fail(e, "copy shared down");
+  }
+  if (h->fp8) {
+    // scale rows interleaved like the weight rows: gate block b -> 2b, up block b -> 2b+1
+    const size_t kb = H / 128, rowb = kb * 4;
+    auto interleave = [&](float** dst, const float* g, const float* u, size_t blocks) -> cudaError_t {
+      cudaError_t r = cudaMalloc(dst, 2 * blocks * rowb);
+      if (r == cudaSuccess) r = cudaMemcpy2DAsync(*dst, 2 * rowb, g, rowb, rowb, blocks, cudaMemcpyDeviceToDevice, st);
+      if (r == cudaSuccess)
+        r = cudaMemcpy2DAsync(reinterpret_cast<char*>(*dst) + rowb, 2 * rowb, u, rowb, rowb, blocks,
+                              cudaMemcpyDeviceToDevice, st);
+      return r;
+    };
+    if ((e = interleave(&L.gu_scales, wts->s_gate, wts->s_up, E * (I / 128))) != cudaSuccess)
+      return cuda_fail(e, "gate/up scales");
+    const size_t dsb = E * (H / 128) * (I / 128) * 4;
+    if ((e = cudaMalloc(&L.d_scales, dsb)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(L.d_scales, wts->s_down, dsb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+      return cuda_fail(e, "down scales");
+    if (c.n_shared) {
+      if ((e = interleave(&L.sh_gu_scales, wts->sh_s_gate, wts->sh_s_up, Is / 128)) != cudaSuccess)
+        return cuda_fail(e, "shared gate/up scales");
+      const size_t sdb = (H / 128) * (Is / 128) * 4;
+      if ((e = cudaMalloc(&L.sh_d_scales, sdb)) != cudaSuccess ||
+          (e = cudaMemcpyAsync(L.sh_d_scales, wts->sh_s_down, sdb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
+        return cuda_fail(e, "shared down scales");
+    }
+  }
+  return ASAP_OK;
+}
+
+// The table entry of one layer: TMA descriptors of its packed weights (the
+// pre-computed addresses of Section 3.4.2) and its plain pointers.
+int encode_layer(asap_moe_t h, const LayerWeights& L, asap::LayerEntry* out) {
+  const asap_moe_config& c = h->cfg;
+  const uint64_t H = c.hidden, E = c.n_experts, I = c.inter, Is = c.shared_inter;
+  std::memset(out, 0, sizeof(*out));
+  std::string err;
+  if (h->tc_router && !asap::encode_tmap_bf16(&out->map[asap::MAP_ROUTER], L.router_w, E, H, asap::kGemmBN, &err))
+    return fail(ASAP_ERR_CUDA, "router map: " + err);
+  auto enc = [&](int which, const void* p, uint64_t rows, uint64_t cols) {
+    return h->fp8 ? asap::encode_tmap_u8(&out->map[which], p, rows, cols, asap::kGemmBN, &err)
+                  : asap::encode_tmap_bf16(&out->map[which], p, rows, cols, asap::kGemmBN, &err);
+  };
+  if (!enc(asap::MAP_GATE_UP, L.gate_up, E * 2 * I, H)) return fail(ASAP_ERR_CUDA, "gate/up map: " + err);
+  if (!enc(asap::MAP_DOWN, L.down, E * H, I)) return fail(ASAP_ERR_CUDA, "down map: " + err);
+  if (c.n_shared) {
+    if (!enc(asap::MAP_SH_GATE_UP, L.sh_gate_up, 2 * Is, H)) return fail(ASAP_ERR_CUDA, "shared gate/up map: " + err);
+    if (!enc(asap::MAP_SH_DOWN, L.sh_down, H, Is)) return fail(ASAP_ERR_CUDA, "shared down map: " + err);
+  }
+  out->scale[asap::MAP_GATE_UP] = L.gu_scales;
+  out->scale[asap::MAP_DOWN] = L.d_scales;
+  out->scale[asap::MAP_SH_GATE_UP] = L.sh_gu_scales;
+  out->scale[asap::MAP_SH_DOWN] = L.sh_d_scales;
+  out->router_w = L.router_w;
+  out->router_bias = L.router_bias;
+  return ASAP_OK;
+}
+
+}  // namespace
+
+ASAP_API int asap_moe_create_layers(const asap_moe_config* cfg, const asap_moe_weights* wts, int32_t n_layers,
+                                    asap_moe_t* out) {
   if (!out) return fail(ASAP_ERR_INVALID, "NULL out");
   *out = nullptr;
   int r = asap_moe_check_config(cfg);
   if (r != ASAP_OK) return r;
-  if (!wts || !wts->router_w || !wts->w_gate || !wts->w_up || !wts->w_down)
-    return fail(ASAP_ERR_INVALID, "router and expert weights are required");
-  if (cfg->n_shared && (!wts->sh_gate || !wts->sh_up || !wts->sh_down))
-    return fail(ASAP_ERR_INVALID, "shared-expert weights are required when n_shared == 1");
-  if (cfg->dtype == ASAP_FP8_E4M3_BLOCK128 &&
-      (!wts->s_gate || !wts->s_up || !wts->s_down ||
-       (cfg->n_shared && (!wts->sh_s_gate || !wts->sh_s_up || !wts->sh_s_down))))
-    return fail(ASAP_ERR_INVALID, "the FP8 configuration needs the fp32 block scales of every expert matrix");
+  if (n_layers < 1 || n_layers > kMaxLayers)
+    return fail(ASAP_ERR_INVALID, "n_layers must be in [1, " + std::to_string(kMaxLayers) + "]");
+  if (!wts) return fail(ASAP_ERR_INVALID, "router and expert weights are required");
+  for (int l = 0; l < n_layers; ++l)
+    if ((r = check_weights(*cfg, wts + l)) != ASAP_OK) return fail(r, "layer " + std::to_string(l) + ": " + g_last_error);
   const asap_moe_config& c = *cfg;
   asap_moe_s* h = new asap_moe_s();
   h->cfg = c;
+  h->layers.resize(n_layers);
   cudaStream_t st = nullptr;
   auto bail = [&](int code) {
     if (st) cudaStreamDestroy(st);
@@ -521,85 +651,43 @@ ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights*
   if (e == cudaSuccess) e = asap::fp8_gemm_set_attributes();
   if (e != cudaSuccess) return bail(cuda_fail(e, "GEMM attributes"));
   h->fp8 = c.dtype == ASAP_FP8_E4M3_BLOCK128;
+  h->tc_router = (c.n_experts == asap::kGemmBN);
   e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking);
   if (e != cudaSuccess) return bail(cuda_fail(e, "stream"));
-
-  const size_t H = c.hidden, E = c.n_experts, I = c.inter, Is = c.shared_inter;
-  const size_t wb = h->fp8 ? 1 : 2;  // bytes per expert-weight element
-  const size_t router_bytes = E * H * 2, gu_bytes = E * 2 * I * H * wb, down_bytes = E * H * I * wb;
   if ((e = cudaMalloc(&h->status, 256)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc status"));
   if ((e = cudaMemsetAsync(h->status, 0, 256, st)) != cudaSuccess) return bail(cuda_fail(e, "memset"));
-  if ((e = cudaMalloc(&h->router_w, router_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc router"));
-  if ((e = cudaMemcpyAsync(h->router_w, wts->router_w, router_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-    return bail(cuda_fail(e, "copy router"));
-  if (wts->router_bias) {
-    if ((e = cudaMalloc(&h->router_bias, E * 4)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc bias"));
-    if ((e = cudaMemcpyAsync(h->router_bias, wts->router_bias, E * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-      return bail(cuda_fail(e, "copy bias"));
+  for (int l = 0; l < n_layers; ++l)
+    if ((r = pack_layer(h, wts + l, h->layers[l], st)) != ASAP_OK)
+      return bail(fail(r, "layer " + std::to_string(l) + ": " + g_last_error));
+  // the layer table and the fixed ids 0 .. n_layers-1
+  std::vector<asap::LayerEntry> table(n_layers);
+  std::vector<int32_t> ids(n_layers);
+  for (int l = 0; l < n_layers; ++l) {
+    if ((r = encode_layer(h, h->layers[l], &table[l])) != ASAP_OK)
+      return bail(fail(r, "layer " + std::to_string(l) + ": " + g_last_error));
+    ids[l] = l;
   }
-  if ((e = cudaMalloc(&h->gate_up, gu_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc gate/up"));
-  if ((e = asap::launch_pack_gate_up(wts->w_gate, wts->w_up, static_cast<int>(E), static_cast<int>(I),
-                                     static_cast<long long>(H * wb), h->gate_up, st)) != cudaSuccess)
-    return bail(cuda_fail(e, "pack gate/up"));
-  if ((e = cudaMalloc(&h->down, down_bytes)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc down"));
-  if ((e = cudaMemcpyAsync(h->down, wts->w_down, down_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-    return bail(cuda_fail(e, "copy down"));
-  if (c.n_shared) {
-    if ((e = cudaMalloc(&h->sh_gate_up, 2 * Is * H * wb)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared"));
-    if ((e = asap::launch_pack_gate_up(wts->sh_gate, wts->sh_up, 1, static_cast<int>(Is), static_cast<long long>(H * wb),
-                                       h->sh_gate_up, st)) != cudaSuccess)
-      return bail(cuda_fail(e, "pack shared"));
-    if ((e = cudaMalloc(&h->sh_down, H * Is * wb)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc shared down"));
-    if ((e = cudaMemcpyAsync(h->sh_down, wts->sh_down, H * Is * wb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-      return bail(cuda_fail(e, "copy shared down"));
-  }
-  if (h->fp8) {
-    // scale rows interleaved like the weight rows: gate block b -> 2b, up block b -> 2b+1
-    const size_t kb = H / 128, rowb = kb * 4;
-    auto interleave = [&](float** dst, const float* g, const float* u, size_t blocks) -> cudaError_t {
-      cudaError_t r = cudaMalloc(dst, 2 * blocks * rowb);
-      if (r == cudaSuccess) r = cudaMemcpy2DAsync(*dst, 2 * rowb, g, rowb, rowb, blocks, cudaMemcpyDeviceToDevice, st);
-      if (r == cudaSuccess)
-        r = cudaMemcpy2DAsync(reinterpret_cast<char*>(*dst) + rowb, 2 * rowb, u, rowb, rowb, blocks,
-                              cudaMemcpyDeviceToDevice, st);
-      return r;
-    };
-    if ((e = interleave(&h->gu_scales, wts->s_gate, wts->s_up, E * (I / 128))) != cudaSuccess)
-      return bail(cuda_fail(e, "gate/up scales"));
-    const size_t dsb = E * (H / 128) * (I / 128) * 4;
-    if ((e = cudaMalloc(&h->d_scales, dsb)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(h->d_scales, wts->s_down, dsb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-      return bail(cuda_fail(e, "down scales"));
-    if (c.n_shared) {
-      if ((e = interleave(&h->sh_gu_scales, wts->sh_s_gate, wts->sh_s_up, Is / 128)) != cudaSuccess)
-        return bail(cuda_fail(e, "shared gate/up scales"));
-      const size_t sdb = (H / 128) * (Is / 128) * 4;
-      if ((e = cudaMalloc(&h->sh_d_scales, sdb)) != cudaSuccess ||
-          (e = cudaMemcpyAsync(h->sh_d_scales, wts->sh_s_down, sdb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-        return bail(cuda_fail(e, "shared down scales"));
-    }
-  }
+  const size_t tb = sizeof(asap::LayerEntry) * n_layers;
+  if ((e = cudaMalloc(&h->table, tb)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc layer table"));
+  if ((e = cudaMalloc(&h->layer_ids, 4 * n_layers)) != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc layer ids"));
+  // (pageable host sources, complete by the stream synchronisation below)
+  if ((e = cudaMemcpyAsync(h->table, table.data(), tb, cudaMemcpyHostToDevice, st)) != cudaSuccess ||
+      (e = cudaMemcpyAsync(h->layer_ids, ids.data(), 4 * n_layers, cudaMemcpyHostToDevice, st)) != cudaSuccess)
+    return bail(cuda_fail(e, "copy layer table"));
   if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return bail(cuda_fail(e, "create sync"));
   cudaStreamDestroy(st);
   st = nullptr;
-
-  std::string err;
-  h->tc_router = (c.n_experts == asap::kGemmBN);
-  if (h->tc_router && !asap::encode_tmap_bf16(&h->tm_router, h->router_w, E, H, asap::kGemmBN, &err))
-    return bail(fail(ASAP_ERR_CUDA, "router map: " + err));
-  auto enc = [&](CUtensorMap* m, const void* p, uint64_t rows, uint64_t cols) {
-    return h->fp8 ? asap::encode_tmap_u8(m, p, rows, cols, asap::kGemmBN, &err)
-                  : asap::encode_tmap_bf16(m, p, rows, cols, asap::kGemmBN, &err);
-  };
-  if (!enc(&h->tm_gate_up, h->gate_up, E * 2 * I, H)) return bail(fail(ASAP_ERR_CUDA, "gate/up map: " + err));
-  if (!enc(&h->tm_down, h->down, E * H, I)) return bail(fail(ASAP_ERR_CUDA, "down map: " + err));
-  if (c.n_shared) {
-    if (!enc(&h->tm_sh_gate_up, h->sh_gate_up, 2 * Is, H))
-      return bail(fail(ASAP_ERR_CUDA, "shared gate/up map: " + err));
-    if (!enc(&h->tm_sh_down, h->sh_down, H, Is)) return bail(fail(ASAP_ERR_CUDA, "shared down map: " + err));
-  }
   *out = h;
   return ASAP_OK;
+}
+
+ASAP_API int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* wts, asap_moe_t* out) {
+  if (!out) return fail(ASAP_ERR_INVALID, "NULL out");
+  *out = nullptr;
+  int r = asap_moe_check_config(cfg);
+  if (r != ASAP_OK) return r;
+  if ((r = check_weights(*cfg, wts)) != ASAP_OK) return r;
+  return asap_moe_create_layers(cfg, wts, 1, out);
 }
 
 ASAP_API int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, float* logits, void* ws,
@@ -609,10 +697,10 @@ ASAP_API int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, floa
   if (!x || !logits || !aligned16(x) || !aligned16(logits))
     return fail(ASAP_ERR_INVALID, "x and logits must be non-NULL and 16-byte aligned");
   const int splits = router_splits(h, n);
-  if (splits == 1) return run_router_logits(h, x, n, logits, 1, S(stream));
+  if (splits == 1) return run_router_logits(h, x, n, logits, 1, h->layer_ids, S(stream));
   // the same K slices and the same order of addition as asap_moe_route
   float* parts = at<float>(ws, layout(h->cfg, n).logits);
-  if ((r = run_router_logits(h, x, n, parts, splits, S(stream))) != ASAP_OK) return r;
+  if ((r = run_router_logits(h, x, n, parts, splits, h->layer_ids, S(stream))) != ASAP_OK) return r;
   CU_TRY(asap::launch_reduce_splits(parts, splits, static_cast<long long>(n) * h->cfg.n_experts, logits, S(stream)),
          "logit reduction launch");
   return ASAP_OK;
@@ -623,7 +711,7 @@ ASAP_API int asap_moe_route_logits(asap_moe_t h, const float* logits, int32_t n,
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!logits || !idx || !w || !counts || !offsets) return fail(ASAP_ERR_INVALID, "NULL tensor");
-  return run_gate_scan(h, logits, 1, n, idx, w, counts, offsets, ws, S(stream));
+  return run_gate_scan(h, logits, 1, n, idx, w, counts, offsets, ws, h->layer_ids, S(stream));
 }
 
 ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w, int32_t* counts,
@@ -633,9 +721,9 @@ ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx
   if (!x || !idx || !w || !counts || !offsets || !aligned16(x)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   float* logits = at<float>(ws, layout(h->cfg, n).logits);
   const int splits = router_splits(h, n);
-  r = run_router_logits(h, x, n, logits, splits, S(stream));
+  r = run_router_logits(h, x, n, logits, splits, h->layer_ids, S(stream));
   if (r != ASAP_OK) return r;
-  return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, S(stream));
+  return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, h->layer_ids, S(stream));
 }
 
 ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx, void* x_perm,
@@ -677,6 +765,8 @@ ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* 
     return fail(ASAP_ERR_INVALID, "x and y_shared are required for the shared expert");
   const Layout L = layout(h->cfg, n);
   cudaStream_t st = S(stream);
+  int32_t* counters = at<int32_t>(ws, L.tile_counters);
+  CU_TRY(cudaMemsetAsync(counters, 0, asap::kTileCounters * sizeof(int32_t), st), "tile counters");
   if (h->fp8) {
     if (!x_perm_scales) return fail(ASAP_ERR_INVALID, "the FP8 configuration needs x_perm_scales");
     const asap_moe_config& c = h->cfg;
@@ -684,12 +774,14 @@ ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* 
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
     if (c.n_shared) CU_TRY(asap::launch_quantize_rows(x, n, c.hidden, xq_sh, xs_sh, st), "quantise launch");
     if ((r = run_gate_up_fp8(h, x_perm, x_perm_scales, offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
-                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), st)) != ASAP_OK)
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), h->layer_ids,
+                             counters, st)) != ASAP_OK)
       return r;
     return run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
-                        at<float>(ws, L.hs_sh), n, y_perm, y_shared, st);
+                        at<float>(ws, L.hs_sh), n, y_perm, y_shared, h->layer_ids, counters + 1, st);
   }
-  return run_expert_ffn(h, x_perm, offsets, x, n, y_perm, y_shared, at<void>(ws, L.h), at<void>(ws, L.h_sh), st);
+  return run_expert_ffn(h, x_perm, offsets, x, n, y_perm, y_shared, at<void>(ws, L.h), at<void>(ws, L.h_sh),
+                        h->layer_ids, counters, st);
 }
 
 ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
@@ -703,7 +795,7 @@ ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const flo
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!x || !h_shared || !aligned16(x) || !aligned16(h_shared)))
     return fail(ASAP_ERR_INVALID, "x and h_shared are required for the shared expert");
-  return run_gate_up(h, x_perm, offsets, x, n, h_perm, h_shared, S(stream));
+  return run_gate_up(h, x_perm, offsets, x, n, h_perm, h_shared, h->layer_ids, nullptr, S(stream));
 }
 
 ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float* h_perm_scales,
@@ -717,7 +809,7 @@ ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float*
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!h_shared || !y_shared || !aligned16(h_shared) || !aligned16(y_shared)))
     return fail(ASAP_ERR_INVALID, "h_shared and y_shared are required for the shared expert");
-  return run_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, S(stream));
+  return run_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, h->layer_ids, nullptr, S(stream));
 }
 
 ASAP_API int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared, const float* w,
@@ -733,8 +825,11 @@ ASAP_API int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_sh
   return ASAP_OK;
 }
 
-ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_t ws_bytes,
-                            void* stream) {
+namespace {
+
+// The whole layer for one micro-batch, weights of layer *layer (device).
+int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_t ws_bytes, const int32_t* layer,
+              void* stream) {
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !out || !aligned16(x) || !aligned16(out)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
@@ -748,10 +843,11 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
   int32_t* offsets = at<int32_t>(ws, L.offsets);
   int32_t* perm_src = at<int32_t>(ws, L.perm_src);
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
+  int32_t* counters = at<int32_t>(ws, L.tile_counters);  // zeroed by the scan kernel
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
   const int splits = router_splits(h, n);
-  if ((r = run_router_logits(h, x, n, logits, splits, st)) != ASAP_OK) return r;
-  if ((r = run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, st)) != ASAP_OK) return r;
+  if ((r = run_router_logits(h, x, n, logits, splits, layer, st)) != ASAP_OK) return r;
+  if ((r = run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, layer, st)) != ASAP_OK) return r;
   if (h->fp8) {
     void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
@@ -760,11 +856,12 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
                                      h->status, st),
            "dispatch launch");
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
-                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), st)) != ASAP_OK)
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), layer, counters,
+                             st)) != ASAP_OK)
       return r;
     void* y_perm = at<void>(ws, L.y_perm);
     if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
-                          at<float>(ws, L.hs_sh), n, y_perm, y_sh, st)) != ASAP_OK)
+                          at<float>(ws, L.hs_sh), n, y_perm, y_sh, layer, counters + 1, st)) != ASAP_OK)
       return r;
     CU_TRY(asap::launch_combine(y_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
            "combine launch");
@@ -775,16 +872,16 @@ ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, v
                                perm_src, perm_dst, h->status, st),
          "dispatch launch");
   // y_perm reuses x_perm's rows: the down GEMM never reads x_perm
-  if ((r = run_expert_ffn(h, x_perm, offsets, x, n, x_perm, y_sh, at<void>(ws, L.h), at<void>(ws, L.h_sh), st)) !=
-      ASAP_OK)
+  if ((r = run_expert_ffn(h, x_perm, offsets, x, n, x_perm, y_sh, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer,
+                          counters, st)) != ASAP_OK)
     return r;
   CU_TRY(asap::launch_combine(x_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
          "combine launch");
   return ASAP_OK;
 }
 
-ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,
-                                    void* const* outs, void* ws, size_t ws_bytes, void* stream) {
+int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns, void* const* outs,
+                      void* ws, size_t ws_bytes, const int32_t* layer, void* stream) {
   if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
   if (count < 1 || count > kMaxBatch || !xs || !ns || !outs)
     return fail(ASAP_ERR_INVALID, "count must be in [1, 64] with host arrays xs, ns, outs");
@@ -813,6 +910,7 @@ ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* con
   int32_t* offsets = at<int32_t>(ws, L.offsets);
   int32_t* perm_src = at<int32_t>(ws, L.perm_src);
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
+  int32_t* counters = at<int32_t>(ws, L.tile_counters);  // zeroed by the scan kernel
   int chunks_total = 0;
   for (int i = 0; i < count; ++i) chunks_total += asap::ceil_div(ns[i], asap::kChunkTokens);
   // routing: each micro-batch exactly as asap_moe_route would route it alone
@@ -822,8 +920,8 @@ ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* con
     if (n > 0) {
       const int splits = router_splits(h, n);
       float* lg = logits + static_cast<long long>(asap::kMaxRouterSplits) * tok0 * E;
-      if ((r = run_router_logits(h, xs[i], n, lg, splits, st)) != ASAP_OK) return r;
-      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h), idx + static_cast<long long>(tok0) * k,
+      if ((r = run_router_logits(h, xs[i], n, lg, splits, layer, st)) != ASAP_OK) return r;
+      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, layer), idx + static_cast<long long>(tok0) * k,
                                    w + static_cast<long long>(tok0) * k, hist, chunk0, chunks_total, st),
              "gate launch");
     }
@@ -832,7 +930,9 @@ ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* con
   }
   // one histogram scan over every chunk: expert segments hold the rows of all
   // micro-batches, in (micro-batch, token, slot) order
-  CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, st), "scan launch");
+  CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, st,
+                           at<int32_t>(ws, L.tile_counters)),
+         "scan launch");
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
   tok0 = 0;
   chunk0 = 0;
@@ -872,17 +972,19 @@ ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* con
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n_all,
                              at<void>(ws, L.hq), at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh),
-                             st)) != ASAP_OK)
+                             layer, counters, st)) != ASAP_OK)
       return r;
     y_perm = at<void>(ws, L.y_perm);
     if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
-                          at<float>(ws, L.hs_sh), n_all, y_perm, y_sh, st)) != ASAP_OK)
+                          at<float>(ws, L.hs_sh), n_all, y_perm, y_sh, layer, counters + 1, st)) != ASAP_OK)
       return r;
   } else {
     y_perm = at<void>(ws, L.x_perm);
-    if ((r = run_gate_up(h, y_perm, offsets, y_sh, n_all, at<void>(ws, L.h), at<void>(ws, L.h_sh), st)) != ASAP_OK)
+    if ((r = run_gate_up(h, y_perm, offsets, y_sh, n_all, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer, counters,
+                         st)) != ASAP_OK)
       return r;
-    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), n_all, y_perm, y_sh, st)) != ASAP_OK)
+    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), n_all, y_perm, y_sh, layer, counters + 1,
+                      st)) != ASAP_OK)
       return r;
   }
   tok0 = 0;
@@ -897,6 +999,45 @@ ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* con
     }
     tok0 += n;
   }
+  return ASAP_OK;
+}
+
+bool valid_layer_ptr(const int32_t* layer) {
+  return layer && (reinterpret_cast<uintptr_t>(layer) & 3u) == 0;
+}
+
+}  // namespace
+
+ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_t ws_bytes,
+                            void* stream) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  return run_layer(h, x, n, out, ws, ws_bytes, h->layer_ids, stream);
+}
+
+ASAP_API int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int32_t n, void* out,
+                                void* ws, size_t ws_bytes, void* stream) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  if (!valid_layer_ptr(layer_id)) return fail(ASAP_ERR_INVALID, "layer_id must be a non-NULL 4-byte aligned device pointer");
+  return run_layer(h, x, n, out, ws, ws_bytes, layer_id, stream);
+}
+
+ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,
+                                    void* const* outs, void* ws, size_t ws_bytes, void* stream) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  return run_layer_batched(h, count, xs, ns, outs, ws, ws_bytes, h->layer_ids, stream);
+}
+
+ASAP_API int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t count, const void* const* xs,
+                                        const int32_t* ns, void* const* outs, void* ws, size_t ws_bytes,
+                                        void* stream) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  if (!valid_layer_ptr(layer_id)) return fail(ASAP_ERR_INVALID, "layer_id must be a non-NULL 4-byte aligned device pointer");
+  return run_layer_batched(h, count, xs, ns, outs, ws, ws_bytes, layer_id, stream);
+}
+
+ASAP_API int asap_moe_n_layers(asap_moe_t h, int32_t* n_layers) {
+  if (!h || !n_layers) return fail(ASAP_ERR_INVALID, "NULL handle or output");
+  *n_layers = static_cast<int32_t>(h->layers.size());
   return ASAP_OK;
 }
 
@@ -990,8 +1131,8 @@ ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int3
   // every scratch element read below is written earlier on the same stream
   // (logits by the router, all E entries of each chunk's histogram by the
   // gate kernel), so nothing has to be cleared between calls
-  if ((r = run_router_logits(h, x, n, logits, 1, st)) != ASAP_OK) return r;
-  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h), idx, w, hist, st), "gate launch");
+  if ((r = run_router_logits(h, x, n, logits, 1, h->layer_ids, st)) != ASAP_OK) return r;
+  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h, h->layer_ids), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base, st),
          "scan launch");
   return ASAP_OK;

@@ -18,6 +18,7 @@ enum : uint32_t {
   ST_BAD_POSITION = 1u << 1,      // permutation position outside [0, n*k)
   ST_WAIT_TIMEOUT = 1u << 2,      // an mbarrier wait passed its time limit
   ST_BAD_OFFSETS = 1u << 3,       // offsets not monotone or past the rows
+  ST_BAD_LAYER = 1u << 4,         // layer id outside [0, n_layers); layer 0 was used
 };
 
 __device__ __forceinline__ void record_status(uint32_t* st, uint32_t bits) {
@@ -96,6 +97,24 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* m) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
+}
+
+// A descriptor that sits in global memory (the layer table, written before the
+// launch) is read by the tensor-map proxy: the issuing thread acquires it once.
+__device__ __forceinline__ void tensormap_acquire(const CUtensorMap* m) {
+  asm volatile("fence.proxy.tensormap::generic.acquire.sys [%0], 128;" ::"l"(reinterpret_cast<uint64_t>(m))
+               : "memory");
+}
+
+// Layer id of a layer-oblivious launch (Section 3.4.2), loaded when the kernel
+// runs.  Ids outside [0, n_layers) become 0 and are recorded when ``report``.
+__device__ __forceinline__ int load_layer(const int32_t* layer, int n_layers, uint32_t* status, bool report) {
+  int l = *reinterpret_cast<const volatile int32_t*>(layer);
+  if (l < 0 || l >= n_layers) {
+    if (report) record_status(status, ST_BAD_LAYER);
+    l = 0;
+  }
+  return l;
 }
 
 // 2-D tiled load of one box into shared memory; completes on ``bar`` with the

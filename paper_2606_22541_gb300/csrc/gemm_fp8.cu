@@ -48,10 +48,12 @@ constexpr uint32_t kTmemCols = 2 * BN;          // two partial buffers
 // both K-major, N >> 3 in bits 17-22, M >> 4 in bits 24-28.
 constexpr uint32_t kIdescF8 = (1u << 4) | (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
 
-constexpr int kBarBytes = 256;
+constexpr int kBarBytes = 384;
 constexpr size_t kSmemBytes = 1024 + SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 4 * BM * sizeof(float);
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-static_assert(8 * (2 * SA + 2 * SB + 7) + 8 <= kBarBytes, "barrier area");
+static_assert(8 * (2 * SA + 2 * SB + 7) + kTileQBytes + 12 <= kBarBytes, "barrier area");
+// consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
+constexpr int kTileQConsumers = 2 + kEpiWarps;
 
 __device__ __forceinline__ void tc_mma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t accumulate) {
   asm volatile(
@@ -87,8 +89,7 @@ __device__ __forceinline__ void promote32(float* acc, uint32_t taddr, float s) {
 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-    grouped_gemm_fp8_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
-                            const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+    grouped_gemm_fp8_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                             const Fp8Args fa) {
   const GemmArgs& args = fa.g;
   extern __shared__ uint8_t smem_raw[];
@@ -108,17 +109,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t drain_bar = bar0 + 8u * (2 * SA + 2 * SB + 4);
   // amax exchange between the two epilogue halves of a row (per tile parity)
   auto xchg = [&](int b) { return bar0 + 8u * (2 * SA + 2 * SB + 5 + b); };
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 7));
+  const uint32_t tq_base = bar0 + 8u * (2 * SA + 2 * SB + 7);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 7) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* layer_slot = reinterpret_cast<int*>(tmem_slot + 2);  // layer id, shared with the epilogue
   Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
   float* amax_x = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sch) + sizeof(Sched));  // [2][4][BM]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int G = args.offsets ? args.groups : 1;
+  // weight descriptors of this launch's layer (read by the B producer)
+  const CUtensorMap* tmB0 = nullptr;
+  const CUtensorMap* tmB1 = nullptr;
 
   if (warp == 0) {
     if (lane == 0) {
+      const int l = load_layer(args.lref.layer, args.lref.n_layers, args.status, blockIdx.x == 0);
+      *layer_slot = l;
+      tmB0 = &args.lref.table[l].map[args.bmap0];
+      tmB1 = &args.lref.table[l].map[args.bmap1];
+      tensormap_acquire(tmB0);
+      if (args.m1 > 0) tensormap_acquire(tmB1);
       for (int s = 0; s < SA; ++s) {
         mbar_init(fullA(s), 1);
         mbar_init(emptyA(s), 1);
@@ -134,13 +146,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(drain_bar, 1);
       mbar_init(xchg(0), kEpiWarps * 32);
       mbar_init(xchg(1), kEpiWarps * 32);
+      TileQueue{tq_base}.init(kTileQConsumers);
       *abort_flag = 0;
       fence_barrier_init();
       tma_prefetch_desc(&tmA0);
-      tma_prefetch_desc(&tmB0);
+      tma_prefetch_desc(tmB0);
       if (args.m1 > 0) {
         tma_prefetch_desc(&tmA1);
-        tma_prefetch_desc(&tmB1);
+        tma_prefetch_desc(tmB1);
       }
     }
     build_schedule(args, sch, G, lane);
@@ -154,6 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int total0 = sch->tile_start[G];
   const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+  TileQueue tq{tq_base};
 
   if ((warp == 0 || warp == kAProdWarp) && lane == 0) {
     // ------------------------------------------------------------ producers
@@ -166,10 +180,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     uint32_t pending = 0, issued_phase = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    int t = blockIdx.x;
+    while (ok) {
+      int cur;
+      if (isB) {  // warp 0 claims the tiles
+        cur = t < total ? t : -1;
+        if (!tq.push(cur, abort_flag)) {
+          ok = false;
+          break;
+        }
+        if (cur >= 0) t = next_tile(args, cur);
+      } else if (!tq.pop(cur, abort_flag, true)) {
+        ok = false;
+        break;
+      }
+      if (cur < 0) break;
       Tile T;
-      decode_tile(t, sch, G, total0, args, T);
-      const CUtensorMap* m = isB ? (T.p1 ? &tmB1 : &tmB0) : (T.p1 ? &tmA1 : &tmA0);
+      decode_tile(cur, sch, G, total0, args, T);
+      const CUtensorMap* m = isB ? (T.p1 ? tmB1 : tmB0) : (T.p1 ? &tmA1 : &tmA0);
       const int row = isB ? T.b_row : T.a_row;
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
         const uint32_t full = isB ? fullB(stage) : fullA(stage);
@@ -200,7 +228,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t pa = 0, pb = 0;
     uint32_t kc = 0;  // K blocks issued by this CTA (partial-buffer ping-pong)
     bool ok = true, issued = false;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    while (ok) {
+      int t;
+      if (!tq.pop(t, abort_flag, true)) {
+        ok = false;
+        break;
+      }
+      if (t < 0) break;
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
       for (int kb = T.kb0; kb < T.kb1; ++kb, ++kc) {
@@ -251,9 +285,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = q * 32 + lane;
     const uint32_t lane_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
     uint32_t kc = 0;
-    int it = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+    for (int it = 0; ok; ++it) {
+      int t = -1;
+      const uint32_t qslot = tq.slot();
+      if (!__all_sync(0xffffffffu, tq.pop(t, abort_flag, false))) {
+        if (lane == 0) {
+          *abort_flag = 1;
+          record_status(args.status, ST_WAIT_TIMEOUT);
+        }
+        break;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tq.empty(qslot));
+      if (t < 0) break;
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
       const int mrows = T.p1 ? args.m1 : args.m0;
@@ -262,7 +307,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int asld = T.p1 ? fa.a_sld1 : fa.a_sld0;
       const float* arow = (T.p1 ? fa.a_scale1 : fa.a_scale0) + srow * asld;
       const int nblk = T.p1 ? fa.b_nblk1 : fa.b_nblk0;
-      const float* bs = (T.p1 ? fa.b_scale1 : fa.b_scale0) + static_cast<long long>(T.group) * nblk * asld;
+      // B scales of this layer (looked up per tile: no registers held across tiles)
+      const float* bs = args.lref.table[*layer_slot].scale[T.p1 ? args.bmap1 : args.bmap0] +
+                        static_cast<long long>(T.group) * nblk * asld;
       // scale rows of this warp's columns: SwiGLU tiles hold gate block nt
       // (scale row 2nt) and up block nt (2nt+1); plain tiles blocks 2nt, 2nt+1
       const int lo_blk = EPI == EPI_SWIGLU ? 0 : (cq * kCols) / 128;
@@ -419,11 +466,9 @@ cudaError_t fp8_gemm_set_attributes() {
 cudaError_t fp8_gemm_launch(int epi, const CUtensorMap* maps, const Fp8Args& args, int grid, cudaStream_t stream) {
   if (grid <= 0) return cudaSuccess;
   if (epi == EPI_SWIGLU)
-    grouped_gemm_fp8_kernel<EPI_SWIGLU><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3],
-                                                                                 args);
+    grouped_gemm_fp8_kernel<EPI_SWIGLU><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], args);
   else
-    grouped_gemm_fp8_kernel<EPI_BF16><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3],
-                                                                               args);
+    grouped_gemm_fp8_kernel<EPI_BF16><<<grid, kThreads, kSmemBytes, stream>>>(maps[0], maps[1], args);
   return cudaGetLastError();
 }
 

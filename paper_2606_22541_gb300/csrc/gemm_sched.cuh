@@ -20,6 +20,62 @@ struct Tile {
   bool p1;
 };
 
+// ------------------------------------------------------------ tile queue
+// Which tiles a CTA computes is decided while the launch runs: the B producer
+// takes tile blockIdx.x first, then claims the next unclaimed tile from a
+// global counter (args.tile_counter, zero when the launch starts; without one
+// the order is static, blockIdx.x + i * gridDim.x).  A CTA that starts late
+// because its SM was busy with another kernel then simply takes fewer tiles,
+// instead of running its share after everyone else.  Claimed ids reach the
+// other roles of the CTA through a ring of kTileQ shared-memory slots guarded
+// by mbarriers; id -1 ends every role's loop.
+constexpr int kTileQ = 4;
+// Shared-memory bytes of the queue: kTileQ full and kTileQ empty mbarriers,
+// then kTileQ int slots.
+constexpr int kTileQBytes = 20 * kTileQ;
+
+struct TileQueue {
+  uint32_t full0;  // shared address of the queue (8-byte aligned)
+  uint32_t n = 0;  // ids this thread has pushed or popped
+
+  __device__ __forceinline__ uint32_t slot() const { return n % kTileQ; }
+  __device__ __forceinline__ uint32_t phase() const { return (n / kTileQ) & 1u; }
+  __device__ __forceinline__ uint32_t full(uint32_t s) const { return full0 + 8u * s; }
+  __device__ __forceinline__ uint32_t empty(uint32_t s) const { return full0 + 8u * (kTileQ + s); }
+  __device__ __forceinline__ uint32_t id_addr(uint32_t s) const { return full0 + 16u * kTileQ + 4u * s; }
+
+  __device__ __forceinline__ void init(int consumers) const {
+    for (uint32_t s = 0; s < kTileQ; ++s) {
+      mbar_init(full(s), 1);
+      mbar_init(empty(s), consumers);
+    }
+  }
+  // producer: publish the next tile id (or -1)
+  __device__ __forceinline__ bool push(int t, volatile int* abort_flag) {
+    const uint32_t s = slot();
+    if (!mbar_wait(empty(s), phase() ^ 1u, abort_flag)) return false;
+    asm volatile("st.shared.b32 [%0], %1;" ::"r"(id_addr(s)), "r"(t) : "memory");
+    mbar_arrive(full(s));
+    ++n;
+    return true;
+  }
+  // consumer: read the next tile id; ``release`` arrives on the slot's empty
+  // barrier (one arrival per consuming thread or warp, as initialised)
+  __device__ __forceinline__ bool pop(int& t, volatile int* abort_flag, bool release) {
+    const uint32_t s = slot();
+    if (!mbar_wait(full(s), phase(), abort_flag)) return false;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(t) : "r"(id_addr(s)) : "memory");
+    if (release) mbar_arrive(empty(s));
+    ++n;
+    return true;
+  }
+};
+
+// The tile after t for this CTA.
+__device__ __forceinline__ int next_tile(const GemmArgs& a, int t) {
+  return a.tile_counter ? static_cast<int>(gridDim.x) + atomicAdd(a.tile_counter, 1) : t + static_cast<int>(gridDim.x);
+}
+
 // Tile t of the launch: problem 0 groups in order (inside a group: K slice,
 // then n-tile, then m-tile innermost), then problem 1 (n-tile, m-tile).
 __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int total0,

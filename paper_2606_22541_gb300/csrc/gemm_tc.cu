@@ -19,6 +19,9 @@
 //   warps 2-5: epilogue.  tcgen05.ld 32x32b (warp w reads TMEM lanes
 //              32*(w%4) ...), fused SwiGLU (gate and up columns of a tile are
 //              the two 128-column halves), bf16 or fp32 store.
+// Weights: the B descriptors come from the layer table (one entry per layer,
+// in global memory) at the layer id the kernel loads when it starts, so one
+// launch sequence serves any layer (the MoE Super Kernel of Section 3.4.2).
 // Tile order: expert-major; inside an expert the m-tiles of one n-tile are
 // adjacent so CTAs running at the same time share the weight tile through L2.
 // Rows of a tile past the segment end belong to the next expert (or are
@@ -55,7 +58,7 @@ constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
 
-constexpr int kBarBytes = 256;  // 2*SA + 2*SB + 5 mbarriers, tmem slot, abort flag
+constexpr int kBarBytes = 384;  // 2*SA + 2*SB + 5 + 2*kTileQ mbarriers, tmem slot, abort flag, tile ids
 template <int EPI>
 __host__ __device__ constexpr size_t smem_bytes() {
   return 1024 + Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
@@ -137,11 +140,9 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
-                        const __grid_constant__ CUtensorMap tmB0,
-                        const __grid_constant__ CUtensorMap tmA1,
-                        const __grid_constant__ CUtensorMap tmB1, const GemmArgs args) {
+                        const __grid_constant__ CUtensorMap tmA1, const GemmArgs args) {
   constexpr int SA = Rings<EPI>::A, SB = Rings<EPI>::B;
-  static_assert(8 * (2 * SA + 2 * SB + 5) + 8 <= kBarBytes, "barrier area");
+  static_assert(8 * (2 * SA + 2 * SB + 5) + kTileQBytes + 8 <= kBarBytes, "barrier area");
   static_assert(smem_bytes<EPI>() <= 227 * 1024, "shared memory budget");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -152,7 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;
   const uint32_t bar0 = smem_u32(bar_area);
   // mbarriers (8 bytes each): fullA[SA], emptyA[SA], fullB[SB], emptyB[SB],
-  // tfull[2], tempty[2], drain
+  // tfull[2], tempty[2], drain, tile queue full[kTileQ], empty[kTileQ]
   auto fullA = [&](int s) { return bar0 + 8u * s; };
   auto emptyA = [&](int s) { return bar0 + 8u * (SA + s); };
   auto fullB = [&](int s) { return bar0 + 8u * (2 * SA + s); };
@@ -160,16 +161,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * SA + 2 * SB + a); };
   auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * SA + 2 * SB + 2 + a); };
   const uint32_t drain_bar = bar0 + 8u * (2 * SA + 2 * SB + 4);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5));
+  const uint32_t tq_base = bar0 + 8u * (2 * SA + 2 * SB + 5);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
+  // consumers of each queued tile id: A producer, MMA issuer, 4 epilogue warps
+  constexpr int kTileQConsumers = 6;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int G = args.offsets ? args.groups : 1;
+  // weight descriptors of this launch's layer (only the B producer reads them)
+  const CUtensorMap* tmB0 = nullptr;
+  const CUtensorMap* tmB1 = nullptr;
 
   if (warp == 0) {
     if (lane == 0) {
+      const LayerEntry& le =
+          args.lref.table[load_layer(args.lref.layer, args.lref.n_layers, args.status, blockIdx.x == 0)];
+      tmB0 = &le.map[args.bmap0];
+      tmB1 = &le.map[args.bmap1];
+      tensormap_acquire(tmB0);
+      if (args.m1 > 0) tensormap_acquire(tmB1);
       for (int s = 0; s < SA; ++s) {
         mbar_init(fullA(s), 1);
         mbar_init(emptyA(s), 1);
@@ -183,13 +196,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(tempty_bar(a), 128);
       }
       mbar_init(drain_bar, 1);
+      TileQueue{tq_base}.init(kTileQConsumers);
       *abort_flag = 0;
       fence_barrier_init();
       tma_prefetch_desc(&tmA0);
-      tma_prefetch_desc(&tmB0);
+      tma_prefetch_desc(tmB0);
       if (args.m1 > 0) {
         tma_prefetch_desc(&tmA1);
-        tma_prefetch_desc(&tmB1);
+        tma_prefetch_desc(tmB1);
       }
     }
     build_schedule(args, sch, G, lane);
@@ -203,11 +217,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int total0 = sch->tile_start[G];
   const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+  TileQueue tq{tq_base};
 
   if ((warp == 0 || warp == 6) && lane == 0) {
     // ------------------------------------------------------------ producers
-    // warp 0 streams the weight tiles (B) into its ring, warp 6 the
-    // activation tiles (A) into its own; the MMA issuer joins them per k-step.
+    // warp 0 claims the tiles and streams their weight boxes (B) into its
+    // ring, warp 6 the activation boxes (A) into its own; the MMA issuer joins
+    // them per k-step.
     const bool isB = warp == 0;
     const int nst = isB ? SB : SA;
     const uint32_t bytes = isB ? B_BYTES : A_BYTES;
@@ -217,10 +233,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     uint32_t pending = 0, issued_phase = 0;  // bit s: stage s has a load in flight
     bool ok = true;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    int t = blockIdx.x;
+    while (ok) {
+      int cur;
+      if (isB) {
+        cur = t < total ? t : -1;
+        if (!tq.push(cur, abort_flag)) {
+          ok = false;
+          break;
+        }
+        if (cur >= 0) t = next_tile(args, cur);  // claimed now, used after this tile's loads
+      } else if (!tq.pop(cur, abort_flag, true)) {
+        ok = false;
+        break;
+      }
+      if (cur < 0) break;
       Tile T;
-      decode_tile(t, sch, G, total0, args, T);
-      const CUtensorMap* m = isB ? (T.p1 ? &tmB1 : &tmB0) : (T.p1 ? &tmA1 : &tmA0);
+      decode_tile(cur, sch, G, total0, args, T);
+      const CUtensorMap* m = isB ? (T.p1 ? tmB1 : tmB0) : (T.p1 ? &tmA1 : &tmA0);
       const int row = isB ? T.b_row : T.a_row;
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
         const uint32_t full = isB ? fullB(stage) : fullA(stage);
@@ -251,8 +281,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     int sa = 0, sb = 0;
     uint32_t pa = 0, pb = 0;
     bool ok = true, issued = false;
-    int it = 0;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+    for (int it = 0; ok; ++it) {
+      int t;
+      if (!tq.pop(t, abort_flag, true)) {
+        ok = false;
+        break;
+      }
+      if (t < 0) break;
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
       const int acc = it & 1;
@@ -304,8 +339,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    int it = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      int t = -1;
+      const uint32_t qslot = tq.slot();
+      if (!__all_sync(0xffffffffu, tq.pop(t, abort_flag, false))) {
+        if (lane == 0) {
+          *abort_flag = 1;
+          record_status(args.status, ST_WAIT_TIMEOUT);
+        }
+        break;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tq.empty(qslot));
+      if (t < 0) break;
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
       const int acc = it & 1;
@@ -376,13 +422,13 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, 
   const dim3 g(grid), b(kThreads);
   switch (epi) {
     case EPI_SWIGLU:
-      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, smem_bytes<EPI_SWIGLU>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, smem_bytes<EPI_SWIGLU>(), stream>>>(maps[0], maps[1], args);
       break;
     case EPI_BF16:
-      grouped_gemm_kernel<EPI_BF16><<<g, b, smem_bytes<EPI_BF16>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_BF16><<<g, b, smem_bytes<EPI_BF16>(), stream>>>(maps[0], maps[1], args);
       break;
     default:
-      grouped_gemm_kernel<EPI_F32><<<g, b, smem_bytes<EPI_F32>(), stream>>>(maps[0], maps[1], maps[2], maps[3], args);
+      grouped_gemm_kernel<EPI_F32><<<g, b, smem_bytes<EPI_F32>(), stream>>>(maps[0], maps[1], args);
       break;
   }
   return cudaGetLastError();

@@ -19,6 +19,29 @@ namespace asap {
 // C = A B^T with A [rows, K] and B [N, K] both K-major bf16.
 enum { EPI_SWIGLU = 0, EPI_BF16 = 1, EPI_F32 = 2 };
 
+// ------------------------------------------------------------ layer table
+// The layer-oblivious kernels of Section 3.4.2: every weight a kernel reads is
+// found through a device array with one entry per layer, indexed by a layer id
+// the kernel loads from device memory when it runs.  The entry holds the TMA
+// descriptors of that layer's packed weights (the pre-computed addresses) and
+// plain pointers for what is not read by TMA.
+enum { MAP_ROUTER = 0, MAP_GATE_UP = 1, MAP_DOWN = 2, MAP_SH_GATE_UP = 3, MAP_SH_DOWN = 4, kLayerMaps = 5 };
+
+struct alignas(128) LayerEntry {
+  CUtensorMap map[kLayerMaps];     // indexed by MAP_*; unused maps are zero
+  const float* scale[kLayerMaps];  // FP8 block scales of the same matrices, else nullptr
+  const void* router_w;            // [E, H] bf16
+  const float* router_bias;        // [E] fp32 or nullptr
+};
+
+// Which entry a launch uses: table[*layer].  An id outside [0, n_layers) is
+// recorded as ST_BAD_LAYER and replaced by 0, so no access leaves the table.
+struct LayerRef {
+  const LayerEntry* table;  // device [n_layers]
+  const int32_t* layer;     // device int32, read by the kernel
+  int n_layers;
+};
+
 struct GemmArgs {
   const int32_t* offsets;  // [groups + 1] or nullptr
   int groups;              // 1 when offsets == nullptr
@@ -37,8 +60,12 @@ struct GemmArgs {
   int hint_a, hint_b;      // L2 priority of A / B loads: 0 normal, 1 first, 2 last
   int k_splits;            // problem 0 split into this many K slices (>= 1)
   long long split_rows0;   // output rows between the planes of consecutive K slices
+  LayerRef lref;           // B of problem p is lref.table[layer].map[bmap_p]
+  int bmap0, bmap1;
+  int* tile_counter;       // zero at launch: tiles are claimed dynamically; nullptr: static order
 };
 
+constexpr int kTileCounters = 2;  // per call: gate/up GEMM, down GEMM
 constexpr int kGemmBM = 128;
 constexpr int kGemmBN = 256;
 #ifndef ASAP_GEMM_BK
@@ -47,7 +74,8 @@ constexpr int kGemmBN = 256;
 constexpr int kGemmBK = ASAP_GEMM_BK;  // 64 (128-byte swizzle) or 32 (64-byte swizzle)
 
 cudaError_t gemm_set_attributes();
-// maps: A0, B0, A1, B1 (A1/B1 may repeat A0/B0 when m1 == 0)
+// maps: A0, A1 (A1 may repeat A0 when m1 == 0); the B maps come from the
+// layer table.
 cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, int grid,
                         cudaStream_t stream);
 // Encode a 2-D row-major bf16 tensor [rows, cols] for 128-byte-swizzled
@@ -70,8 +98,8 @@ struct Fp8Args {
   const float* a_scale0;  // [m0][a_sld0]
   const float* a_scale1;  // [m1][a_sld1]
   int a_sld0, a_sld1;     // K/128
-  const float* b_scale0;  // [groups][b_nblk0][a_sld0]
-  const float* b_scale1;  // [b_nblk1][a_sld1]
+  // B scales: table[layer].scale[bmap_p], [groups][b_nblk0][a_sld0] for
+  // problem 0 and [b_nblk1][a_sld1] for problem 1
   int b_nblk0, b_nblk1;   // N/128
   float* out_scale0;      // EPI_SWIGLU only: [m0][o_sld0]
   float* out_scale1;
@@ -93,10 +121,12 @@ cudaError_t launch_quantize_rows(const void* x, int rows, int cols, void* q, flo
 struct GateParams {
   int n_experts, top_k, gating, n_groups, topk_groups;
   float route_scale;
-  const float* bias;  // [E] or nullptr
+  LayerRef lref;  // selection bias: table[layer].router_bias ([E] or nullptr)
+  uint32_t* status;
 };
-cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int E, float* logits,
-                                cudaStream_t s);
+// Router on the CUDA cores (E < 256): weights table[layer].router_w.
+cudaError_t launch_router_small(const void* x, const LayerRef& lref, int n, int H, int E, float* logits,
+                                uint32_t* status, cudaStream_t s);
 // logits: ``splits`` planes of [n, E] partial sums, added in plane order.
 // hist is written expert-major: hist[e * n_chunks + chunk].
 cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
@@ -109,8 +139,10 @@ cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GatePa
                             int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s);
 cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
                         cudaStream_t s);
+// tile_counters (nullable): kTileCounters ints zeroed for the grouped GEMMs
+// that follow on the stream.
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
-                        int32_t* chunk_base, cudaStream_t s);
+                        int32_t* chunk_base, cudaStream_t s, int32_t* tile_counters = nullptr);
 
 // ------------------------------------------------------------ permute
 // Place of one micro-batch among several served by one call: its chunks start

@@ -25,12 +25,14 @@ constexpr unsigned kFull = 0xffffffffu;
 // fixed reduction order (per-lane strided partial sums, then a butterfly).
 constexpr int kRouterEB = 16;  // experts per pass
 
-__global__ void __launch_bounds__(256) router_small_kernel(const uint4* __restrict__ x,
-                                                           const uint4* __restrict__ wr, int n,
-                                                           int V, int E, float* __restrict__ logits) {
+__global__ void __launch_bounds__(256) router_small_kernel(const uint4* __restrict__ x, LayerRef lref,
+                                                           uint32_t* status, int n, int V, int E,
+                                                           float* __restrict__ logits) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int t = blockIdx.x * 8 + warp;
   if (t >= n) return;
+  const uint4* __restrict__ wr = static_cast<const uint4*>(
+      lref.table[load_layer(lref.layer, lref.n_layers, status, t == 0 && lane == 0)].router_w);
   const uint4* xr = x + static_cast<long long>(t) * V;
   for (int e0 = 0; e0 < E; e0 += kRouterEB) {
     float acc[kRouterEB];
@@ -105,6 +107,11 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
   const int t1 = min(n, t0 + kChunkTokens);
   const bool grouped = p.gating == 2;
   const int gsz = grouped ? E / p.n_groups : E;
+  // selection bias of this launch's layer
+  const float* __restrict__ bias =
+      grouped ? p.lref.table[load_layer(p.lref.layer, p.lref.n_layers, p.status, threadIdx.x == 0 && blockIdx.x == 0)]
+                    .router_bias
+              : nullptr;
 
   for (int t = t0 + warp; t < t1; t += kGateWarps) {
     const float* lrow = logits + static_cast<long long>(t) * E;
@@ -120,7 +127,7 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
       if (grouped) {
         const float s = 1.0f / (1.0f + expf(-l));
         sv[i] = s;
-        key[i] = e < E ? s + (p.bias ? p.bias[e] : 0.0f) : -CUDART_INF_F;
+        key[i] = e < E ? s + (bias ? bias[e] : 0.0f) : -CUDART_INF_F;
       } else {
         sv[i] = l;
         key[i] = l;
@@ -277,10 +284,13 @@ __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ i
 __global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ hist, int n_chunks, int E,
                                                     int32_t* __restrict__ counts,
                                                     int32_t* __restrict__ offsets,
-                                                    int32_t* __restrict__ chunk_base) {
+                                                    int32_t* __restrict__ chunk_base,
+                                                    int32_t* __restrict__ tile_counters) {
   __shared__ int scount[kMaxExperts];
   __shared__ int soff[kMaxExperts + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the grouped GEMMs that follow on this stream claim tiles from these
+  if (tile_counters && threadIdx.x < kTileCounters) tile_counters[threadIdx.x] = 0;
   for (int e = warp; e < E; e += 32) {
     const int32_t* hrow = hist + static_cast<long long>(e) * n_chunks;
     int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
@@ -350,11 +360,11 @@ __global__ void reduce_splits_kernel(const float* __restrict__ parts, int splits
 
 }  // namespace
 
-cudaError_t launch_router_small(const void* x, const void* wr, int n, int H, int E, float* logits,
-                                cudaStream_t s) {
+cudaError_t launch_router_small(const void* x, const LayerRef& lref, int n, int H, int E, float* logits,
+                                uint32_t* status, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  router_small_kernel<<<ceil_div(n, 8), 256, 0, s>>>(static_cast<const uint4*>(x),
-                                                       static_cast<const uint4*>(wr), n, H / 8, E, logits);
+  router_small_kernel<<<ceil_div(n, 8), 256, 0, s>>>(static_cast<const uint4*>(x), lref, status, n, H / 8, E,
+                                                       logits);
   return cudaGetLastError();
 }
 
@@ -388,8 +398,8 @@ cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane
 }
 
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
-                        int32_t* chunk_base, cudaStream_t s) {
-  scan_kernel<<<1, 1024, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base);
+                        int32_t* chunk_base, cudaStream_t s, int32_t* tile_counters) {
+  scan_kernel<<<1, 1024, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters);
   return cudaGetLastError();
 }
 

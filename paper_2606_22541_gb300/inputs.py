@@ -107,6 +107,18 @@ def make_weights(cfg, device):
     return w
 
 
+def layer_config(cfg, layer):
+    """The configuration whose make_weights draws layer ``layer`` of a model
+    with several MoE layers of cfg's shape (layer 0 is cfg itself)."""
+    from dataclasses import replace
+    return cfg if layer == 0 else replace(cfg, seed=cfg.seed + 7919 * layer)
+
+
+def make_layer_weights(cfg, n_layers, device):
+    """Weights of layers 0 .. n_layers-1, one make_weights dict per layer."""
+    return [make_weights(layer_config(cfg, layer), device) for layer in range(n_layers)]
+
+
 def expert_weights_bf16(cfg, e, device):
     """(Wg_e [I, H], Wu_e [I, H], Wd_e [H, I]) of one routed expert, the same
     values make_weights draws for it (bf16 configurations)."""

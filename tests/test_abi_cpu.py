@@ -87,3 +87,18 @@ def test_calls_reject_null_handle(L):
     assert L.asap_moe_layer(None, None, 1, None, None, 0, None) == _native.ASAP_ERR_INVALID
     assert L.asap_moe_combine(None, None, None, None, None, 1, None, None) == _native.ASAP_ERR_INVALID
     assert L.asap_moe_status(None, None) == _native.ASAP_ERR_INVALID
+
+
+def test_create_layers_rejects_bad_layer_counts_before_touching_cuda(L):
+    c = api.make_config(TINY, 16)
+    ws = (_native.AsapMoeWeights * 2)()
+    out = ctypes.c_void_p(1234)
+    for n in (0, -1, 5000):
+        assert L.asap_moe_create_layers(ctypes.byref(c), ws, n, ctypes.byref(out)) == _native.ASAP_ERR_INVALID
+        assert out.value is None
+    assert L.asap_moe_create_layers(ctypes.byref(c), ws, 2, ctypes.byref(out)) == _native.ASAP_ERR_INVALID
+    assert "layer 0" in api.asap_moe_last_error()
+    assert L.asap_moe_layer_dyn(None, None, None, 1, None, None, 0, None) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_layer_batched_dyn(None, None, 1, None, None, None, None, 0, None) == _native.ASAP_ERR_INVALID
+    n = ctypes.c_int32(0)
+    assert L.asap_moe_n_layers(None, ctypes.byref(n)) == _native.ASAP_ERR_INVALID
