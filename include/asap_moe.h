@@ -327,7 +327,8 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
  * raw status word (0 = clean) to *word if non-NULL, then clear it.  Bits:
  * 1 expert index outside [0, E); 2 permutation position out of range;
  * 4 a wait passed its time limit; 8 offsets not monotone or past the rows;
- * 16 layer id outside [0, n_layers). */
+ * 16 layer id outside [0, n_layers); 32 a grouped GEMM found its dynamic
+ * shared memory misaligned and did nothing. */
 int asap_moe_status(asap_moe_t h, uint32_t* word);
 
 /* Thread-local text of this thread's last failure ("" if none). */

@@ -19,6 +19,7 @@ enum : uint32_t {
   ST_WAIT_TIMEOUT = 1u << 2,      // an mbarrier wait passed its time limit
   ST_BAD_OFFSETS = 1u << 3,       // offsets not monotone or past the rows
   ST_BAD_LAYER = 1u << 4,         // layer id outside [0, n_layers); layer 0 was used
+  ST_SMEM_ALIGN = 1u << 5,        // dynamic shared memory not 1024-byte aligned; the GEMM did nothing
 };
 
 __device__ __forceinline__ void record_status(uint32_t* st, uint32_t bits) {

@@ -49,7 +49,8 @@ constexpr uint32_t kTmemCols = 2 * BN;          // two partial buffers
 constexpr uint32_t kIdescF8 = (1u << 4) | (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
 
 constexpr int kBarBytes = 384;
-constexpr size_t kSmemBytes = 1024 + SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 4 * BM * sizeof(float);
+// rings first (1024-byte aligned, declared and checked), then barriers, schedule, amax exchange
+constexpr size_t kSmemBytes = SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 4 * BM * sizeof(float);
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(8 * (2 * SA + 2 * SB + 7) + kTileQBytes + 12 <= kBarBytes, "barrier area");
 // consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
@@ -92,10 +93,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_fp8_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                             const Fp8Args fa) {
   const GemmArgs& args = fa.g;
-  extern __shared__ uint8_t smem_raw[];
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = (raw + 1023u) & ~1023u;
-  uint8_t* gbase = smem_raw + (base - raw);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t base = smem_u32(smem_raw);
+  if (base & 1023u) {  // uniform for the CTA: nothing is initialised yet
+    if (threadIdx.x == 0) record_status(args.status, ST_SMEM_ALIGN);
+    return;
+  }
+  uint8_t* gbase = smem_raw;
   const uint32_t sA = base;
   const uint32_t sB = base + SA * A_BYTES;
   uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;

@@ -8,11 +8,11 @@
 
 namespace asap {
 
+// Per-group tile starts and row segments of problem 0 (group g: rows
+// [row_base[g], row_base[g+1]), tiles [tile_start[g], tile_start[g+1])).
 struct Sched {
   int tile_start[kMaxExperts + 1];
-  int mtiles[kMaxExperts];
-  int row_base[kMaxExperts];
-  int mrows[kMaxExperts];
+  int row_base[kMaxExperts + 1];
 };
 
 struct Tile {
@@ -88,14 +88,16 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
     }
     const int g = lo;
     int local = t - s->tile_start[g];
-    const int mt = s->mtiles[g];
+    const int r0 = s->row_base[g];
+    const int mrows = s->row_base[g + 1] - r0;
+    const int mt = (mrows + kGemmBM - 1) / kGemmBM;
     const int per_split = mt * a.n_tiles0;
     const int split = local / per_split;   // K slice (split-K of problem 0)
     local -= split * per_split;
     const int nt = local / mt;
     const int mi = local - nt * mt;
-    T.a_row = s->row_base[g] + mi * kGemmBM;
-    T.rows = min(kGemmBM, s->mrows[g] - mi * kGemmBM);
+    T.a_row = r0 + mi * kGemmBM;
+    T.rows = min(kGemmBM, mrows - mi * kGemmBM);
     T.b_row = g * a.b_stride0 + nt * kGemmBN;
     T.n_tile = nt;
     T.split = split;
@@ -122,52 +124,58 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
 
 // Warp-level construction of the schedule table (called by one full warp):
 // per-group m-tile counts and their exclusive prefix; each lane owns up to 8
-// consecutive groups.  Offsets that are not monotone or run past the rows
-// make the group empty and are reported in the status word.
+// consecutive groups.  Offsets that are negative, not monotone or run past
+// the rows are reported in the status word and leave problem 0 empty.
 __device__ __forceinline__ void build_schedule(const GemmArgs& args, Sched* sch, int G, int lane) {
-    // Per-group m-tile counts and their exclusive prefix (warp scan; each
-    // lane owns up to 8 consecutive groups).  Bad offsets -> empty group.
-    int local = 0;
-    int cnt[8];
+  int local = 0;
+  int cnt[8];
+  int lo[8];
+  bool bad = false;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int g = lane * 8 + i;
-      cnt[i] = 0;
-      if (g < G) {
-        int lo = 0, m = args.m0;
-        if (args.offsets) {
-          lo = __ldg(args.offsets + g);
-          const int hi = __ldg(args.offsets + g + 1);
-          m = hi - lo;
-          if (lo < 0 || m < 0 || hi > args.m0) {
-            record_status(args.status, ST_BAD_OFFSETS);
-            lo = 0;
-            m = 0;
-          }
-        }
-        sch->row_base[g] = lo;
-        sch->mrows[g] = m;
-        cnt[i] = (m + kGemmBM - 1) / kGemmBM;
-        sch->mtiles[g] = cnt[i];
-        local += cnt[i] * args.n_tiles0 * args.k_splits;
+  for (int i = 0; i < 8; ++i) {
+    const int g = lane * 8 + i;
+    cnt[i] = 0;
+    lo[i] = 0;
+    if (g < G) {
+      int m = args.m0;
+      if (args.offsets) {
+        lo[i] = __ldg(args.offsets + g);
+        const int hi = __ldg(args.offsets + g + 1);
+        m = hi - lo[i];
+        bad |= lo[i] < 0 || m < 0 || hi > args.m0;
       }
+      cnt[i] = (max(m, 0) + kGemmBM - 1) / kGemmBM;
+      local += cnt[i] * args.n_tiles0 * args.k_splits;
     }
-    int incl = local;
+  }
+  if (__any_sync(0xffffffffu, bad)) {
+    if (lane == 0) record_status(args.status, ST_BAD_OFFSETS);
+    for (int g = lane; g <= G; g += 32) {
+      sch->tile_start[g] = 0;
+      sch->row_base[g] = 0;
+    }
+    return;
+  }
+  int incl = local;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    int run = incl - local;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  int run = incl - local;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int g = lane * 8 + i;
-      if (g < G) {
-        sch->tile_start[g] = run;
-        run += cnt[i] * args.n_tiles0 * args.k_splits;
-      }
+  for (int i = 0; i < 8; ++i) {
+    const int g = lane * 8 + i;
+    if (g < G) {
+      sch->tile_start[g] = run;
+      sch->row_base[g] = lo[i];
+      run += cnt[i] * args.n_tiles0 * args.k_splits;
     }
-    if (lane == 31) sch->tile_start[G] = incl;
+  }
+  if (lane == 31) {
+    sch->tile_start[G] = incl;
+    sch->row_base[G] = args.offsets ? __ldg(args.offsets + G) : args.m0;
+  }
 }
 
 }  // namespace asap

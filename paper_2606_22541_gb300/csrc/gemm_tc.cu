@@ -44,10 +44,22 @@ namespace {
 // are still in L2 from the gate/up launch, so its weight ring gets 5 stages
 // and its activation ring 3 (measured on GB300: 1.84 -> 1.73 ms per launch at
 // 4096 DeepSeek-V3 tokens, while 3 + 5 would slow the gate/up GEMM by 15 %).
+#ifndef ASAP_RING_GU_A
+#define ASAP_RING_GU_A 4
+#endif
+#ifndef ASAP_RING_GU_B
+#define ASAP_RING_GU_B 4
+#endif
+#ifndef ASAP_RING_DN_A
+#define ASAP_RING_DN_A 3
+#endif
+#ifndef ASAP_RING_DN_B
+#define ASAP_RING_DN_B 5
+#endif
 template <int EPI>
 struct Rings {
-  static constexpr int A = EPI == EPI_BF16 ? 3 : 4;
-  static constexpr int B = EPI == EPI_BF16 ? 5 : 4;
+  static constexpr int A = EPI == EPI_BF16 ? ASAP_RING_DN_A : EPI == EPI_SWIGLU ? ASAP_RING_GU_A : 4;
+  static constexpr int B = EPI == EPI_BF16 ? ASAP_RING_DN_B : EPI == EPI_SWIGLU ? ASAP_RING_GU_B : 4;
 };
 constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK;
 
@@ -59,9 +71,11 @@ constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
 
 constexpr int kBarBytes = 384;  // 2*SA + 2*SB + 5 + 2*kTileQ mbarriers, tmem slot, abort flag, tile ids
+// Dynamic shared memory: rings (1024-byte aligned for the 128-byte swizzle,
+// the alignment the kernel declares and checks), barriers, schedule table.
 template <int EPI>
 __host__ __device__ constexpr size_t smem_bytes() {
-  return 1024 + Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
+  return Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
 }
 
 
@@ -144,10 +158,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int SA = Rings<EPI>::A, SB = Rings<EPI>::B;
   static_assert(8 * (2 * SA + 2 * SB + 5) + kTileQBytes + 8 <= kBarBytes, "barrier area");
   static_assert(smem_bytes<EPI>() <= 227 * 1024, "shared memory budget");
-  extern __shared__ uint8_t smem_raw[];
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = (raw + 1023u) & ~1023u;
-  uint8_t* gbase = smem_raw + (base - raw);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t base = smem_u32(smem_raw);
+  if (base & 1023u) {  // uniform for the CTA: nothing is initialised yet
+    if (threadIdx.x == 0) record_status(args.status, ST_SMEM_ALIGN);
+    return;
+  }
+  uint8_t* gbase = smem_raw;
   const uint32_t sA = base;
   const uint32_t sB = base + SA * A_BYTES;
   uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;

@@ -405,6 +405,33 @@ def test_bad_indices_are_reported_not_trapped():
     assert code == 0 and word == 0
 
 
+@pytest.mark.parametrize("bad", ["decreasing", "past_rows", "negative"])
+def test_bad_offsets_are_reported_and_computed_nothing(bad):
+    """Offsets the grouped GEMMs cannot use (the kernels' own checks, no
+    out-of-range access) leave the routed outputs untouched and set status
+    bit 8; the shared expert (problem 1) is still computed."""
+    c = Case.get(DS_SMALL)
+    cfg = DS_SMALL
+    n, k, E, H = 64, cfg.top_k, cfg.n_experts, cfg.hidden
+    x = c.tokens(0, n)
+    offs = torch.arange(E + 1, dtype=torch.int32, device=DEV) * 2   # offsets[E] = 512 = n * k
+    if bad == "decreasing":
+        offs[10] = 30
+    elif bad == "past_rows":
+        offs[E] = n * k + 128
+    else:
+        offs[0] = -128
+    x_perm = c.tokens(1, n * k)
+    y = torch.full((n * k, H), 7.0, dtype=torch.bfloat16, device=DEV)
+    y_sh = torch.zeros((n, H), dtype=torch.bfloat16, device=DEV)
+    api.asap_moe_expert_ffn(c.h, x_perm, offs, x, y, y_sh, c.ws(n))
+    code, word = api.asap_moe_status(c.h)
+    assert code != 0 and word == 8, word
+    assert bool((y == 7.0).all())
+    compare_rows(bf16_to_f64(y_sh), oracle.swiglu(bf16_to_f64(x), *c.shared))
+    assert_clean(c)
+
+
 @pytest.mark.parametrize("cfg", [MX_SMALL, DS_SMALL], ids=lambda c: c.name)
 def test_ffn_halves_equal_expert_ffn_and_h_matches_oracle(cfg):
     """gate_up then down give the same bits as expert_ffn; the intermediate h
