@@ -393,9 +393,9 @@ def kernel_pass(args, h, cfg, xs, dev):
     out = torch.empty((n, H), dtype=torch.bfloat16, device=dev)
     ws = api.workspace(h, n, dev)
     fp8 = cfg.dtype != "bf16"
-    names = ["router_gemm", "gate_scan", "dispatch", "gemm_gate_up_swiglu", "gemm_down", "combine"]
+    names = ["route", "dispatch", "gemm_gate_up_swiglu", "gemm_down", "combine"]
     if fp8:
-        names = ["router_gemm", "gate_scan", "dispatch", "expert_ffn_fp8", "combine"]
+        names = ["route", "dispatch", "expert_ffn_fp8", "combine"]
         x_perm = torch.empty((n * k, H), dtype=torch.uint8, device=dev)
         xsc = torch.empty((n * k, H // 128), dtype=torch.float32, device=dev)
     times = {nm: [] for nm in names}
@@ -406,25 +406,23 @@ def kernel_pass(args, h, cfg, xs, dev):
             m = x.shape[0]
             ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
             ev[0].record(s)
-            api.asap_moe_router_logits(h, x, logits[:m], ws, stream=s)
+            api.asap_moe_route(h, x, idx[:m], w[:m], counts, offsets, ws, stream=s)
             ev[1].record(s)
-            api.asap_moe_route_logits(h, logits[:m], idx[:m], w[:m], counts, offsets, ws, stream=s)
-            ev[2].record(s)
             api.asap_moe_dispatch(h, x, idx[:m], x_perm[:m * k], perm_src[:m * k], perm_dst[:m], ws, stream=s,
                                   x_perm_scales=xsc[:m * k] if fp8 else None)
-            ev[3].record(s)
+            ev[2].record(s)
             if fp8:
                 api.asap_moe_expert_ffn(h, x_perm[:m * k], offsets, x, y_perm[:m * k],
                                         y_sh[:m] if y_sh is not None else None, ws, stream=s,
                                         x_perm_scales=xsc[:m * k])
-                ev[4].record(s)
+                ev[3].record(s)
             else:
                 api.asap_moe_expert_gate_up(h, x_perm[:m * k], offsets, x, hbuf[:m * k],
-                                            hsh[:m] if hsh is not None else None, stream=s)
-                ev[4].record(s)
+                                            hsh[:m] if hsh is not None else None, stream=s, ws=ws)
+                ev[3].record(s)
                 api.asap_moe_expert_down(h, hbuf[:m * k], offsets, hsh[:m] if hsh is not None else None, m,
-                                         y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s)
-                ev[5].record(s)
+                                         y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s, ws=ws)
+                ev[4].record(s)
             api.asap_moe_combine(h, y_perm[:m * k], y_sh[:m] if y_sh is not None else None, w[:m], perm_dst[:m],
                                  out[:m], stream=s)
             ev[len(names)].record(s)
@@ -447,8 +445,9 @@ def kernel_pass(args, h, cfg, xs, dev):
     wb = 2  # bf16 activations
     eb = 1 if fp8 else 2  # expert-weight element bytes
     alg = {
-        "router_gemm": dict(bytes=m * H * wb + E * H * wb + m * E * 4, flops=2.0 * m * H * E),
-        "gate_scan": dict(bytes=m * E * 4 + nk * 8, flops=0.0),
+        # route: read x and the router weights, write idx, w, counts, offsets
+        # (the logits between the router GEMM and the gate are not algorithmic)
+        "route": dict(bytes=m * H * wb + E * H * wb + nk * 8 + (2 * E + 1) * 4, flops=2.0 * m * H * E),
         "dispatch": dict(bytes=m * H * wb + nk * H * wb + nk * 12, flops=0.0),
         "gemm_gate_up_swiglu": dict(
             bytes=mean_active * 2 * I * H * eb + (2 * Is * H * eb if cfg.n_shared else 0)
@@ -548,7 +547,6 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
     ps = torch.empty(n_all * k, dtype=torch.int32, device=dev)
     pd = torch.empty((n_all, k), dtype=torch.int32, device=dev)
     api.asap_moe_dispatch(h, x, idx, x_perm, ps, pd, ws)
-    del ws
     hb = torch.empty((n_all * k, I), dtype=torch.bfloat16, device=dev)
     hsh = torch.empty((n_all, Is), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
     y = torch.empty_like(x_perm)
@@ -557,9 +555,9 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
     for it in range(args.kernel_steps + 1):
         e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
         e[0].record(s)
-        api.asap_moe_expert_gate_up(h, x_perm, offsets, x, hb, hsh)
+        api.asap_moe_expert_gate_up(h, x_perm, offsets, x, hb, hsh, ws=ws)
         e[1].record(s)
-        api.asap_moe_expert_down(h, hb, offsets, hsh, n_all, y, ysh)
+        api.asap_moe_expert_down(h, hb, offsets, hsh, n_all, y, ysh, ws=ws)
         e[2].record(s)
         torch.cuda.synchronize()
         if it:

@@ -238,15 +238,19 @@ int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* x_perm_sc
  *   gate_up: h_perm [n*k, I] = silu(X_e Wg_e^T) * (X_e Wu_e^T) per segment,
  *            h_shared [n, I_s] likewise for the shared expert on x;
  *   down   : y_perm = h_perm Wd_e^T per segment, y_shared = h_shared Ws_d^T.
- * No workspace.  bf16 configuration only (the FP8 configuration returns
- * ASAP_ERR_UNSUPPORTED; its h is e4m3 with scales, use asap_moe_expert_ffn);
- * *_scales are ignored (pass NULL). */
+ * The workspace is optional.  With one (asap_moe_workspace_size for n) the
+ * CTAs claim tiles dynamically from a counter in it, as asap_moe_expert_ffn
+ * does; with ws == NULL they take tiles in a fixed order, which is slower
+ * when other kernels share the GPU.  Same bits either way.  bf16
+ * configuration only (the FP8 configuration returns ASAP_ERR_UNSUPPORTED; its
+ * h is e4m3 with scales, use asap_moe_expert_ffn); *_scales are ignored
+ * (pass NULL). */
 int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
                             const int32_t* offsets, const void* x, int32_t n, void* h_perm,
-                            void* h_shared, void* stream);
+                            void* h_shared, void* ws, size_t ws_bytes, void* stream);
 int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float* h_perm_scales,
                          const int32_t* offsets, const void* h_shared, int32_t n, void* y_perm,
-                         void* y_shared, void* stream);
+                         void* y_shared, void* ws, size_t ws_bytes, void* stream);
 
 /* Combine (Section 3.2.2): out[t] = sum_{j<k} w[t,j] y_perm[perm_dst[t*k+j]]
  * (+ y_shared[t]), fp32 in slot order then the shared row, rounded to bf16.

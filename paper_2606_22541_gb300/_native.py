@@ -50,8 +50,8 @@ SIGNATURES = {
     "asap_moe_route_logits": [_P, _P, _I, _P, _P, _P, _P, _P, _SZ, _P],
     "asap_moe_dispatch": [_P, _P, _I, _P, _P, _P, _P, _P, _P, _SZ, _P],
     "asap_moe_expert_ffn": [_P, _P, _P, _P, _P, _I, _P, _P, _P, _SZ, _P],
-    "asap_moe_expert_gate_up": [_P, _P, _P, _P, _P, _I, _P, _P, _P],
-    "asap_moe_expert_down": [_P, _P, _P, _P, _P, _I, _P, _P, _P],
+    "asap_moe_expert_gate_up": [_P, _P, _P, _P, _P, _I, _P, _P, _P, _SZ, _P],
+    "asap_moe_expert_down": [_P, _P, _P, _P, _P, _I, _P, _P, _P, _SZ, _P],
     "asap_moe_combine": [_P, _P, _P, _P, _P, _I, _P, _P],
     "asap_moe_layer": [_P, _P, _I, _P, _P, _SZ, _P],
     "asap_moe_route_noalloc": [_P, _P, _I, _P, _P, _P, _P, _P],

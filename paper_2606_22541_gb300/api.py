@@ -148,16 +148,21 @@ def asap_moe_expert_ffn(h, x_perm, offsets, x, y_perm, y_shared, ws, stream=None
                                     x.shape[0], _ptr(y_perm), _ptr(y_shared), p, n, _stream(stream)))
 
 
-def asap_moe_expert_gate_up(h, x_perm, offsets, x, h_perm, h_shared, stream=None, x_perm_scales=None):
+def asap_moe_expert_gate_up(h, x_perm, offsets, x, h_perm, h_shared, stream=None, x_perm_scales=None, ws=None):
+    """ws (optional): a workspace for x.shape[0] tokens; with it the GEMM claims
+    its tiles dynamically."""
+    p, nb = _ws(ws)
     check("asap_moe_expert_gate_up",
           lib().asap_moe_expert_gate_up(h.ptr, _ptr(x_perm), _ptr(x_perm_scales), _ptr(offsets), _ptr(x),
-                                        x.shape[0], _ptr(h_perm), _ptr(h_shared), _stream(stream)))
+                                        x.shape[0], _ptr(h_perm), _ptr(h_shared), p, nb, _stream(stream)))
 
 
-def asap_moe_expert_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, stream=None, h_perm_scales=None):
+def asap_moe_expert_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, stream=None, h_perm_scales=None,
+                         ws=None):
+    p, nb = _ws(ws)
     check("asap_moe_expert_down",
           lib().asap_moe_expert_down(h.ptr, _ptr(h_perm), _ptr(h_perm_scales), _ptr(offsets), _ptr(h_shared),
-                                     int(n), _ptr(y_perm), _ptr(y_shared), _stream(stream)))
+                                     int(n), _ptr(y_perm), _ptr(y_shared), p, nb, _stream(stream)))
 
 
 def asap_moe_combine(h, y_perm, y_shared, w, perm_dst, out, stream=None):

@@ -806,9 +806,25 @@ ASAP_API int asap_moe_expert_ffn(asap_moe_t h, const void* x_perm, const float* 
                         h->layer_ids, counters, st);
 }
 
+namespace {
+
+// Tile counter of a standalone GEMM call: workspace slot 0, cleared on the
+// stream; nullptr (static tile order) without a workspace.
+int standalone_counter(asap_moe_t h, int32_t n, void* ws, size_t ws_bytes, cudaStream_t st, int32_t** out) {
+  *out = nullptr;
+  if (!ws) return ASAP_OK;
+  int r = check_call(h, n, ws, ws_bytes, true);
+  if (r != ASAP_OK) return r;
+  *out = at<int32_t>(ws, layout(h->cfg, n).tile_counters);
+  CU_TRY(cudaMemsetAsync(*out, 0, sizeof(int32_t), st), "tile counter");
+  return ASAP_OK;
+}
+
+}  // namespace
+
 ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const float* x_perm_scales,
                                      const int32_t* offsets, const void* x, int32_t n, void* h_perm,
-                                     void* h_shared, void* stream) {
+                                     void* h_shared, void* ws, size_t ws_bytes, void* stream) {
   (void)x_perm_scales;
   int r = check_call(h, n, nullptr, 0, false);
   if (r != ASAP_OK || n == 0) return r;
@@ -817,12 +833,14 @@ ASAP_API int asap_moe_expert_gate_up(asap_moe_t h, const void* x_perm, const flo
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!x || !h_shared || !aligned16(x) || !aligned16(h_shared)))
     return fail(ASAP_ERR_INVALID, "x and h_shared are required for the shared expert");
-  return run_gate_up(h, x_perm, offsets, x, n, h_perm, h_shared, h->layer_ids, nullptr, S(stream));
+  int32_t* counter = nullptr;
+  if ((r = standalone_counter(h, n, ws, ws_bytes, S(stream), &counter)) != ASAP_OK) return r;
+  return run_gate_up(h, x_perm, offsets, x, n, h_perm, h_shared, h->layer_ids, counter, S(stream));
 }
 
 ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float* h_perm_scales,
                                   const int32_t* offsets, const void* h_shared, int32_t n, void* y_perm,
-                                  void* y_shared, void* stream) {
+                                  void* y_shared, void* ws, size_t ws_bytes, void* stream) {
   (void)h_perm_scales;
   int r = check_call(h, n, nullptr, 0, false);
   if (r != ASAP_OK || n == 0) return r;
@@ -831,7 +849,9 @@ ASAP_API int asap_moe_expert_down(asap_moe_t h, const void* h_perm, const float*
     return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
   if (h->cfg.n_shared && (!h_shared || !y_shared || !aligned16(h_shared) || !aligned16(y_shared)))
     return fail(ASAP_ERR_INVALID, "h_shared and y_shared are required for the shared expert");
-  return run_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, h->layer_ids, nullptr, S(stream));
+  int32_t* counter = nullptr;
+  if ((r = standalone_counter(h, n, ws, ws_bytes, S(stream), &counter)) != ASAP_OK) return r;
+  return run_down(h, h_perm, offsets, h_shared, n, y_perm, y_shared, h->layer_ids, counter, S(stream));
 }
 
 ASAP_API int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_shared, const float* w,

@@ -454,10 +454,20 @@ def test_ffn_halves_equal_expert_ffn_and_h_matches_oracle(cfg):
     y2 = torch.empty_like(x_perm)
     ysh2 = torch.empty_like(ysh1) if cfg.n_shared else None
     api.asap_moe_expert_down(c.h, hb, offsets, hsh, n, y2, ysh2)
+    # the same halves with a workspace: tiles claimed dynamically, same bits
+    hb3 = torch.empty_like(hb)
+    hsh3 = torch.empty_like(hsh) if cfg.n_shared else None
+    api.asap_moe_expert_gate_up(c.h, x_perm, offsets, x, hb3, hsh3, ws=ws)
+    y3 = torch.empty_like(x_perm)
+    ysh3 = torch.empty_like(ysh1) if cfg.n_shared else None
+    api.asap_moe_expert_down(c.h, hb3, offsets, hsh3, n, y3, ysh3, ws=ws)
     torch.cuda.synchronize()
     assert torch.equal(y1.view(torch.int16), y2.view(torch.int16))
+    assert torch.equal(y1.view(torch.int16), y3.view(torch.int16))
+    assert torch.equal(hb.view(torch.int16), hb3.view(torch.int16))
     if cfg.n_shared:
         assert torch.equal(ysh1.view(torch.int16), ysh2.view(torch.int16))
+        assert torch.equal(ysh1.view(torch.int16), ysh3.view(torch.int16))
     off = offsets.cpu().numpy()
     xp = bf16_to_f64(x_perm)
     hg = bf16_to_f64(hb)
