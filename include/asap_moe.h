@@ -289,9 +289,9 @@ int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int
  * that reserved the GPU at start-up), or allocation on that path is forbidden
  * or would synchronise the device.  This call takes the same inputs and
  * outputs as asap_moe_route but keeps its scratch (router logits, per-chunk
- * histograms and chunk bases) in one static device array of the library:
- * 4096 tokens x 256 experts, 4 MiB + 256 KiB, held by every GPU that loads
- * libasap_moe until the process exits.  It calls no cudaMalloc, cudaFree or
+ * histograms, chunk bases and a counter) in one static device array of the
+ * library: 4096 tokens x 256 experts, 4 MiB + 256 KiB + 256 B, held by every
+ * GPU that loads libasap_moe until the process exits.  It calls no cudaMalloc, cudaFree or
  * other allocating routine.
  *  - n > 4096 (or n > max_tokens) returns ASAP_ERR_INVALID with a message.
  *  - The first call on a device looks up the array's device address

@@ -86,7 +86,7 @@ constexpr int kHintA = ASAP_HINT_BF16_A, kHintB = ASAP_HINT_BF16_B;
 constexpr int kHintF8A = ASAP_HINT_FP8_A, kHintF8B = ASAP_HINT_FP8_B;
 
 struct Layout {
-  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst, tile_counters;
+  size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst, tile_counters, ticket;
   // bf16: x_perm (also y_perm in asap_moe_layer), h, h_sh, y_sh
   size_t x_perm, h, h_sh, y_sh;
   // fp8: quantised rows and their per-128-channel scales, bf16 expert outputs
@@ -117,6 +117,7 @@ Layout layout(const asap_moe_config& c, long long n) {
   L.perm_src = take(nk * 4);
   L.perm_dst = take(nk * 4);
   L.tile_counters = take(asap::kTileCounters * 4);
+  L.ticket = take(4);
   if (c.dtype == ASAP_FP8_E4M3_BLOCK128) {
     L.xq = take(nk * H);
     L.xs = take(nk * (H / 128) * 4);
@@ -219,7 +220,8 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
   return ASAP_OK;
 }
 
-asap::GateParams gate_params(asap_moe_t h, const int32_t* layer) {
+// ticket: the scan's ticket in the call's scratch (zeroed by the gate launch).
+asap::GateParams gate_params(asap_moe_t h, const int32_t* layer, int32_t* ticket) {
   const asap_moe_config& c = h->cfg;
   asap::GateParams p{};
   p.n_experts = c.n_experts;
@@ -230,6 +232,7 @@ asap::GateParams gate_params(asap_moe_t h, const int32_t* layer) {
   p.route_scale = c.route_scale;
   p.lref = lref(h, layer);
   p.status = h->status;
+  p.ticket = ticket;
   return p;
 }
 
@@ -238,9 +241,10 @@ int run_gate_scan(asap_moe_t h, const float* logits, int splits, int n, int32_t*
   const Layout L = layout(h->cfg, n);
   int32_t* hist = at<int32_t>(ws, L.hist);
   int32_t* base = at<int32_t>(ws, L.chunk_base);
-  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h, layer), idx, w, hist, st), "gate launch");
+  int32_t* ticket = at<int32_t>(ws, L.ticket);
+  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h, layer, ticket), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
-                           st, at<int32_t>(ws, L.tile_counters)),
+                           ticket, st, at<int32_t>(ws, L.tile_counters)),
          "scan launch");
   return ASAP_OK;
 }
@@ -762,15 +766,17 @@ ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int
   cudaStream_t st = S(stream);
   int32_t* hist = at<int32_t>(ws, L.hist);
   int32_t* base = at<int32_t>(ws, L.chunk_base);
-  CU_TRY(asap::launch_hist(idx, n, c.top_k, c.n_experts, hist, h->status, st), "hist launch");
-  CU_TRY(asap::launch_scan(hist, chunks, c.n_experts, at<int32_t>(ws, L.counts), at<int32_t>(ws, L.offsets), base, st),
+  int32_t* ticket = at<int32_t>(ws, L.ticket);
+  int32_t* offs = at<int32_t>(ws, L.offsets);
+  CU_TRY(asap::launch_hist(idx, n, c.top_k, c.n_experts, hist, h->status, ticket, st), "hist launch");
+  CU_TRY(asap::launch_scan(hist, chunks, c.n_experts, at<int32_t>(ws, L.counts), offs, base, ticket, st),
          "scan launch");
   if (h->fp8)
-    CU_TRY(asap::launch_dispatch_fp8(x, n, c.hidden, c.top_k, c.n_experts, idx, base, x_perm, x_perm_scales, nullptr,
-                                     nullptr, perm_src, perm_dst, h->status, st),
+    CU_TRY(asap::launch_dispatch_fp8(x, n, c.hidden, c.top_k, c.n_experts, idx, base, offs, x_perm, x_perm_scales,
+                                     nullptr, nullptr, perm_src, perm_dst, h->status, st),
            "dispatch launch");
   else
-    CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, base, x_perm, perm_src, perm_dst,
+    CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, base, offs, x_perm, perm_src, perm_dst,
                                  h->status, st),
            "dispatch launch");
   return ASAP_OK;
@@ -894,8 +900,8 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
     void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
     CU_TRY(asap::launch_dispatch_fp8(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base),
-                                     at<void>(ws, L.xq), at<float>(ws, L.xs), xq_sh, xs_sh, perm_src, perm_dst,
-                                     h->status, st),
+                                     offsets, at<void>(ws, L.xq), at<float>(ws, L.xs), xq_sh, xs_sh, perm_src,
+                                     perm_dst, h->status, st),
            "dispatch launch");
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
                              at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), layer, counters,
@@ -910,8 +916,8 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
     return ASAP_OK;
   }
   void* x_perm = at<void>(ws, L.x_perm);
-  CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base), x_perm,
-                               perm_src, perm_dst, h->status, st),
+  CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base), offsets,
+                               x_perm, perm_src, perm_dst, h->status, st),
          "dispatch launch");
   // y_perm reuses x_perm's rows: the down GEMM never reads x_perm
   if ((r = run_expert_ffn(h, x_perm, offsets, x, n, x_perm, y_sh, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer,
@@ -963,7 +969,8 @@ int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const 
       const int splits = router_splits(h, n);
       float* lg = logits + static_cast<long long>(asap::kMaxRouterSplits) * tok0 * E;
       if ((r = run_router_logits(h, xs[i], n, lg, splits, layer, st)) != ASAP_OK) return r;
-      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, layer), idx + static_cast<long long>(tok0) * k,
+      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, layer, at<int32_t>(ws, L.ticket)),
+                                   idx + static_cast<long long>(tok0) * k,
                                    w + static_cast<long long>(tok0) * k, hist, chunk0, chunks_total, st),
              "gate launch");
     }
@@ -972,8 +979,8 @@ int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const 
   }
   // one histogram scan over every chunk: expert segments hold the rows of all
   // micro-batches, in (micro-batch, token, slot) order
-  CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, st,
-                           at<int32_t>(ws, L.tile_counters)),
+  CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, at<int32_t>(ws, L.ticket),
+                           st, at<int32_t>(ws, L.tile_counters)),
          "scan launch");
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
   tok0 = 0;
@@ -982,6 +989,7 @@ int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const 
     const int n = ns[i];
     if (n > 0) {
       asap::DispatchSeg seg{};
+      seg.expert_offsets = offsets;
       seg.chunk0 = chunk0;
       seg.n_chunks_total = chunks_total;
       seg.tok0 = tok0;
@@ -1118,7 +1126,7 @@ constexpr size_t kStaticLogitsBytes =
     static_cast<size_t>(kStaticRouteMaxTokens) * ASAP_MOE_MAX_EXPERTS * sizeof(float);   // 4 MiB
 constexpr size_t kStaticChunkBytes = static_cast<size_t>(kStaticRouteMaxTokens / asap::kChunkTokens) *
                                      ASAP_MOE_MAX_EXPERTS * sizeof(int32_t);                  // 128 KiB
-constexpr size_t kStaticRouteBytes = kStaticLogitsBytes + 2 * kStaticChunkBytes;
+constexpr size_t kStaticRouteBytes = kStaticLogitsBytes + 2 * kStaticChunkBytes + 256;  // + the scan's ticket
 
 constexpr int kStaticMaxDevices = 64;
 std::mutex g_static_route_mu;
@@ -1171,11 +1179,14 @@ ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int3
   int32_t* base = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + kStaticChunkBytes);
   cudaStream_t st = S(stream);
   // every scratch element read below is written earlier on the same stream
-  // (logits by the router, all E entries of each chunk's histogram by the
-  // gate kernel), so nothing has to be cleared between calls
+  // (logits by the router, all E entries of each chunk's histogram and the
+  // scan's ticket by the gate kernel), so nothing has to be cleared between
+  // calls
   if ((r = run_router_logits(h, x, n, logits, 1, h->layer_ids, st)) != ASAP_OK) return r;
-  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h, h->layer_ids), idx, w, hist, st), "gate launch");
-  CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base, st),
+  int32_t* ticket = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + 2 * kStaticChunkBytes);
+  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h, h->layer_ids, ticket), idx, w, hist, st), "gate launch");
+  CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
+                           ticket, st),
          "scan launch");
   return ASAP_OK;
 }

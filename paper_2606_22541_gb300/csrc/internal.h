@@ -123,6 +123,7 @@ struct GateParams {
   float route_scale;
   LayerRef lref;  // selection bias: table[layer].router_bias ([E] or nullptr)
   uint32_t* status;
+  int32_t* ticket;  // the scan's ticket, zeroed by the gate launch (nullable)
 };
 // Router on the CUDA cores (E < 256): weights table[layer].router_w.
 cudaError_t launch_router_small(const void* x, const LayerRef& lref, int n, int H, int E, float* logits,
@@ -137,12 +138,16 @@ cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane
 // n_chunks_total columns.
 cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                             int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s);
-cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
+// hist as launch_gate writes it; zeroes the scan's ticket.
+cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status, int32_t* ticket,
                         cudaStream_t s);
-// tile_counters (nullable): kTileCounters ints zeroed for the grouped GEMMs
-// that follow on the stream.
+// counts, offsets, and chunk_base[e][c] = entries of expert e in chunks
+// before c (relative: the absolute base is offsets[e] + chunk_base[e][c]).
+// ticket: one int, zero at launch (the gate / hist launch zeroes it), left
+// zero.  tile_counters (nullable): kTileCounters ints zeroed for the grouped
+// GEMMs that follow on the stream.
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
-                        int32_t* chunk_base, cudaStream_t s, int32_t* tile_counters = nullptr);
+                        int32_t* chunk_base, int32_t* ticket, cudaStream_t s, int32_t* tile_counters = nullptr);
 
 // ------------------------------------------------------------ permute
 // Place of one micro-batch among several served by one call: its chunks start
@@ -151,6 +156,7 @@ cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* count
 // nullable) receives its rows for the shared expert (pointer already offset
 // to the micro-batch's first token).
 struct DispatchSeg {
+  const int32_t* expert_offsets;  // offsets[e] (the scan's output)
   int chunk0;
   int n_chunks_total;
   int tok0;
@@ -158,14 +164,15 @@ struct DispatchSeg {
   void* x_sh;
 };
 cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
-                            const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
+                            const int32_t* chunk_base, const int32_t* offsets, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s);
 // FP8 dispatch: every token row is quantised once (e4m3, fp32 scale per 128
 // channels) and written to its k positions of xq / xs, and to row t of
 // xq_sh / xs_sh when those are non-null (shared expert input).
 cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
-                                const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
-                                int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+                                const int32_t* chunk_base, const int32_t* offsets, void* xq, float* xs,
+                                void* xq_sh, float* xs_sh, int32_t* perm_src, int32_t* perm_dst, uint32_t* status,
+                                cudaStream_t s);
 // rows_total: rows of y_perm the positions may address (0 = n * k).
 cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float* w,
                            const int32_t* perm_dst, int n, int H, int k, void* out,

@@ -25,7 +25,9 @@ constexpr int kRankWarps = kChunkTokens * kMaxTopK / 32;  // warps that rank the
 // an entry inside its expert is (entries of that expert in earlier chunks)
 // + (in earlier warps of this chunk) + (in earlier lanes of this warp):
 // positions increase with (t, j) inside every segment.  chunk_base is
-// expert-major: chunk_base[e * n_chunks + chunk].  Then one warp per token
+// expert-major, relative to the expert's offset: the entries of expert e in
+// chunks before ``chunk`` are offsets[e] + chunk_base[e * n_chunks + chunk].
+// Then one warp per token
 // reads its row once and writes it to its k positions.
 // Quantise 8 consecutive values of a 128-channel block held by 16 lanes
 // (lanes 0-15 one block, 16-31 the next): scale = amax / 448 over the block,
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
   }
   __syncthreads();
   for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
-    int run = chunk_base[static_cast<long long>(ee) * n_chunks + seg.chunk0 + c];
+    int run = seg.expert_offsets[ee] + chunk_base[static_cast<long long>(ee) * n_chunks + seg.chunk0 + c];
 #pragma unroll
     for (int w = 0; w < kRankWarps; ++w) {
       const int v = wcnt[w][ee];
@@ -271,9 +273,10 @@ __global__ void pack_gate_up_kernel(const uint4* __restrict__ gate, const uint4*
 }  // namespace
 
 cudaError_t launch_dispatch(const void* x, int n, int H, int k, int E, const int32_t* idx,
-                            const int32_t* chunk_base, void* x_perm, int32_t* perm_src,
+                            const int32_t* chunk_base, const int32_t* offsets, void* x_perm, int32_t* perm_src,
                             int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
   DispatchSeg seg{};
+  seg.expert_offsets = offsets;
   seg.n_chunks_total = ceil_div(n, kChunkTokens);
   seg.rows_total = static_cast<long long>(n) * k;
   return launch_dispatch_seg(x, n, H, k, E, idx, chunk_base, x_perm, perm_src, perm_dst, status, seg, s);
@@ -291,9 +294,11 @@ cudaError_t launch_dispatch_seg(const void* x, int n, int H, int k, int E, const
 }
 
 cudaError_t launch_dispatch_fp8(const void* x, int n, int H, int k, int E, const int32_t* idx,
-                                const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
-                                int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+                                const int32_t* chunk_base, const int32_t* offsets, void* xq, float* xs,
+                                void* xq_sh, float* xs_sh, int32_t* perm_src, int32_t* perm_dst, uint32_t* status,
+                                cudaStream_t s) {
   DispatchSeg seg{};
+  seg.expert_offsets = offsets;
   seg.n_chunks_total = ceil_div(n, kChunkTokens);
   seg.rows_total = static_cast<long long>(n) * k;
   return launch_dispatch_fp8_seg(x, n, H, k, E, idx, chunk_base, xq, xs, xq_sh, xs_sh, perm_src, perm_dst, status,

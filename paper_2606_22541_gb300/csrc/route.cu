@@ -103,6 +103,7 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
   for (int e = threadIdx.x; e < E; e += blockDim.x) shist[e] = 0;
   __syncthreads();
 
+  if (p.ticket && blockIdx.x == 0 && threadIdx.x == 0) *p.ticket = 0;  // for the scan that follows
   const int t0 = blockIdx.x * kChunkTokens;
   const int t1 = min(n, t0 + kChunkTokens);
   const bool grouped = p.gating == 2;
@@ -259,10 +260,241 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
       hist[static_cast<long long>(e) * n_chunks + chunk0 + blockIdx.x] = shist[e];
 }
 
+// ------------------------------------------------------------ gating, a team of lanes per token
+// The same rules as gate_kernel for the common shapes (E = T S experts, T =
+// min(32, E) lanes per token, S in {1, 2, 4, 8}; n_groups a power of two up
+// to 32 for the grouped rule).  Lane q of a team holds experts [q S, (q+1) S)
+// in registers (16-byte loads of the K-slice planes, added in slice order).
+//  - Group scores: a group of gsz = E / G experts spans R = gsz / S lanes of
+//    the team (G <= T), whose local top-2 keys merge over the R lanes.
+//  - Every lane sorts its eligible (key, expert) pairs once (odd-even
+//    transposition network, ties to the lower expert), then each of the k
+//    rounds takes the best head of the team (a butterfly) and the winning
+//    lane drops its head.
+// Weights as in gate_kernel; the softmax sum adds each lane's slice in expert
+// order, then the lanes in a butterfly.  Selection keys, group scores and the
+// tie-breaks are those of gate_kernel, so both give the same experts.  One
+// CTA per chunk of kChunkTokens tokens (32 T threads).
+
+template <int T>
+__device__ __forceinline__ void team_argmax(float& v, int& i, float& x) {
+#pragma unroll
+  for (int o = T / 2; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(kFull, v, o);
+    const int oi = __shfl_xor_sync(kFull, i, o);
+    const float ox = __shfl_xor_sync(kFull, x, o);
+    if (ov > v || (ov == v && oi < i)) {
+      v = ov;
+      i = oi;
+      x = ox;
+    }
+  }
+}
+
+// (a before b) in selection order: larger key, then lower expert
+__device__ __forceinline__ bool sel_before(float ka, int ia, float kb, int ib) {
+  return ka > kb || (ka == kb && ia < ib);
+}
+
+template <int T, int S>
+__global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float* __restrict__ logits, int splits,
+                                                                 long long plane, int n, GateParams p,
+                                                                 int32_t* __restrict__ idx,
+                                                                 float* __restrict__ wout,
+                                                                 int32_t* __restrict__ hist, int n_chunks,
+                                                                 int chunk0) {
+  static_assert(T * S <= kMaxExperts && (T == 8 || T == 16 || T == 32) && S <= 8, "team shape");
+  __shared__ int shist[kMaxExperts];
+  const int lane = threadIdx.x & 31;
+  const int q = lane & (T - 1);  // lane in team
+  const int E = T * S, k = p.top_k;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) shist[e] = 0;
+  if (p.ticket && blockIdx.x == 0 && threadIdx.x == 0) *p.ticket = 0;  // for the scan that follows
+  __syncthreads();
+  const bool grouped = p.gating == 2;
+  const float* __restrict__ bias =
+      grouped ? p.lref.table[load_layer(p.lref.layer, p.lref.n_layers, p.status, threadIdx.x == 0 && blockIdx.x == 0)]
+                    .router_bias
+              : nullptr;
+  const int t = blockIdx.x * kChunkTokens + threadIdx.x / T;
+  const bool valid = t < n;
+  const int e0 = q * S;
+  float key[S], val[S];
+  {
+    const float* row = logits + static_cast<long long>(valid ? t : 0) * E + e0;
+    float l[S];
+    if constexpr (S % 4 == 0) {
+#pragma unroll
+      for (int v = 0; v < S / 4; ++v) {
+        const float4 a = __ldg(reinterpret_cast<const float4*>(row) + v);
+        l[4 * v] = a.x;
+        l[4 * v + 1] = a.y;
+        l[4 * v + 2] = a.z;
+        l[4 * v + 3] = a.w;
+      }
+#pragma unroll 1
+      for (int s2 = 1; s2 < splits; ++s2) {
+#pragma unroll
+        for (int v = 0; v < S / 4; ++v) {
+          const float4 a = __ldg(reinterpret_cast<const float4*>(row + s2 * plane) + v);
+          l[4 * v] += a.x;
+          l[4 * v + 1] += a.y;
+          l[4 * v + 2] += a.z;
+          l[4 * v + 3] += a.w;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < S; ++j) {
+        float a = __ldg(row + j);
+        for (int s2 = 1; s2 < splits; ++s2) a += __ldg(row + s2 * plane + j);
+        l[j] = a;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < S; ++j) {
+      if (!valid) l[j] = 0.f;
+      if (grouped) {
+        const float sg = 1.0f / (1.0f + expf(-l[j]));
+        val[j] = sg;
+        key[j] = sg + (bias ? bias[e0 + j] : 0.0f);
+      } else {
+        val[j] = l[j];
+        key[j] = l[j];
+      }
+    }
+  }
+  uint32_t eligible = (1u << S) - 1u;  // bit j: expert e0 + j may be chosen (S <= 8)
+  if (grouped) {
+    const int G = p.n_groups;  // <= T (checked at launch)
+    uint32_t kept = 0;
+    {
+      const int R = (E / G) / S;  // lanes per group
+      const int g = q / R;
+      float m1 = -CUDART_INF_F, m2 = -CUDART_INF_F;
+#pragma unroll
+      for (int j = 0; j < S; ++j) {
+        if (key[j] > m1) {
+          m2 = m1;
+          m1 = key[j];
+        } else if (key[j] > m2) {
+          m2 = key[j];
+        }
+      }
+      for (int o = 1; o < R; o <<= 1) {
+        const float a1 = __shfl_xor_sync(kFull, m1, o);
+        const float a2 = __shfl_xor_sync(kFull, m2, o);
+        const float hi = fmaxf(m1, a1);  // top two of {m1, m2, a1, a2}
+        const float lo = fmaxf(fminf(m1, a1), fmaxf(m2, a2));
+        m1 = hi;
+        m2 = lo;
+      }
+      const float gs = m1 + m2;
+#pragma unroll 1
+      for (int r = 0; r < p.topk_groups; ++r) {
+        const bool done = (kept >> g) & 1u;
+        float v = done ? -CUDART_INF_F : gs;
+        int gi = done ? 0x7fffffff : g;
+        float unused = 0.f;
+        team_argmax<T>(v, gi, unused);
+        if (gi != 0x7fffffff) kept |= 1u << gi;
+      }
+      if (!((kept >> g) & 1u)) eligible = 0;
+    }
+  }
+  // softmax: the sum of exp(l - max l) over all experts, before the sort
+  // reorders this lane's values
+  float z = 0.f, lmax = -CUDART_INF_F;
+  if (p.gating == 0) {
+#pragma unroll
+    for (int j = 0; j < S; ++j) lmax = fmaxf(lmax, key[j]);
+#pragma unroll
+    for (int o = 1; o < T; o <<= 1) lmax = fmaxf(lmax, __shfl_xor_sync(kFull, lmax, o));
+#pragma unroll
+    for (int j = 0; j < S; ++j) z += expf(key[j] - lmax);
+#pragma unroll
+    for (int o = 1; o < T; o <<= 1) z += __shfl_xor_sync(kFull, z, o);
+  }
+  // this lane's eligible candidates, sorted in selection order
+  int ci[S];
+#pragma unroll
+  for (int j = 0; j < S; ++j) {
+    ci[j] = ((eligible >> j) & 1u) ? e0 + j : 0x7fffffff;
+    if (!((eligible >> j) & 1u)) key[j] = -CUDART_INF_F;
+  }
+#pragma unroll
+  for (int pass = 0; pass < S; ++pass) {
+#pragma unroll
+    for (int j = pass & 1; j + 1 < S; j += 2) {
+      if (sel_before(key[j + 1], ci[j + 1], key[j], ci[j])) {
+        const float tk = key[j], tv = val[j];
+        const int ti = ci[j];
+        key[j] = key[j + 1];
+        val[j] = val[j + 1];
+        ci[j] = ci[j + 1];
+        key[j + 1] = tk;
+        val[j + 1] = tv;
+        ci[j + 1] = ti;
+      }
+    }
+  }
+  // k rounds over the team's heads
+  int e_mine = 0x7fffffff;
+  float x_mine = 0.f, sum = 0.f, m = 0.f, zsel = 0.f;
+#pragma unroll 1
+  for (int r = 0; r < k; ++r) {
+    float v = key[0], x = val[0];
+    int ei = ci[0];
+    team_argmax<T>(v, ei, x);
+    if (ei == ci[0] && ei != 0x7fffffff) {  // this lane's head won: drop it
+#pragma unroll
+      for (int j = 0; j + 1 < S; ++j) {
+        key[j] = key[j + 1];
+        val[j] = val[j + 1];
+        ci[j] = ci[j + 1];
+      }
+      key[S - 1] = -CUDART_INF_F;
+      ci[S - 1] = 0x7fffffff;
+    }
+    if (grouped) {
+      sum += x;
+      if (r == q) {
+        e_mine = ei;
+        x_mine = x;
+      }
+    } else {
+      if (r == 0) m = v;  // the largest logit
+      const float ex = expf(v - m);
+      zsel += ex;
+      if (r == q) {
+        e_mine = ei;
+        x_mine = ex;
+      }
+    }
+  }
+  float w_mine;
+  if (grouped) {
+    w_mine = x_mine / sum * p.route_scale;
+  } else {
+    w_mine = x_mine / (p.gating == 0 ? z : zsel);
+  }
+  if (valid && q < k) {
+    idx[static_cast<long long>(t) * k + q] = e_mine;
+    wout[static_cast<long long>(t) * k + q] = w_mine;
+    if (e_mine >= 0 && e_mine < E) atomicAdd(&shist[e_mine], 1);
+  }
+  __syncthreads();
+  if (hist)
+    for (int e = threadIdx.x; e < E; e += blockDim.x)
+      hist[static_cast<long long>(e) * n_chunks + chunk0 + blockIdx.x] = shist[e];
+}
+
 // ------------------------------------------------------------ histogram only
 __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ idx, int n, int k, int E,
-                                                   int32_t* __restrict__ hist, int n_chunks, uint32_t* status) {
+                                                   int32_t* __restrict__ hist, int n_chunks, uint32_t* status,
+                                                   int32_t* ticket) {
   __shared__ int shist[kMaxExperts];
+  if (blockIdx.x == 0 && threadIdx.x == 0) *ticket = 0;  // for the scan that follows
   for (int e = threadIdx.x; e < E; e += blockDim.x) shist[e] = 0;
   __syncthreads();
   const int t0 = blockIdx.x * kChunkTokens;
@@ -277,74 +509,87 @@ __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ i
 }
 
 // ------------------------------------------------------------ scan
-// One CTA.  hist and chunk_base are stored expert-major ([E][n_chunks]), so
-// warp w scans experts w, w+32, ... over 32 consecutive chunks per coalesced
-// load, giving each (expert, chunk) the number of earlier entries of that
-// expert; then counts, the exclusive offsets, and the absolute chunk bases.
-__global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ hist, int n_chunks, int E,
-                                                    int32_t* __restrict__ counts,
-                                                    int32_t* __restrict__ offsets,
-                                                    int32_t* __restrict__ chunk_base,
-                                                    int32_t* __restrict__ tile_counters) {
-  __shared__ int scount[kMaxExperts];
-  __shared__ int soff[kMaxExperts + 1];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // the grouped GEMMs that follow on this stream claim tiles from these
-  if (tile_counters && threadIdx.x < kTileCounters) tile_counters[threadIdx.x] = 0;
-  for (int e = warp; e < E; e += 32) {
-    const int32_t* hrow = hist + static_cast<long long>(e) * n_chunks;
-    int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
-    int run = 0;
-    for (int c0 = 0; c0 < n_chunks; c0 += 32) {
-      const int c = c0 + lane;
-      const int v = c < n_chunks ? hrow[c] : 0;
-      int incl = v;
+// One CTA per expert.  hist and chunk_base are stored expert-major
+// ([E][n_chunks]); CTA e scans its row with coalesced loads, writes
+// chunk_base[e][c] = the expert's entries in chunks before c (relative to the
+// expert's offset, which dispatch adds) and counts[e].  The last CTA to finish
+// (a ticket counter, zeroed by the kernel that wrote hist and reset here)
+// scans the counts into the exclusive offsets and clears the grouped GEMMs'
+// tile counters.
+constexpr int kScanThreads = 256;
+
+__device__ __forceinline__ int block_exclusive_scan(int v, int* swarp, int& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int incl = v;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int u = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += u;
-      }
-      if (c < n_chunks) brow[c] = run + incl - v;
-      run += __shfl_sync(kFull, incl, 31);
-    }
-    if (lane == 0) scount[e] = run;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int u = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += u;
   }
+  if (lane == 31) swarp[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    int loc[8];
-    int local = 0;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int e = lane * 8 + i;
-      loc[i] = e < E ? scount[e] : 0;
-      local += loc[i];
-    }
-    int incl = local;
+    const int nw = blockDim.x >> 5;
+    int w = lane < nw ? swarp[lane] : 0;
+    int wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int u = __shfl_up_sync(kFull, incl, o);
-      if (lane >= o) incl += u;
+      const int u = __shfl_up_sync(kFull, wi, o);
+      if (lane >= o) wi += u;
     }
-    int run = incl - local;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int e = lane * 8 + i;
-      if (e < E) soff[e] = run;
-      run += loc[i];
-    }
-    if (lane == 31) soff[E] = incl;
+    if (lane < nw) swarp[lane] = wi - w;
+    if (lane == nw - 1) swarp[32] = wi;
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < E; e += blockDim.x) {
-    counts[e] = scount[e];
-    offsets[e] = soff[e];
+  total = swarp[32];
+  const int r = swarp[warp] + incl - v;
+  __syncthreads();  // swarp may be reused by the caller
+  return r;
+}
+
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __restrict__ hist, int n_chunks, int E,
+                                                            int32_t* __restrict__ counts,
+                                                            int32_t* __restrict__ offsets,
+                                                            int32_t* __restrict__ chunk_base,
+                                                            int32_t* __restrict__ tile_counters,
+                                                            int32_t* __restrict__ ticket) {
+  __shared__ int swarp[33];
+  __shared__ bool last;
+  const int e = blockIdx.x;
+  const int32_t* hrow = hist + static_cast<long long>(e) * n_chunks;
+  int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
+  int run = 0;
+  for (int c0 = 0; c0 < n_chunks; c0 += kScanThreads) {
+    const int c = c0 + threadIdx.x;
+    const int v = c < n_chunks ? hrow[c] : 0;
+    int tot = 0;
+    const int ex = block_exclusive_scan(v, swarp, tot);
+    if (c < n_chunks) brow[c] = run + ex;
+    run += tot;
   }
-  if (threadIdx.x == 0) offsets[E] = soff[E];
-  for (int e = warp; e < E; e += 32) {
-    int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
-    const int base = soff[e];
-    for (int c = lane; c < n_chunks; c += 32) brow[c] += base;
+  if (threadIdx.x == 0) {
+    counts[e] = run;
+    __threadfence();
+    last = atomicAdd(ticket, 1) == E - 1;
   }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  int base = 0;
+  for (int e0 = 0; e0 < E; e0 += kScanThreads) {
+    const int ee = e0 + threadIdx.x;
+    const int v = ee < E ? __ldcg(counts + ee) : 0;
+    int tot = 0;
+    const int ex = block_exclusive_scan(v, swarp, tot);
+    if (ee < E) offsets[ee] = base + ex;
+    base += tot;
+  }
+  if (threadIdx.x == 0) {
+    offsets[E] = base;
+    *ticket = 0;
+  }
+  // the grouped GEMMs that follow on this stream claim tiles from these
+  if (tile_counters && threadIdx.x < kTileCounters) tile_counters[threadIdx.x] = 0;
 }
 
 // Sum of the K-slice planes of the router GEMM, added in slice order.
@@ -377,16 +622,39 @@ cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GatePa
                             int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
-  gate_kernel<<<chunks, kGateWarps * 32, 0, s>>>(logits, splits, static_cast<long long>(n) * p.n_experts, n, p,
-                                                  idx, w, hist, n_chunks_total, chunk0);
+  const long long plane = static_cast<long long>(n) * p.n_experts;
+  // a team of T = min(32, E) lanes per token when the shape allows it
+  const int E = p.n_experts;
+  const int T = E >= 32 ? 32 : E;
+  const int S = E / T;
+  const int G = p.gating == 2 ? p.n_groups : 1;
+  // (16-byte vector loads of the logits rows need a 16-byte aligned base)
+  const bool team = (T == 8 || T == 16 || T == 32) && E % T == 0 && (S == 1 || S == 2 || S == 4 || S == 8) &&
+                    (G & (G - 1)) == 0 && G <= T && (S < 4 || (reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
+  if (team) {
+#define ASAP_GATE_TEAM(TV, SV)                                                                                  \
+  if (T == TV && S == SV) {                                                                                     \
+    gate_team_kernel<TV, SV><<<chunks, kChunkTokens * TV, 0, s>>>(logits, splits, plane, n, p, idx, w, hist,    \
+                                                                  n_chunks_total, chunk0);                      \
+    return cudaGetLastError();                                                                                  \
+  }
+    ASAP_GATE_TEAM(32, 8)
+    ASAP_GATE_TEAM(32, 4)
+    ASAP_GATE_TEAM(32, 2)
+    ASAP_GATE_TEAM(32, 1)
+    ASAP_GATE_TEAM(16, 1)
+    ASAP_GATE_TEAM(8, 1)
+#undef ASAP_GATE_TEAM
+  }
+  gate_kernel<<<chunks, kGateWarps * 32, 0, s>>>(logits, splits, plane, n, p, idx, w, hist, n_chunks_total, chunk0);
   return cudaGetLastError();
 }
 
-cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status,
+cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status, int32_t* ticket,
                         cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
-  hist_kernel<<<chunks, 256, 0, s>>>(idx, n, k, E, hist, chunks, status);
+  hist_kernel<<<chunks, 256, 0, s>>>(idx, n, k, E, hist, chunks, status, ticket);
   return cudaGetLastError();
 }
 
@@ -398,8 +666,8 @@ cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane
 }
 
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
-                        int32_t* chunk_base, cudaStream_t s, int32_t* tile_counters) {
-  scan_kernel<<<1, 1024, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters);
+                        int32_t* chunk_base, int32_t* ticket, cudaStream_t s, int32_t* tile_counters) {
+  scan_kernel<<<E, kScanThreads, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters, ticket);
   return cudaGetLastError();
 }
 
