@@ -17,8 +17,18 @@ namespace asap {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kDispatchWarps = kChunkTokens;  // one warp per token for the copies
+// The bf16 dispatch splits a chunk's row copies over two CTAs (every one
+// ranks the chunk's entries, the first writes the permutation), so 4096
+// tokens run 256 CTAs, more than the 152 SMs (measured on GB300: 112 -> 107
+// us); the FP8 dispatch, which also quantises, is faster with one CTA per
+// chunk (85 us vs 100 us).
+template <bool FP8>
+__host__ __device__ constexpr int dispatch_parts() { return FP8 ? 1 : 2; }
 constexpr int kRankWarps = kChunkTokens * kMaxTopK / 32;  // warps that rank the chunk's entries
+template <bool FP8>
+__host__ __device__ constexpr int dispatch_warps() {
+  return kChunkTokens / dispatch_parts<FP8>() > kRankWarps ? kChunkTokens / dispatch_parts<FP8>() : kRankWarps;
+}
 
 // One CTA per chunk of kChunkTokens tokens.  Entry i = t_local * k + j is
 // ranked by thread i, so warp order and lane order follow (t, j); the rank of
@@ -54,7 +64,7 @@ __device__ __forceinline__ uint2 quantize8(uint4 v, float& scale) {
 }
 
 template <bool FP8>
-__global__ void __launch_bounds__(kDispatchWarps * 32)
+__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
     dispatch_kernel(const uint4* __restrict__ x, int n, int V, int k, int E,
                     const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
                     void* __restrict__ x_perm_v, float* __restrict__ xs, uint2* __restrict__ xq_sh,
@@ -62,7 +72,9 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
                     int32_t* __restrict__ perm_dst, uint32_t* status, const DispatchSeg seg) {
   __shared__ int wcnt[kRankWarps][kMaxExperts];
   __shared__ int spos[kChunkTokens * kMaxTopK];
-  const int c = blockIdx.x;
+  constexpr int kParts = dispatch_parts<FP8>();
+  const int c = blockIdx.x / kParts;
+  const int part = blockIdx.x % kParts;
   const int t0 = c * kChunkTokens;
   const int nt = min(kChunkTokens, n - t0);
   const int ne = nt * k;
@@ -106,21 +118,24 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
       }
     }
     spos[i] = pos;
-    perm_dst[static_cast<long long>(t0) * k + i] = pos;
-    if (pos >= 0) perm_src[pos] = seg.tok0 + t0 + i / k;
+    if (part == 0) {
+      perm_dst[static_cast<long long>(t0) * k + i] = pos;
+      if (pos >= 0) perm_src[pos] = seg.tok0 + t0 + i / k;
+    }
   }
   __syncthreads();
-  // row copies: one warp per token, read once, write k times
-  if (warp < nt) {
-    const uint4* src = x + static_cast<long long>(t0 + warp) * V;
+  // row copies: one warp per token of this CTA's part, read once, write k times
+  const int tl = part * (kChunkTokens / kParts) + warp;  // token of the chunk
+  if (warp < kChunkTokens / kParts && tl < nt) {
+    const uint4* src = x + static_cast<long long>(t0 + tl) * V;
     int p[kMaxTopK];
 #pragma unroll
-    for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[warp * k + j] : -1;
+    for (int j = 0; j < kMaxTopK; ++j) p[j] = j < k ? spos[tl * k + j] : -1;
     if constexpr (!FP8) {
       uint4* x_perm = static_cast<uint4*>(x_perm_v);
       // optional copy of the row for the shared expert (calls that serve
       // several micro-batches gather their tokens into one matrix)
-      uint4* sh = seg.x_sh ? static_cast<uint4*>(seg.x_sh) + static_cast<long long>(t0 + warp) * V : nullptr;
+      uint4* sh = seg.x_sh ? static_cast<uint4*>(seg.x_sh) + static_cast<long long>(t0 + tl) * V : nullptr;
       int v = lane;
       for (; v + 32 < V; v += 64) {
         const uint4 a = __ldg(src + v);
@@ -149,7 +164,7 @@ __global__ void __launch_bounds__(kDispatchWarps * 32)
       // vectors (128 channels); a warp covers two blocks per step
       uint2* xq = static_cast<uint2*>(x_perm_v);
       const int nb = V / 16;
-      const long long t = t0 + warp;
+      const long long t = t0 + tl;
       for (int v = lane; v < V; v += 32) {
         float scale;
         const uint2 q = quantize8(__ldg(src + v), scale);
@@ -287,7 +302,7 @@ cudaError_t launch_dispatch_seg(const void* x, int n, int H, int k, int E, const
                                 uint32_t* status, const DispatchSeg& seg, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
-  dispatch_kernel<false><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
+  dispatch_kernel<false><<<chunks * dispatch_parts<false>(), dispatch_warps<false>() * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
                                                                 chunk_base, seg.n_chunks_total, x_perm, nullptr,
                                                                 nullptr, nullptr, perm_src, perm_dst, status, seg);
   return cudaGetLastError();
@@ -311,7 +326,7 @@ cudaError_t launch_dispatch_fp8_seg(const void* x, int n, int H, int k, int E, c
                                     cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int chunks = ceil_div(n, kChunkTokens);
-  dispatch_kernel<true><<<chunks, kDispatchWarps * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
+  dispatch_kernel<true><<<chunks * dispatch_parts<true>(), dispatch_warps<true>() * 32, 0, s>>>(static_cast<const uint4*>(x), n, H / 8, k, E, idx,
                                                                chunk_base, seg.n_chunks_total, xq, xs,
                                                                static_cast<uint2*>(xq_sh), xs_sh, perm_src, perm_dst,
                                                                status, seg);
