@@ -99,4 +99,12 @@ DSV3_FP8_E32 = LayerConfig("dsv3_fp8_e32_profile", hidden=7168, n_experts=32, to
                            shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
                            route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[512], seed=1004)
 
-CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32, DSV3_FP8_E32)}
+# Profiling case of route, dispatch and combine: the DeepSeek-V3 routing shape
+# (H = 7168, 256 experts, top-8, grouped sigmoid, 4096 tokens), whose bytes do
+# not depend on the expert FFN width, with a narrow FFN (I = 256) so the device
+# holds 2.8 GB of weights.
+DSV3_ROUTING = LayerConfig("dsv3_routing_profile", hidden=7168, n_experts=256, top_k=8, inter=256, n_shared=1,
+                           shared_inter=256, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
+                           route_scale=2.5, microbatches=[4096], seed=1002)
+
+CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32, DSV3_FP8_E32, DSV3_ROUTING)}
