@@ -267,10 +267,11 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
 // in registers (16-byte loads of the K-slice planes, added in slice order).
 //  - Group scores: a group of gsz = E / G experts spans R = gsz / S lanes of
 //    the team (G <= T), whose local top-2 keys merge over the R lanes.
-//  - Every lane sorts its eligible (key, expert) pairs once (odd-even
-//    transposition network, ties to the lower expert), then each of the k
-//    rounds takes the best head of the team (a butterfly) and the winning
-//    lane drops its head.
+//  - Groups are kept by rank: a group's rank is the number of groups with a
+//    larger score, or an equal score and a lower index.
+//  - Each of the k rounds takes every lane's best remaining eligible
+//    expert, keeps the team's best (a butterfly, ties to the lower expert)
+//    and marks it taken in its owner lane.
 // Weights as in gate_kernel; the softmax sum adds each lane's slice in expert
 // order, then the lanes in a butterfly.  Selection keys, group scores and the
 // tie-breaks are those of gate_kernel, so both give the same experts.  One
@@ -289,11 +290,6 @@ __device__ __forceinline__ void team_argmax(float& v, int& i, float& x) {
       x = ox;
     }
   }
-}
-
-// (a before b) in selection order: larger key, then lower expert
-__device__ __forceinline__ bool sel_before(float ka, int ia, float kb, int ib) {
-  return ka > kb || (ka == kb && ia < ib);
 }
 
 template <int T, int S>
@@ -367,7 +363,7 @@ __global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float
   uint32_t eligible = (1u << S) - 1u;  // bit j: expert e0 + j may be chosen (S <= 8)
   if (grouped) {
     const int G = p.n_groups;  // <= T (checked at launch)
-    uint32_t kept = 0;
+    uint32_t kept = 0;  // this lane's group is kept
     {
       const int R = (E / G) / S;  // lanes per group
       const int g = q / R;
@@ -390,20 +386,20 @@ __global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float
         m2 = lo;
       }
       const float gs = m1 + m2;
+      // rank of this lane's group among all G: groups with a larger score,
+      // or an equal score and a lower index, come first (score of group gg
+      // read from its first lane, gg R)
+      int rank = 0;
 #pragma unroll 1
-      for (int r = 0; r < p.topk_groups; ++r) {
-        const bool done = (kept >> g) & 1u;
-        float v = done ? -CUDART_INF_F : gs;
-        int gi = done ? 0x7fffffff : g;
-        float unused = 0.f;
-        team_argmax<T>(v, gi, unused);
-        if (gi != 0x7fffffff) kept |= 1u << gi;
+      for (int gg = 0; gg < G; ++gg) {
+        const float o = __shfl_sync(kFull, gs, (lane & ~(T - 1)) + gg * R);
+        rank += (o > gs || (o == gs && gg < g)) ? 1 : 0;
       }
-      if (!((kept >> g) & 1u)) eligible = 0;
+      kept = rank < p.topk_groups ? 1u : 0u;
+      if (!kept) eligible = 0;
     }
   }
-  // softmax: the sum of exp(l - max l) over all experts, before the sort
-  // reorders this lane's values
+  // softmax: the sum of exp(l - max l) over all experts
   float z = 0.f, lmax = -CUDART_INF_F;
   if (p.gating == 0) {
 #pragma unroll
@@ -415,47 +411,26 @@ __global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float
 #pragma unroll
     for (int o = 1; o < T; o <<= 1) z += __shfl_xor_sync(kFull, z, o);
   }
-  // this lane's eligible candidates, sorted in selection order
-  int ci[S];
-#pragma unroll
-  for (int j = 0; j < S; ++j) {
-    ci[j] = ((eligible >> j) & 1u) ? e0 + j : 0x7fffffff;
-    if (!((eligible >> j) & 1u)) key[j] = -CUDART_INF_F;
-  }
-#pragma unroll
-  for (int pass = 0; pass < S; ++pass) {
-#pragma unroll
-    for (int j = pass & 1; j + 1 < S; j += 2) {
-      if (sel_before(key[j + 1], ci[j + 1], key[j], ci[j])) {
-        const float tk = key[j], tv = val[j];
-        const int ti = ci[j];
-        key[j] = key[j + 1];
-        val[j] = val[j + 1];
-        ci[j] = ci[j + 1];
-        key[j + 1] = tk;
-        val[j + 1] = tv;
-        ci[j + 1] = ti;
-      }
-    }
-  }
-  // k rounds over the team's heads
+  // k rounds: every lane offers its best remaining eligible expert (larger
+  // key, then lower expert), the team keeps the best offer, and its owner
+  // marks it taken
   int e_mine = 0x7fffffff;
   float x_mine = 0.f, sum = 0.f, m = 0.f, zsel = 0.f;
+  uint32_t avail = eligible;
 #pragma unroll 1
   for (int r = 0; r < k; ++r) {
-    float v = key[0], x = val[0];
-    int ei = ci[0];
-    team_argmax<T>(v, ei, x);
-    if (ei == ci[0] && ei != 0x7fffffff) {  // this lane's head won: drop it
+    float v = -CUDART_INF_F, x = 0.f;
+    int ei = 0x7fffffff;
 #pragma unroll
-      for (int j = 0; j + 1 < S; ++j) {
-        key[j] = key[j + 1];
-        val[j] = val[j + 1];
-        ci[j] = ci[j + 1];
+    for (int j = 0; j < S; ++j) {
+      if (((avail >> j) & 1u) && (ei == 0x7fffffff || key[j] > v)) {
+        v = key[j];
+        x = val[j];
+        ei = e0 + j;
       }
-      key[S - 1] = -CUDART_INF_F;
-      ci[S - 1] = 0x7fffffff;
     }
+    team_argmax<T>(v, ei, x);
+    if (ei >= e0 && ei < e0 + S) avail &= ~(1u << (ei - e0));
     if (grouped) {
       sum += x;
       if (r == q) {
