@@ -24,6 +24,13 @@ DS_SMALL = inputs.small_variant(DSV3, name="dsv3_small", hidden=512, inter=256, 
 ST_SMALL = inputs.small_variant(STRESS, name="stress_small", hidden=512, inter=256, shared_inter=256,
                                 microbatches=[700, 129, 1])
 SMALL = [TINY, MX_SMALL, DS_SMALL, ST_SMALL]
+# Shapes outside the 32-lane-team gate (expert counts and groups that are not
+# powers of two): routed by the warp-per-token gate kernel.
+ODD_SOFTMAX = inputs.small_variant(TINY, name="odd_softmax", n_experts=12, top_k=3, gating="softmax_renorm",
+                                   microbatches=[200, 33])
+ODD_GROUPED = inputs.small_variant(DSV3, name="odd_grouped", hidden=256, n_experts=24, top_k=4, inter=128,
+                                   shared_inter=128, n_groups=3, topk_groups=2, microbatches=[200, 33])
+ODD = [ODD_SOFTMAX, ODD_GROUPED]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -92,7 +99,7 @@ def test_router_logits_within_bound(cfg):
     assert_clean(c)
 
 
-@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", SMALL + ODD, ids=lambda c: c.name)
 def test_route_matches_oracle(cfg):
     c = Case.get(cfg)
     for i in range(len(cfg.microbatches)):
@@ -168,6 +175,33 @@ def test_route_logits_grouped_exact_ties_and_all_to_one_group():
 
 
 # ---------------------------------------------------------------- dispatch / combine
+
+def test_gate_kernels_agree():
+    """The 32-lane-team gate and the warp-per-token gate (taken for logits
+    that are not 16-byte aligned) route the same logits to the same experts
+    with the same weights (grouped sigmoid: the same arithmetic in the same
+    order)."""
+    c = Case.get(DS_SMALL)
+    n, k, E = 300, DS_SMALL.top_k, DS_SMALL.n_experts
+    x = c.tokens(0, n)
+    logits = torch.empty((n, E), dtype=torch.float32, device=DEV)
+    api.asap_moe_router_logits(c.h, x, logits, c.ws(n))
+    raw = torch.empty(n * E + 1, dtype=torch.float32, device=DEV)
+    shifted = raw[1:].view(n, E)                              # 4-byte offset: warp-per-token gate
+    shifted.copy_(logits)
+    outs = []
+    for lg in (logits, shifted):
+        idx = torch.empty((n, k), dtype=torch.int32, device=DEV)
+        w = torch.empty((n, k), dtype=torch.float32, device=DEV)
+        counts = torch.empty(E, dtype=torch.int32, device=DEV)
+        offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
+        api.asap_moe_route_logits(c.h, lg, idx, w, counts, offsets, c.ws(n))
+        outs.append((idx, w, counts, offsets))
+    torch.cuda.synchronize()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+    assert_clean(c)
+
 
 @pytest.mark.parametrize("cfg", [TINY, DS_SMALL], ids=lambda c: c.name)
 def test_dispatch_exact(cfg):
@@ -270,7 +304,7 @@ def oracle_layer(c, x):
                             c.ocfg, shared=c.shared)
 
 
-@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", SMALL + ODD, ids=lambda c: c.name)
 def test_layer_matches_oracle(cfg):
     c = Case.get(cfg)
     for i, n in enumerate(cfg.microbatches):
@@ -288,7 +322,7 @@ def test_layer_matches_oracle(cfg):
     assert_clean(c)
 
 
-@pytest.mark.parametrize("cfg", [TINY, DS_SMALL, ST_SMALL], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", [TINY, DS_SMALL, ST_SMALL] + ODD, ids=lambda c: c.name)
 def test_route_equals_route_logits_of_router_logits(cfg):
     """asap_moe_route == asap_moe_route_logits(asap_moe_router_logits(x))."""
     c = Case.get(cfg)
