@@ -232,8 +232,7 @@ def sources_sha256(files):
 
 
 GEMM_SOURCES = ["paper_2606_22541_gb300/csrc/gemm_tc.cu", "paper_2606_22541_gb300/csrc/common.cuh",
-                "paper_2606_22541_gb300/csrc/gemm_sched.cuh", "paper_2606_22541_gb300/csrc/internal.h",
-                "paper_2606_22541_gb300/csrc/api.cu"]
+                "paper_2606_22541_gb300/csrc/gemm_sched.cuh", "paper_2606_22541_gb300/csrc/gemm_config.h"]
 
 
 def weight_gb(cfg):

@@ -4,6 +4,7 @@
 #include "../../include/asap_moe.h"
 #include "common.cuh"
 #include "internal.h"
+#include "gemm_config.h"
 
 #include <cstdio>
 #include <cstring>
@@ -63,25 +64,6 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 constexpr int kMaxBatch = 64;  // micro-batches one asap_moe_layer_batched call may serve
 
-// L2 priority of the grouped GEMMs' loads (0 normal, 1 evict-first, 2
-// evict-last): activations (A) are re-read by every n-tile of their expert
-// and stay evict-last; the bf16 weights (B) are read by the m-tiles of one
-// expert at about the same time, which find them in L2 only at normal
-// priority (measured on GB300 at 4096 DeepSeek-V3 tokens: gate/up 2.90 ->
-// 2.59 ms, down 1.78 -> 1.54 ms against evict-first weights).  The FP8 GEMMs
-// measured 2 % faster with evict-first weights.
-#ifndef ASAP_HINT_BF16_A
-#define ASAP_HINT_BF16_A 2
-#endif
-#ifndef ASAP_HINT_BF16_B
-#define ASAP_HINT_BF16_B 0
-#endif
-#ifndef ASAP_HINT_FP8_A
-#define ASAP_HINT_FP8_A 2
-#endif
-#ifndef ASAP_HINT_FP8_B
-#define ASAP_HINT_FP8_B 1
-#endif
 constexpr int kHintA = ASAP_HINT_BF16_A, kHintB = ASAP_HINT_BF16_B;
 constexpr int kHintF8A = ASAP_HINT_FP8_A, kHintF8B = ASAP_HINT_FP8_B;
 

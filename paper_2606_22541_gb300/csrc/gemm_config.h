@@ -1,0 +1,50 @@
+// Tuning parameters of the grouped GEMMs (ring depths per launch kind and
+// the L2 priority of their loads), measured on GB300; build-time defines
+// override them.
+#pragma once
+
+// Ring depths (stages of A [128 x 64] and B [256 x 64] bf16 boxes).  A k-step
+// needs both boxes, so the pipeline depth that counts is that of the
+// shallowest ring whose operand comes from HBM.  gate/up (GU): both operands
+// from HBM, 4 + 4.  down (DN): its activations h are still in L2 from the
+// gate/up launch, 3 + 5 (1.84 -> 1.73 ms at 4096 DeepSeek-V3 tokens).  router
+// (RT): activations from HBM, the 256 x H router weights from L2, 6 + 3
+// (70.5 -> 64.5 us at 16384 tokens).
+#ifndef ASAP_RING_GU_A
+#define ASAP_RING_GU_A 4
+#endif
+#ifndef ASAP_RING_GU_B
+#define ASAP_RING_GU_B 4
+#endif
+#ifndef ASAP_RING_DN_A
+#define ASAP_RING_DN_A 3
+#endif
+#ifndef ASAP_RING_DN_B
+#define ASAP_RING_DN_B 5
+#endif
+#ifndef ASAP_RING_RT_A
+#define ASAP_RING_RT_A 6
+#endif
+#ifndef ASAP_RING_RT_B
+#define ASAP_RING_RT_B 3
+#endif
+
+// L2 priority of the grouped GEMMs' loads (0 normal, 1 evict-first, 2
+// evict-last): activations (A) are re-read by every n-tile of their expert
+// and stay evict-last; the bf16 weights (B) are read by the m-tiles of one
+// expert at about the same time, which find them in L2 only at normal
+// priority (measured on GB300 at 4096 DeepSeek-V3 tokens: gate/up 2.90 ->
+// 2.59 ms, down 1.78 -> 1.54 ms against evict-first weights).  The FP8 GEMMs
+// measured 2 % faster with evict-first weights.
+#ifndef ASAP_HINT_BF16_A
+#define ASAP_HINT_BF16_A 2
+#endif
+#ifndef ASAP_HINT_BF16_B
+#define ASAP_HINT_BF16_B 0
+#endif
+#ifndef ASAP_HINT_FP8_A
+#define ASAP_HINT_FP8_A 2
+#endif
+#ifndef ASAP_HINT_FP8_B
+#define ASAP_HINT_FP8_B 1
+#endif

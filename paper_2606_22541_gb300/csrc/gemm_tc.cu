@@ -27,6 +27,7 @@
 // Rows of a tile past the segment end belong to the next expert (or are
 // zero-filled by TMA past the tensor end) and are masked at the store.
 #include "common.cuh"
+#include "gemm_config.h"
 #include "gemm_sched.cuh"
 #include "internal.h"
 
@@ -36,34 +37,7 @@ namespace asap {
 
 namespace {
 
-// Separate rings for the two operands.  The kernel streams HBM, and a k-step
-// can start only when both of its boxes have landed, so the useful pipeline
-// depth is that of the shallowest ring whose operand comes from HBM.  The
-// gate/up GEMM reads its activations (x_perm, just written by dispatch) from
-// HBM as well, so both rings get 4 stages; the down GEMM's activations (h)
-// are still in L2 from the gate/up launch, so its weight ring gets 5 stages
-// and its activation ring 3 (measured on GB300: 1.84 -> 1.73 ms per launch at
-// 4096 DeepSeek-V3 tokens, while 3 + 5 would slow the gate/up GEMM by 15 %).
-#ifndef ASAP_RING_GU_A
-#define ASAP_RING_GU_A 4
-#endif
-#ifndef ASAP_RING_GU_B
-#define ASAP_RING_GU_B 4
-#endif
-#ifndef ASAP_RING_DN_A
-#define ASAP_RING_DN_A 3
-#endif
-#ifndef ASAP_RING_DN_B
-#define ASAP_RING_DN_B 5
-#endif
-// router GEMM: its activations come from HBM, the 256 x H router weights
-// from L2 (measured at 16384 tokens: 6 + 3 stages 64.5 us vs 4 + 4 70.5 us)
-#ifndef ASAP_RING_RT_A
-#define ASAP_RING_RT_A 6
-#endif
-#ifndef ASAP_RING_RT_B
-#define ASAP_RING_RT_B 3
-#endif
+// Separate rings for the two operands, depths per launch kind (gemm_config.h).
 template <int EPI>
 struct Rings {
   static constexpr int A = EPI == EPI_BF16 ? ASAP_RING_DN_A : EPI == EPI_SWIGLU ? ASAP_RING_GU_A : ASAP_RING_RT_A;
