@@ -341,7 +341,7 @@ def run_ours(args, dist):
         # e4m3 tensor peak: the measured bf16 figure times the nominal fp8/bf16 ratio (4.5 / 2.25)
         tensor_peak = 2.0 * peaks["bf16_tflops_sustained"]
         result["dtype"] = "e4m3 (fp32 accumulate, bf16 out)"
-    result["roofline"] = roofline(kern, peaks, peaks_src, tensor_peak)
+    result["roofline"] = roofline(kern, peaks, peaks_src, tensor_peak, cfg.name)
     gemm_flops = kern["gemm_flops"]
     gemm_ms = kern["gemm_ms"]
     result["grouped_gemm_tensor_frac"] = {
@@ -437,36 +437,43 @@ def kernel_pass(args, h, cfg, xs, dev):
                 times[nm].append(ev[j].elapsed_time(ev[j + 1]))
     avg = {nm: sum(v) / len(v) for nm, v in times.items()}
     mins = {nm: min(v) for nm, v in times.items()}
-    m = xs[0].shape[0]
-    nk = m * k
     mean_active = sum(active) / len(active)
-    # algorithmic bytes / FLOPs per launch (one micro-batch of m tokens)
     wb = 2  # bf16 activations
     eb = 1 if fp8 else 2  # expert-weight element bytes
-    alg = {
-        # route: read x and the router weights, write idx, w, counts, offsets
-        # (the logits between the router GEMM and the gate are not algorithmic)
-        "route": dict(bytes=m * H * wb + E * H * wb + nk * 8 + (2 * E + 1) * 4, flops=2.0 * m * H * E),
-        "dispatch": dict(bytes=m * H * wb + nk * H * wb + nk * 12, flops=0.0),
-        "gemm_gate_up_swiglu": dict(
-            bytes=mean_active * 2 * I * H * eb + (2 * Is * H * eb if cfg.n_shared else 0)
-            + nk * H * wb + (m * H * wb if cfg.n_shared else 0) + nk * I * wb + (m * Is * wb if cfg.n_shared else 0),
-            flops=2.0 * nk * H * 2 * I + (2.0 * m * H * 2 * Is if cfg.n_shared else 0.0)),
-        "gemm_down": dict(
-            bytes=mean_active * H * I * eb + (H * Is * eb if cfg.n_shared else 0)
-            + nk * I * wb + (m * Is * wb if cfg.n_shared else 0) + nk * H * wb + (m * H * wb if cfg.n_shared else 0),
-            flops=2.0 * nk * I * H + (2.0 * m * Is * H if cfg.n_shared else 0.0)),
-        "combine": dict(bytes=nk * H * wb + (m * H * wb if cfg.n_shared else 0) + m * H * wb + nk * 8, flops=0.0),
-    }
-    if fp8:
-        # e4m3 activations (x_perm, h) and bf16 outputs
-        alg["dispatch"] = dict(bytes=m * H * wb + nk * H + nk * (H // 128) * 4 + nk * 12, flops=0.0)
-        g1 = alg["gemm_gate_up_swiglu"]
-        g2 = alg["gemm_down"]
-        alg["expert_ffn_fp8"] = dict(
-            bytes=mean_active * 3 * I * H + (3 * Is * H if cfg.n_shared else 0) + nk * H + 2 * nk * I
-            + (m * H * 2 + m * H + 2 * m * Is if cfg.n_shared else 0) + nk * H * 2 + (m * H * 2 if cfg.n_shared else 0),
-            flops=g1["flops"] + g2["flops"])
+
+    def alg_of(m, act):
+        """Algorithmic bytes / FLOPs of each step for one micro-batch of m
+        tokens whose routing reaches ``act`` experts."""
+        nk = m * k
+        a = {
+            # route: read x and the router weights, write idx, w, counts, offsets
+            # (the logits between the router GEMM and the gate are not algorithmic)
+            "route": dict(bytes=m * H * wb + E * H * wb + nk * 8 + (2 * E + 1) * 4, flops=2.0 * m * H * E),
+            "dispatch": dict(bytes=m * H * wb + nk * H * wb + nk * 12, flops=0.0),
+            "gemm_gate_up_swiglu": dict(
+                bytes=act * 2 * I * H * eb + (2 * Is * H * eb if cfg.n_shared else 0)
+                + nk * H * wb + (m * H * wb if cfg.n_shared else 0) + nk * I * wb + (m * Is * wb if cfg.n_shared else 0),
+                flops=2.0 * nk * H * 2 * I + (2.0 * m * H * 2 * Is if cfg.n_shared else 0.0)),
+            "gemm_down": dict(
+                bytes=act * H * I * eb + (H * Is * eb if cfg.n_shared else 0)
+                + nk * I * wb + (m * Is * wb if cfg.n_shared else 0) + nk * H * wb + (m * H * wb if cfg.n_shared else 0),
+                flops=2.0 * nk * I * H + (2.0 * m * Is * H if cfg.n_shared else 0.0)),
+            "combine": dict(bytes=nk * H * wb + (m * H * wb if cfg.n_shared else 0) + m * H * wb + nk * 8, flops=0.0),
+        }
+        if fp8:
+            # e4m3 activations (x_perm, h) and bf16 outputs
+            a["dispatch"] = dict(bytes=m * H * wb + nk * H + nk * (H // 128) * 4 + nk * 12, flops=0.0)
+            a["expert_ffn_fp8"] = dict(
+                bytes=act * 3 * I * H + (3 * Is * H if cfg.n_shared else 0) + nk * H + 2 * nk * I
+                + (m * H * 2 + m * H + 2 * m * Is if cfg.n_shared else 0) + nk * H * 2 + (m * H * 2 if cfg.n_shared else 0),
+                flops=a["gemm_gate_up_swiglu"]["flops"] + a["gemm_down"]["flops"])
+        return a
+
+    # per launch: the mean over the micro-batches (work and time alike), so
+    # rates are total work over total time also when the sizes differ
+    per_mb = [alg_of(x.shape[0], act) for x, act in zip(xs, active)]
+    alg = {nm: dict(bytes=sum(a[nm]["bytes"] for a in per_mb) / len(per_mb),
+                    flops=sum(a[nm]["flops"] for a in per_mb) / len(per_mb)) for nm in per_mb[0]}
     table = {}
     for nm in names:
         sec = avg[nm] / 1e3
@@ -481,14 +488,16 @@ def kernel_pass(args, h, cfg, xs, dev):
             "active_experts": mean_active, "serial_ms_per_microbatch": total_ms}
 
 
-def roofline(kern, peaks, peaks_src, tensor_peak=None):
+def roofline(kern, peaks, peaks_src, tensor_peak=None, workload=None):
     nm = max(kern["avg"], key=kern["avg"].get)
     a = kern["alg"][nm]
     sec = kern["avg"][nm] / 1e3
     tpk = tensor_peak or peaks["bf16_tflops_sustained"]
     t_hbm = a["bytes"] / (peaks["hbm_gbs"] * 1e9)
     t_tc = a["flops"] / (tpk * 1e12) if a["flops"] else 0.0
-    traffic, src = profile_traffic("gemm_gate_up_swiglu_dsv3.md", GEMM_SOURCES) if nm.startswith("gemm") else (None, None)
+    # the committed capture covers the DeepSeek-V3 BF16 gate/up launch only
+    traffic, src = (profile_traffic("gemm_gate_up_swiglu_dsv3.md", GEMM_SOURCES)
+                    if workload == "dsv3_bf16" and nm == "gemm_gate_up_swiglu" else (None, None))
     if t_tc >= t_hbm:
         achieved = a["flops"] / sec / 1e12
         peak = tpk
