@@ -22,8 +22,11 @@ constexpr unsigned kFull = 0xffffffffu;
 
 // ------------------------------------------------------------ router logits
 // One warp per token; logits[t, e] = sum_h x[t, h] Wr[e, h] in fp32 with a
-// fixed reduction order (per-lane strided partial sums, then a butterfly).
-constexpr int kRouterEB = 16;  // experts per pass
+// fixed reduction order (per-lane strided partial sums in increasing h, then
+// a butterfly).  Each lane loads kRouterAhead of its 16-byte pieces of the
+// token row before using them, so their HBM latencies overlap.
+constexpr int kRouterEB = 16;    // experts per pass
+constexpr int kRouterAhead = 8;  // row pieces in flight per lane
 
 __global__ void __launch_bounds__(256) router_small_kernel(const uint4* __restrict__ x, LayerRef lref,
                                                            uint32_t* status, int n, int V, int E,
@@ -38,20 +41,31 @@ __global__ void __launch_bounds__(256) router_small_kernel(const uint4* __restri
     float acc[kRouterEB];
 #pragma unroll
     for (int i = 0; i < kRouterEB; ++i) acc[i] = 0.f;
-    for (int v = lane; v < V; v += 32) {
-      const uint4 xv = __ldg(xr + v);
-      const float xf[8] = {bf16_lo(xv.x), bf16_hi(xv.x), bf16_lo(xv.y), bf16_hi(xv.y),
-                           bf16_lo(xv.z), bf16_hi(xv.z), bf16_lo(xv.w), bf16_hi(xv.w)};
+    for (int v0 = lane; v0 < V; v0 += 32 * kRouterAhead) {
+      uint4 xv[kRouterAhead];
 #pragma unroll
-      for (int i = 0; i < kRouterEB; ++i) {
-        if (e0 + i < E) {
-          const uint4 wv = __ldg(wr + static_cast<long long>(e0 + i) * V + v);
-          const float wf[8] = {bf16_lo(wv.x), bf16_hi(wv.x), bf16_lo(wv.y), bf16_hi(wv.y),
-                               bf16_lo(wv.z), bf16_hi(wv.z), bf16_lo(wv.w), bf16_hi(wv.w)};
-          float a = acc[i];
+      for (int u = 0; u < kRouterAhead; ++u) {
+        const int v = v0 + 32 * u;
+        xv[u] = v < V ? __ldg(xr + v) : make_uint4(0, 0, 0, 0);
+      }
 #pragma unroll
-          for (int q = 0; q < 8; ++q) a = fmaf(xf[q], wf[q], a);
-          acc[i] = a;
+      for (int u = 0; u < kRouterAhead; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < V) {
+          const float xf[8] = {bf16_lo(xv[u].x), bf16_hi(xv[u].x), bf16_lo(xv[u].y), bf16_hi(xv[u].y),
+                               bf16_lo(xv[u].z), bf16_hi(xv[u].z), bf16_lo(xv[u].w), bf16_hi(xv[u].w)};
+#pragma unroll
+          for (int i = 0; i < kRouterEB; ++i) {
+            if (e0 + i < E) {
+              const uint4 wv = __ldg(wr + static_cast<long long>(e0 + i) * V + v);
+              const float wf[8] = {bf16_lo(wv.x), bf16_hi(wv.x), bf16_lo(wv.y), bf16_hi(wv.y),
+                                   bf16_lo(wv.z), bf16_hi(wv.z), bf16_lo(wv.w), bf16_hi(wv.w)};
+              float a = acc[i];
+#pragma unroll
+              for (int q = 0; q < 8; ++q) a = fmaf(xf[q], wf[q], a);
+              acc[i] = a;
+            }
+          }
         }
       }
     }
