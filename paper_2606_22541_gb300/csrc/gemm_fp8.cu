@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < kH; ++j) {
           const float gv = acc[j];
-          const float hv = gv / (1.0f + __expf(-gv)) * acc[kH + j];
+          const float hv = __fdividef(gv, 1.0f + __expf(-gv)) * acc[kH + j];
           acc[j] = hv;
           amax = fmaxf(amax, fabsf(hv));
         }
@@ -387,6 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int u = 0; u < kColGroups; ++u) amax = fmaxf(amax, xs[u * BM + r]);
         const float scale = amax > 0.f ? amax / 448.0f : 1.0f;
+        const float inv = 1.0f / scale;  // one division; the quotients below are products
         if (valid) {
           uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
           const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
@@ -397,9 +398,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
               const __nv_fp8x2_storage_t lo = __nv_cvt_float2_to_fp8x2(
-                  make_float2(acc[j + 4 * u] / scale, acc[j + 4 * u + 1] / scale), __NV_SATFINITE, __NV_E4M3);
+                  make_float2(acc[j + 4 * u] * inv, acc[j + 4 * u + 1] * inv), __NV_SATFINITE, __NV_E4M3);
               const __nv_fp8x2_storage_t hi = __nv_cvt_float2_to_fp8x2(
-                  make_float2(acc[j + 4 * u + 2] / scale, acc[j + 4 * u + 3] / scale), __NV_SATFINITE, __NV_E4M3);
+                  make_float2(acc[j + 4 * u + 2] * inv, acc[j + 4 * u + 3] * inv), __NV_SATFINITE, __NV_E4M3);
               w4[u] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
             }
             *reinterpret_cast<uint4*>(dst + j) = make_uint4(w4[0], w4[1], w4[2], w4[3]);

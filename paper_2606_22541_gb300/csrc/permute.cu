@@ -41,7 +41,9 @@ __host__ __device__ constexpr int dispatch_warps() {
 // reads its row once and writes it to its k positions.
 // Quantise 8 consecutive values of a 128-channel block held by 16 lanes
 // (lanes 0-15 one block, 16-31 the next): scale = amax / 448 over the block,
-// q = e4m3(v / scale) with round-to-nearest-even and saturation.
+// q = e4m3(v / scale) with round-to-nearest-even and saturation; the
+// quotient is taken as v * (1 / scale) in fp32, which can differ from the
+// exact quotient by an ulp before the e4m3 rounding.
 __device__ __forceinline__ uint2 quantize8(uint4 v, float& scale) {
   float f[8] = {bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y),
                 bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w)};
@@ -51,13 +53,14 @@ __device__ __forceinline__ uint2 quantize8(uint4 v, float& scale) {
 #pragma unroll
   for (int o = 8; o > 0; o >>= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, o));
   scale = am > 0.f ? am / 448.0f : 1.0f;
+  const float inv = 1.0f / scale;  // one division; the quotients below are products
   uint32_t w[2];
 #pragma unroll
   for (int u = 0; u < 2; ++u) {
     const __nv_fp8x2_storage_t lo =
-        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u] / scale, f[4 * u + 1] / scale), __NV_SATFINITE, __NV_E4M3);
+        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u] * inv, f[4 * u + 1] * inv), __NV_SATFINITE, __NV_E4M3);
     const __nv_fp8x2_storage_t hi =
-        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u + 2] / scale, f[4 * u + 3] / scale), __NV_SATFINITE, __NV_E4M3);
+        __nv_cvt_float2_to_fp8x2(make_float2(f[4 * u + 2] * inv, f[4 * u + 3] * inv), __NV_SATFINITE, __NV_E4M3);
     w[u] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
   }
   return make_uint2(w[0], w[1]);
