@@ -189,6 +189,29 @@ def test_one_graph_replayed_for_every_layer(cfg):
     assert_clean(L.h)
 
 
+def test_layers_on_concurrent_streams():
+    """Different layers at the same time on different streams, each call
+    with its own id slot and workspace, equal the single-layer handles."""
+    cfg = DS_SMALL
+    L = Layers.get(cfg)
+    xs = [L.tokens(i % len(cfg.microbatches)) for i in range(N_LAYERS)]
+    ref = [single_out(L, l, xs[l]) for l in range(N_LAYERS)]
+    torch.cuda.synchronize()
+    slots = torch.tensor([2, 0, 1], dtype=torch.int32, device=DEV)
+    order = slots.tolist()
+    streams = [torch.cuda.Stream() for _ in range(N_LAYERS)]
+    xin = [xs[l] for l in order]                   # stream j serves layer order[j] on its input
+    outs = [torch.empty_like(x) for x in xin]
+    wss = [api.workspace(L.h, x.shape[0]) for x in xin]
+    for rep in range(3):
+        for j, st in enumerate(streams):
+            api.asap_moe_layer_dyn(L.h, slots[j:j + 1], xin[j], outs[j], wss[j], stream=st)
+    torch.cuda.synchronize()
+    for j in range(N_LAYERS):
+        assert same_bits(outs[j], ref[order[j]]), j
+    assert_clean(L.h)
+
+
 def test_layer_id_out_of_range_is_reported_and_uses_layer_0():
     cfg = DS_SMALL
     L = Layers.get(cfg)

@@ -140,6 +140,52 @@ def test_grouped_sigmoid_matches_brute_force():
         assert np.allclose(w, wb, rtol=1e-13, atol=0)
 
 
+def _brute_grouped_bias(l, b, k, G, kg, scale):
+    """Brute force of the biased rule: experts and groups are chosen by the
+    selection score sigmoid(l) + b; the weights use sigmoid(l) alone."""
+    s = [1 / (1 + math.exp(-v)) for v in l]
+    key = [s[i] + b[i] for i in range(len(l))]
+    E = len(l)
+    gsz = E // G
+    gscore = [max(key[a] + key[c] for a, c in itertools.combinations(range(g * gsz, (g + 1) * gsz), 2))
+              for g in range(G)]
+    best = None
+    for Gs in itertools.combinations(range(G), kg):
+        kk = (sum(gscore[g] for g in Gs), tuple(-g for g in Gs))
+        if best is None or kk > best[0]:
+            best = (kk, Gs)
+    cand = [e for g in best[1] for e in range(g * gsz, (g + 1) * gsz)]
+    bestS = None
+    for S in itertools.combinations(cand, k):
+        kk = (sum(key[i] for i in S), tuple(-i for i in sorted(S)))
+        if bestS is None or kk > bestS[0]:
+            bestS = (kk, S)
+    S = sorted(bestS[1], key=lambda i: (-key[i], i))
+    tot = sum(s[i] for i in S)
+    return S, [s[i] / tot * scale for i in S]
+
+
+def test_grouped_sigmoid_with_bias_matches_brute_force():
+    """The selection bias moves which experts are chosen but not their
+    weights; a large bias on a weak expert must select it."""
+    rng = np.random.default_rng(14)
+    for _ in range(150):
+        l = rng.normal(0, 1.0, 16)
+        b = rng.normal(0, 0.3, 16)
+        idx, w = gating.route_token_sigmoid_grouped(l, 4, 4, 2, 2.5, bias=b)
+        S, wb = _brute_grouped_bias(list(l), list(b), 4, 4, 2, 2.5)
+        assert list(idx) == S
+        assert np.allclose(w, wb, rtol=1e-13, atol=0)
+    l = np.zeros(16)
+    l[0] = 3.0
+    b = np.zeros(16)
+    b[9] = 5.0                                   # expert 9 (group 2) wins on its bias alone
+    idx, w = gating.route_token_sigmoid_grouped(l, 2, 4, 2, 1.0, bias=b)
+    assert list(idx) == [9, 0]
+    s = 1 / (1 + np.exp(-l))
+    assert np.allclose(w, [s[9] / (s[9] + s[0]), s[0] / (s[9] + s[0])], rtol=1e-13)
+
+
 def test_grouped_sigmoid_group_tie_lower_group_wins():
     # groups of 4; groups 1 and 2 tie on the top-2 sum, group 0 is best
     l = np.array([3.0, 2.9, -5, -5,   1.0, 0.5, -5, -5,   0.5, 1.0, -5, -5,   -3, -3, -3, -3])
