@@ -307,7 +307,10 @@ def run_ours(args, dist):
     code, word = api.asap_moe_status(h)
     if code != 0:
         raise RuntimeError(f"device status word {word:#x} after the timed region")
-    launches_per_mb = 7   # router, gate, scan, dispatch, gate/up GEMM, down GEMM, combine
+    # route (one kernel for E = 256 with grouped sigmoid gating, else router,
+    # gate and scan), dispatch, gate/up GEMM, down GEMM, combine
+    fused = cfg.n_experts == 256 and cfg.gating == "sigmoid_grouped" and cfg.n_groups in (1, 2, 4, 8)
+    launches_per_mb = (1 if fused else 3) + 4
     result = {
         "metric": METRIC,
         "value": dist.world * tokens_per_step * args.steps / (elapsed_ms / 1e3),

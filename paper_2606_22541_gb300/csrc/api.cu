@@ -154,7 +154,8 @@ int check_call(asap_moe_t h, int32_t n, void* ws, size_t ws_bytes, bool needs_ws
 
 // Number of K slices of the tensor-core router GEMM for n tokens: enough
 // CTAs to cover the SMs (one 128-row tile x one 256-expert tile per slice),
-// at least 8 k-blocks per slice.
+// at least 8 k-blocks per slice, and 1, 2 or 4 (the fused route kernel's
+// cluster gives each CTA 4 / slices of a tile's 32-token quarters).
 int router_splits(asap_moe_t h, int n) {
   if (!h->tc_router) return 1;
   const int mtiles = asap::ceil_div(n, asap::kGemmBM);
@@ -162,8 +163,28 @@ int router_splits(asap_moe_t h, int n) {
   int s = h->num_sms / std::max(mtiles, 1);
   s = std::min(s, kit / 8);
   s = std::min(s, asap::kMaxRouterSplits);
-  return std::max(s, 1);
+  int p = 1;
+  while (p * 2 <= s) p *= 2;
+  return p;
 }
+
+// Routing in one launch (router GEMM + gating + scan): E = 256 with grouped
+// sigmoid gating in 1, 2, 4 or 8 groups.  Other configurations run the
+// router, gate and scan kernels one after the other.
+bool fused_route(asap_moe_t h) {
+  const asap_moe_config& c = h->cfg;
+  return h->tc_router && c.gating == ASAP_GATE_SIGMOID_GROUPED &&
+         (c.n_groups == 1 || c.n_groups == 2 || c.n_groups == 4 || c.n_groups == 8);
+}
+
+// The fused route launch for n tokens of x.  With ticket (zero at launch)
+// its last CTA scans the histogram into chunk_base, counts and offsets and
+// zeroes tile_counters (nullable); without, hist columns [chunk0, chunk0 +
+// ceil(n/32)) of n_chunks_total are left for one scan over several
+// micro-batches.
+int run_route_fused(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* hist, int chunk0,
+                    int n_chunks_total, int32_t* ticket, int32_t* counts, int32_t* offsets, int32_t* chunk_base,
+                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st);
 
 // Router logits as ``splits`` planes of partial sums [splits][n][E] (planes
 // are added in order by the consumer); splits == 1 writes the logits.
@@ -202,6 +223,43 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
   return ASAP_OK;
 }
 
+int run_route_fused(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* hist, int chunk0,
+                    int n_chunks_total, int32_t* ticket, int32_t* counts, int32_t* offsets, int32_t* chunk_base,
+                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st) {
+  const asap_moe_config& c = h->cfg;
+  CUtensorMap tmx;
+  std::string err;
+  if (!asap::encode_tmap_bf16(&tmx, x, n, c.hidden, asap::kGemmBM, &err)) return fail(ASAP_ERR_INVALID, "x: " + err);
+  asap::RouteFusedArgs a{};
+  a.lref = lref(h, layer);
+  a.status = h->status;
+  a.n = n;
+  a.k_iters = c.hidden / asap::kGemmBK;
+  a.splits = router_splits(h, n);
+  a.top_k = c.top_k;
+  a.n_groups = c.n_groups;
+  a.topk_groups = c.topk_groups;
+  a.route_scale = c.route_scale;
+  a.idx = idx;
+  a.w = w;
+  a.hist = hist;
+  a.chunk0 = chunk0;
+  a.n_chunks_total = n_chunks_total;
+  a.ticket = ticket;
+  a.counts = counts;
+  a.offsets = offsets;
+  a.chunk_base = chunk_base;
+  a.tile_counters = tile_counters;
+  CU_TRY(asap::launch_route_fused(tmx, a, st), "fused route launch");
+  return ASAP_OK;
+}
+
+// Routing of one micro-batch into idx, w, counts, offsets and the
+// workspace's chunk bases; also zeroes the workspace's tile counters for the
+// grouped GEMMs that follow on the stream.
+int run_route(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* counts, int32_t* offsets,
+              void* ws, const int32_t* layer, cudaStream_t st);
+
 // ticket: the scan's ticket in the call's scratch (zeroed by the gate launch).
 asap::GateParams gate_params(asap_moe_t h, const int32_t* layer, int32_t* ticket) {
   const asap_moe_config& c = h->cfg;
@@ -229,6 +287,24 @@ int run_gate_scan(asap_moe_t h, const float* logits, int splits, int n, int32_t*
                            ticket, st, at<int32_t>(ws, L.tile_counters)),
          "scan launch");
   return ASAP_OK;
+}
+
+int run_route(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* counts, int32_t* offsets,
+              void* ws, const int32_t* layer, cudaStream_t st) {
+  const Layout L = layout(h->cfg, n);
+  if (fused_route(h)) {
+    // the tile counters and the ticket, one memset (the ticket follows them)
+    static_assert(asap::kTileCounters * 4 <= 256, "tile counters fit before the ticket");
+    CU_TRY(cudaMemsetAsync(at<char>(ws, L.tile_counters), 0, L.ticket - L.tile_counters + 4, st), "ticket");
+    return run_route_fused(h, x, n, idx, w, at<int32_t>(ws, L.hist), 0, asap::ceil_div(n, asap::kChunkTokens),
+                           at<int32_t>(ws, L.ticket), counts, offsets, at<int32_t>(ws, L.chunk_base),
+                           at<int32_t>(ws, L.tile_counters), layer, st);
+  }
+  float* logits = at<float>(ws, L.logits);
+  const int splits = router_splits(h, n);
+  int r = run_router_logits(h, x, n, logits, splits, layer, st);
+  if (r != ASAP_OK) return r;
+  return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, layer, st);
 }
 
 int ub_mtiles(const asap_moe_config& c, long long nk) {
@@ -657,6 +733,7 @@ ASAP_API int asap_moe_create_layers(const asap_moe_config* cfg, const asap_moe_w
                                                std::to_string(cc_major) + std::to_string(cc_minor)));
   e = asap::gemm_set_attributes();
   if (e == cudaSuccess) e = asap::fp8_gemm_set_attributes();
+  if (e == cudaSuccess) e = asap::route_fused_set_attributes();
   if (e != cudaSuccess) return bail(cuda_fail(e, "GEMM attributes"));
   h->fp8 = c.dtype == ASAP_FP8_E4M3_BLOCK128;
   h->tc_router = (c.n_experts == asap::kGemmBN);
@@ -727,11 +804,7 @@ ASAP_API int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !idx || !w || !counts || !offsets || !aligned16(x)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
-  float* logits = at<float>(ws, layout(h->cfg, n).logits);
-  const int splits = router_splits(h, n);
-  r = run_router_logits(h, x, n, logits, splits, h->layer_ids, S(stream));
-  if (r != ASAP_OK) return r;
-  return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, h->layer_ids, S(stream));
+  return run_route(h, x, n, idx, w, counts, offsets, ws, h->layer_ids, S(stream));
 }
 
 ASAP_API int asap_moe_dispatch(asap_moe_t h, const void* x, int32_t n, const int32_t* idx, void* x_perm,
@@ -875,9 +948,7 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
   int32_t* counters = at<int32_t>(ws, L.tile_counters);  // zeroed by the scan kernel
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
-  const int splits = router_splits(h, n);
-  if ((r = run_router_logits(h, x, n, logits, splits, layer, st)) != ASAP_OK) return r;
-  if ((r = run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, layer, st)) != ASAP_OK) return r;
+  if ((r = run_route(h, x, n, idx, w, counts, offsets, ws, layer, st)) != ASAP_OK) return r;
   if (h->fp8) {
     void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
@@ -947,7 +1018,12 @@ int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const 
   int tok0 = 0, chunk0 = 0;
   for (int i = 0; i < count; ++i) {
     const int n = ns[i];
-    if (n > 0) {
+    if (n > 0 && fused_route(h)) {
+      if ((r = run_route_fused(h, xs[i], n, idx + static_cast<long long>(tok0) * k,
+                               w + static_cast<long long>(tok0) * k, hist, chunk0, chunks_total, nullptr, nullptr,
+                               nullptr, nullptr, nullptr, layer, st)) != ASAP_OK)
+        return r;
+    } else if (n > 0) {
       const int splits = router_splits(h, n);
       float* lg = logits + static_cast<long long>(asap::kMaxRouterSplits) * tok0 * E;
       if ((r = run_router_logits(h, xs[i], n, lg, splits, layer, st)) != ASAP_OK) return r;
@@ -960,7 +1036,9 @@ int run_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const 
     chunk0 += asap::ceil_div(n, asap::kChunkTokens);
   }
   // one histogram scan over every chunk: expert segments hold the rows of all
-  // micro-batches, in (micro-batch, token, slot) order
+  // micro-batches, in (micro-batch, token, slot) order (the scan's ticket is
+  // zero at launch: the gate kernels zero it, the fused route does not)
+  if (fused_route(h)) CU_TRY(cudaMemsetAsync(at<int32_t>(ws, L.ticket), 0, 4, st), "ticket");
   CU_TRY(asap::launch_scan(hist, chunks_total, E, at<int32_t>(ws, L.counts), offsets, base, at<int32_t>(ws, L.ticket),
                            st, at<int32_t>(ws, L.tile_counters)),
          "scan launch");
@@ -1160,12 +1238,19 @@ ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int3
   int32_t* hist = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes);
   int32_t* base = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + kStaticChunkBytes);
   cudaStream_t st = S(stream);
+  int32_t* ticket = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + 2 * kStaticChunkBytes);
+  if (fused_route(h)) {
+    // the same single launch as asap_moe_route (same K slices, same bits);
+    // its ticket must start at zero, the rest is written before it is read
+    CU_TRY(cudaMemsetAsync(ticket, 0, sizeof(int32_t), st), "ticket");
+    return run_route_fused(h, x, n, idx, w, hist, 0, asap::ceil_div(n, asap::kChunkTokens), ticket, counts, offsets,
+                           base, nullptr, h->layer_ids, st);
+  }
   // every scratch element read below is written earlier on the same stream
   // (logits by the router, all E entries of each chunk's histogram and the
   // scan's ticket by the gate kernel), so nothing has to be cleared between
   // calls
   if ((r = run_router_logits(h, x, n, logits, 1, h->layer_ids, st)) != ASAP_OK) return r;
-  int32_t* ticket = reinterpret_cast<int32_t*>(scratch + kStaticLogitsBytes + 2 * kStaticChunkBytes);
   CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h, h->layer_ids, ticket), idx, w, hist, st), "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
                            ticket, st),

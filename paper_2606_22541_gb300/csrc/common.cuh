@@ -27,7 +27,7 @@ __device__ __forceinline__ void record_status(uint32_t* st, uint32_t bits) {
 }
 
 constexpr int kChunkTokens = 32;  // tokens per routing / dispatch chunk (one warp each)
-constexpr int kMaxRouterSplits = 8;  // K slices of the tensor-core router GEMM
+constexpr int kMaxRouterSplits = 4;  // K slices of the tensor-core router GEMM (1, 2 or 4)
 constexpr int kMaxExperts = 256;
 constexpr int kMaxTopK = 8;
 
@@ -39,6 +39,17 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);  // lo -> low half
   return *reinterpret_cast<uint32_t*>(&p);
 }
+
+// ---------------------------------------------------------------- gating
+// Sigmoid score of a router logit (grouped gating): 1 / (1 + e^-l) with the
+// fast exponential and reciprocal.  __expf(x) is within 2 + 1.16|x| ulp
+// (CUDA's documented bound) and __fdividef(1, y) within 2 ulp for y in
+// [1, 2^126]; the sigmoid's slope sigma (1 - sigma) is at most 1/4 and falls
+// like e^-|l|, so the score is within 5 * 2^-24 of the sigmoid of the float32
+// logit.  Every gate kernel uses this one expression, so all routing paths
+// give the same bits.  (No slow-path branch, unlike the IEEE division: the
+// compiler can overlap the scores of one thread.)
+__device__ __forceinline__ float gate_sigmoid(float l) { return __fdividef(1.0f, 1.0f + __expf(-l)); }
 
 // ---------------------------------------------------------------- smem / timers
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

@@ -129,25 +129,54 @@ struct GateParams {
 cudaError_t launch_router_small(const void* x, const LayerRef& lref, int n, int H, int E, float* logits,
                                 uint32_t* status, cudaStream_t s);
 // logits: ``splits`` planes of [n, E] partial sums, added in plane order.
-// hist is written expert-major: hist[e * n_chunks + chunk].
+// hist is written chunk-major: hist[chunk * E + e].
 cudaError_t launch_gate(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                         int32_t* hist, cudaStream_t s);
 cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane, float* out, cudaStream_t s);
 // Gating of one micro-batch among several served together: its chunks are
-// columns [chunk0, chunk0 + ceil(n/32)) of the expert-major histogram with
-// n_chunks_total columns.
+// rows [chunk0, chunk0 + ceil(n/32)) of the chunk-major histogram with
+// n_chunks_total rows.
 cudaError_t launch_gate_seg(const float* logits, int splits, int n, const GateParams& p, int32_t* idx, float* w,
                             int32_t* hist, int chunk0, int n_chunks_total, cudaStream_t s);
 // hist as launch_gate writes it; zeroes the scan's ticket.
 cudaError_t launch_hist(const int32_t* idx, int n, int k, int E, int32_t* hist, uint32_t* status, int32_t* ticket,
                         cudaStream_t s);
-// counts, offsets, and chunk_base[e][c] = entries of expert e in chunks
-// before c (relative: the absolute base is offsets[e] + chunk_base[e][c]).
+// counts, offsets, and chunk_base[c][e] = entries of expert e in chunks
+// before c (relative: the absolute base is offsets[e] + chunk_base[c][e]);
+// hist and chunk_base are chunk-major [n_chunks][E].
 // ticket: one int, zero at launch (the gate / hist launch zeroes it), left
 // zero.  tile_counters (nullable): kTileCounters ints zeroed for the grouped
 // GEMMs that follow on the stream.
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
                         int32_t* chunk_base, int32_t* ticket, cudaStream_t s, int32_t* tile_counters = nullptr);
+
+// Routing of one micro-batch in one launch (E = 256 on the tensor core,
+// grouped sigmoid gating with 1, 2, 4 or 8 groups): router logits over
+// ``splits`` K slices (a cluster of that many CTAs per 128-token tile, slices
+// added in order), gating, idx / w, the chunk-major histogram of its chunks
+// (rows chunk0 + c of n_chunks_total) and, when ticket is non-null, the
+// scan into chunk_base, counts and offsets by the last CTA (ticket zero at
+// launch, left zero) which also zeroes tile_counters (nullable).
+constexpr int kRouteExperts = 256;
+struct RouteFusedArgs {
+  LayerRef lref;  // router weights: table[layer].map[MAP_ROUTER]; selection bias
+  uint32_t* status;
+  int n, k_iters, splits;
+  int top_k, n_groups, topk_groups;
+  float route_scale;
+  int32_t* idx;
+  float* w;
+  int32_t* hist;
+  int chunk0, n_chunks_total;
+  int32_t* ticket;
+  int32_t* counts;
+  int32_t* offsets;
+  int32_t* chunk_base;
+  int32_t* tile_counters;
+};
+cudaError_t route_fused_set_attributes();
+// tmX: x [n, H] for [128, 64] boxes (encode_tmap_bf16).
+cudaError_t launch_route_fused(const CUtensorMap& tmX, const RouteFusedArgs& a, cudaStream_t s);
 
 // ------------------------------------------------------------ permute
 // Place of one micro-batch among several served by one call: its chunks start

@@ -35,8 +35,8 @@ __host__ __device__ constexpr int dispatch_warps() {
 // an entry inside its expert is (entries of that expert in earlier chunks)
 // + (in earlier warps of this chunk) + (in earlier lanes of this warp):
 // positions increase with (t, j) inside every segment.  chunk_base is
-// expert-major, relative to the expert's offset: the entries of expert e in
-// chunks before ``chunk`` are offsets[e] + chunk_base[e * n_chunks + chunk].
+// chunk-major, relative to the expert's offset: the entries of expert e in
+// chunks before ``chunk`` are offsets[e] + chunk_base[chunk * E + e].
 // Then one warp per token
 // reads its row once and writes it to its k positions.
 // Quantise 8 consecutive values of a 128-channel block held by 16 lanes
@@ -102,7 +102,7 @@ __global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
   }
   __syncthreads();
   for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
-    int run = seg.expert_offsets[ee] + chunk_base[static_cast<long long>(ee) * n_chunks + seg.chunk0 + c];
+    int run = seg.expert_offsets[ee] + chunk_base[static_cast<long long>(seg.chunk0 + c) * E + ee];
 #pragma unroll
     for (int w = 0; w < kRankWarps; ++w) {
       const int v = wcnt[w][ee];

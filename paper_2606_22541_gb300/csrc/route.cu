@@ -103,7 +103,7 @@ constexpr int kGateWarps = kChunkTokens;  // one warp per token of the chunk
 // arrive as ``splits`` partial planes (K slices of the router GEMM) that are
 // added in slice order.  Lane l holds experts l, l+32, ..., so expert order
 // and (i, lane) order agree.  The chunk's expert histogram is written
-// transposed: hist[e * n_chunks + chunk].
+// chunk-major: hist[chunk * E + e].
 __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __restrict__ logits, int splits,
                                                                long long plane, int n, GateParams p,
                                                                int32_t* __restrict__ idx,
@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
         for (int s2 = 1; s2 < splits; ++s2) l += lrow[s2 * plane + e];
       }
       if (grouped) {
-        const float s = 1.0f / (1.0f + expf(-l));
+        const float s = gate_sigmoid(l);
         sv[i] = s;
         key[i] = e < E ? s + (bias ? bias[e] : 0.0f) : -CUDART_INF_F;
       } else {
@@ -271,7 +271,7 @@ __global__ void __launch_bounds__(kGateWarps * 32) gate_kernel(const float* __re
   __syncthreads();
   if (hist)
     for (int e = threadIdx.x; e < E; e += blockDim.x)
-      hist[static_cast<long long>(e) * n_chunks + chunk0 + blockIdx.x] = shist[e];
+      hist[static_cast<long long>(chunk0 + blockIdx.x) * E + e] = shist[e];
 }
 
 // ------------------------------------------------------------ gating, a team of lanes per token
@@ -365,7 +365,7 @@ __global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float
     for (int j = 0; j < S; ++j) {
       if (!valid) l[j] = 0.f;
       if (grouped) {
-        const float sg = 1.0f / (1.0f + expf(-l[j]));
+        const float sg = gate_sigmoid(l[j]);
         val[j] = sg;
         key[j] = sg + (bias ? bias[e0 + j] : 0.0f);
       } else {
@@ -475,7 +475,7 @@ __global__ void __launch_bounds__(kChunkTokens * T) gate_team_kernel(const float
   __syncthreads();
   if (hist)
     for (int e = threadIdx.x; e < E; e += blockDim.x)
-      hist[static_cast<long long>(e) * n_chunks + chunk0 + blockIdx.x] = shist[e];
+      hist[static_cast<long long>(chunk0 + blockIdx.x) * E + e] = shist[e];
 }
 
 // ------------------------------------------------------------ histogram only
@@ -494,18 +494,20 @@ __global__ void __launch_bounds__(256) hist_kernel(const int32_t* __restrict__ i
     else record_status(status, ST_BAD_EXPERT_INDEX);
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(e) * n_chunks + blockIdx.x] = shist[e];
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[static_cast<long long>(blockIdx.x) * E + e] = shist[e];
 }
 
 // ------------------------------------------------------------ scan
-// One CTA per expert.  hist and chunk_base are stored expert-major
-// ([E][n_chunks]); CTA e scans its row with coalesced loads, writes
-// chunk_base[e][c] = the expert's entries in chunks before c (relative to the
-// expert's offset, which dispatch adds) and counts[e].  The last CTA to finish
-// (a ticket counter, zeroed by the kernel that wrote hist and reset here)
-// scans the counts into the exclusive offsets and clears the grouped GEMMs'
-// tile counters.
+// hist and chunk_base are chunk-major ([n_chunks][E]).  CTA g handles experts
+// 32g .. 32g+31 (lane = expert) and its 8 warps consecutive ranges of chunks:
+// each warp sums its range (128-byte rows), the warps' sums are combined in
+// shared memory, then each warp writes chunk_base[c][e] = the entries of
+// expert e in chunks before c (relative to the expert's offset, which
+// dispatch adds) over its range.  The last CTA to finish (ticket counter,
+// zero at launch, reset here) scans the counts into the exclusive offsets and
+// clears the grouped GEMMs' tile counters.
 constexpr int kScanThreads = 256;
+constexpr int kScanWarps = kScanThreads / 32;
 
 __device__ __forceinline__ int block_exclusive_scan(int v, int* swarp, int& total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -542,25 +544,41 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
                                                             int32_t* __restrict__ chunk_base,
                                                             int32_t* __restrict__ tile_counters,
                                                             int32_t* __restrict__ ticket) {
+  __shared__ int part[kScanWarps][32];
   __shared__ int swarp[33];
   __shared__ bool last;
-  const int e = blockIdx.x;
-  const int32_t* hrow = hist + static_cast<long long>(e) * n_chunks;
-  int32_t* brow = chunk_base + static_cast<long long>(e) * n_chunks;
-  int run = 0;
-  for (int c0 = 0; c0 < n_chunks; c0 += kScanThreads) {
-    const int c = c0 + threadIdx.x;
-    const int v = c < n_chunks ? hrow[c] : 0;
-    int tot = 0;
-    const int ex = block_exclusive_scan(v, swarp, tot);
-    if (c < n_chunks) brow[c] = run + ex;
-    run += tot;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int e = blockIdx.x * 32 + lane;
+  const bool ve = e < E;
+  const int per = (n_chunks + kScanWarps - 1) / kScanWarps;
+  const int c0 = min(n_chunks, warp * per), c1 = min(n_chunks, c0 + per);
+  int sum = 0;
+  if (ve) {
+#pragma unroll 8
+    for (int c = c0; c < c1; ++c) sum += hist[static_cast<long long>(c) * E + e];
   }
-  if (threadIdx.x == 0) {
-    counts[e] = run;
-    __threadfence();
-    last = atomicAdd(ticket, 1) == E - 1;
+  part[warp][lane] = sum;
+  __syncthreads();
+  int run = 0, total = 0;
+#pragma unroll
+  for (int w = 0; w < kScanWarps; ++w) {
+    const int v = part[w][lane];
+    if (w < warp) run += v;
+    total += v;
   }
+  if (ve) {
+#pragma unroll 8
+    for (int c = c0; c < c1; ++c) {
+      const long long o = static_cast<long long>(c) * E + e;
+      const int v = hist[o];
+      chunk_base[o] = run;
+      run += v;
+    }
+    if (warp == 0) counts[e] = total;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(ticket, 1) == static_cast<int>(gridDim.x) - 1;
   __syncthreads();
   if (!last) return;
   __threadfence();
@@ -656,7 +674,8 @@ cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane
 
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
                         int32_t* chunk_base, int32_t* ticket, cudaStream_t s, int32_t* tile_counters) {
-  scan_kernel<<<E, kScanThreads, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters, ticket);
+  scan_kernel<<<ceil_div(E, 32), kScanThreads, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters,
+                                                      ticket);
   return cudaGetLastError();
 }
 

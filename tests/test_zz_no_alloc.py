@@ -14,18 +14,23 @@ from paper_2606_22541_gb300.configs import DSV3
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda"
-# E = 256 puts the router on the tensor-core GEMM, the path whose logits go
-# into the static scratch; two micro-batches of different lengths
+# E = 256 puts the router on the tensor core; two micro-batches of different
+# lengths.  At hidden 512 the router has one K slice; at 2048 it splits K into
+# 4 slices over a thread-block cluster (700 and 4096 tokens).
 CFG = inputs.small_variant(DSV3, name="dsv3_noalloc", hidden=512, inter=256, shared_inter=256,
                            microbatches=[700, 301])
+CFG_WIDE = inputs.small_variant(DSV3, name="dsv3_noalloc_wide", hidden=2048, inter=128, shared_inter=128,
+                                microbatches=[700, 4096])
 
 
-@pytest.fixture(scope="module")
-def handle():
+@pytest.fixture(scope="module", params=[CFG, CFG_WIDE], ids=lambda c: c.name)
+def handle(request):
     import __graft_entry__
     __graft_entry__.build()
-    w = inputs.make_weights(CFG, DEV)
-    h = api.asap_moe_create(CFG, w, max(CFG.microbatches))
+    cfg = request.param
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
+    h.test_cfg = cfg
     yield h
     h.close()
 
@@ -39,8 +44,9 @@ def _outputs(n):
 
 
 def test_noalloc_route_equals_route_on_consecutive_calls(handle):
-    for i, n in enumerate(CFG.microbatches):       # two calls in a row
-        x = inputs.make_tokens(CFG, n, i, DEV)
+    cfg = handle.test_cfg
+    for i, n in enumerate(cfg.microbatches):       # two calls in a row
+        x = inputs.make_tokens(cfg, n, i, DEV)
         ref = _outputs(n)
         api.asap_moe_route(handle, x, *ref, api.workspace(handle, n))
         got = _outputs(n)
@@ -54,7 +60,7 @@ def test_noalloc_route_equals_route_on_consecutive_calls(handle):
 
 def test_noalloc_route_rejects_more_tokens_than_its_scratch(handle):
     from paper_2606_22541_gb300._native import AsapError
-    big = inputs.small_variant(CFG, name="dsv3_noalloc_big")
+    big = inputs.small_variant(handle.test_cfg, name="dsv3_noalloc_big")
     w = inputs.make_weights(big, DEV)
     h = api.asap_moe_create(big, w, 5000)
     try:
