@@ -83,6 +83,9 @@ __device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint32_t a, uint32_
   asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
                : "memory");
 }
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
 // All threads of every CTA of the cluster; orders shared and global memory
 // (release on arrive, acquire on wait).
 __device__ __forceinline__ void cluster_sync_all() {
@@ -261,23 +264,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int c_lo = (warp >> 2) * (kGemmBN / 2);
     const uint32_t owner = static_cast<uint32_t>(q % splits);
     const int j = q / splits;
-    const uint32_t slot = mapa_shared(base + static_cast<uint32_t>((j * splits + static_cast<int>(rank)) *
-                                                                   kSlotFloat4 * 16),
-                                      owner);
+    const uint32_t local = base + static_cast<uint32_t>((j * splits + static_cast<int>(rank)) * kSlotFloat4 * 16);
+    const bool remote = owner != rank;  // the own quarter stays in this CTA
+    const uint32_t slot = remote ? mapa_shared(local, owner) : local;
     const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-#pragma unroll 1
-    for (int c = c_lo; c < c_lo + kGemmBN / 2; c += 32) {
-      uint32_t v0[16], v1[16];
-      tmem_ld16(taddr + c, v0);
-      tmem_ld16(taddr + c + 16, v1);
-      tmem_ld_wait();
+    // all 128 columns in flight before one wait, then the stores
+    uint32_t v[4][32];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
+    for (int u = 0; u < 4; ++u) tmem_ld32(taddr + c_lo + 32 * u, v[u]);
+    tmem_ld_wait();
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
         // float4 (experts 4f .. 4f+3) of this token: (f * 32 + token) in the slot
-        st_cluster_v4(slot + static_cast<uint32_t>(((c / 4 + i) * 32 + lane) * 16), v0[4 * i], v0[4 * i + 1],
-                      v0[4 * i + 2], v0[4 * i + 3]);
-        st_cluster_v4(slot + static_cast<uint32_t>(((c / 4 + 4 + i) * 32 + lane) * 16), v1[4 * i],
-                      v1[4 * i + 1], v1[4 * i + 2], v1[4 * i + 3]);
+        const uint32_t ad = slot + static_cast<uint32_t>((((c_lo + 32 * u) / 4 + i) * 32 + lane) * 16);
+        if (remote)
+          st_cluster_v4(ad, v[u][4 * i], v[u][4 * i + 1], v[u][4 * i + 2], v[u][4 * i + 3]);
+        else
+          st_shared_v4(ad, v[u][4 * i], v[u][4 * i + 1], v[u][4 * i + 2], v[u][4 * i + 3]);
       }
     }
   }
@@ -485,19 +490,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     if (*last_flag) {
       __threadfence();
-      // thread e: expert e's column of the chunk-major histogram, 32 rows in
+      // thread e: expert e's column of the chunk-major histogram, 64 rows in
       // flight at a time
       const int e = threadIdx.x;
       const int nct = a.n_chunks_total;
       int run = 0;
 #pragma unroll 1
-      for (int c0 = 0; c0 < nct; c0 += 32) {
-        int v[32];
+      for (int c0 = 0; c0 < nct; c0 += 64) {
+        int v[64];
 #pragma unroll
-        for (int u = 0; u < 32; ++u)
+        for (int u = 0; u < 64; ++u)
           v[u] = c0 + u < nct ? __ldcg(a.hist + static_cast<long long>(c0 + u) * kRouteExperts + e) : 0;
 #pragma unroll
-        for (int u = 0; u < 32; ++u) {
+        for (int u = 0; u < 64; ++u) {
           if (c0 + u < nct) a.chunk_base[static_cast<long long>(c0 + u) * kRouteExperts + e] = run;
           run += v[u];
         }
