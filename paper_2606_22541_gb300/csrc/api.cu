@@ -351,6 +351,7 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   a.hint_b = kHintB;
   a.k_splits = 1;
   a.tile_counter = counter;
+  a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -396,6 +397,7 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.hint_b = kHintB;
   a.k_splits = 1;
   a.tile_counter = counter;
+  a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -452,6 +454,7 @@ int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t
   a.hint_b = kHintF8B;
   a.k_splits = 1;
   a.tile_counter = counter;
+  a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
   f.a_scale0 = xs;
   f.a_sld0 = c.hidden / 128;
   f.a_scale1 = xs_sh;
@@ -508,6 +511,7 @@ int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* o
   a.hint_b = kHintF8B;
   a.k_splits = 1;
   a.tile_counter = counter;
+  a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
   f.a_scale0 = hs;
   f.a_sld0 = c.inter / 128;
   f.a_scale1 = hs_sh;
@@ -621,21 +625,25 @@ int pack_layer(asap_moe_t h, const asap_moe_weights* wts, LayerWeights& L, cudaS
     if ((e = cudaMemcpyAsync(L.router_bias, wts->router_bias, E * 4, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
       return cuda_fail(e, "copy bias");
   }
+  // expert weights in the tile-contiguous order of the GEMMs' weight boxes
+  // (gate/up interleaved per 128 rows), so each box is one 32 KB read
   if ((e = cudaMalloc(&L.gate_up, gu_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc gate/up");
-  if ((e = asap::launch_pack_gate_up(wts->w_gate, wts->w_up, static_cast<int>(E), static_cast<int>(I),
-                                     static_cast<long long>(H * wb), L.gate_up, st)) != cudaSuccess)
+  if ((e = asap::launch_retile(wts->w_gate, wts->w_up, static_cast<int>(E), static_cast<int>(2 * I),
+                               static_cast<long long>(H * wb), true, L.gate_up, st)) != cudaSuccess)
     return cuda_fail(e, "pack gate/up");
   if ((e = cudaMalloc(&L.down, down_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc down");
-  if ((e = cudaMemcpyAsync(L.down, wts->w_down, down_bytes, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-    return cuda_fail(e, "copy down");
+  if ((e = asap::launch_retile(wts->w_down, nullptr, static_cast<int>(E), static_cast<int>(H),
+                               static_cast<long long>(I * wb), false, L.down, st)) != cudaSuccess)
+    return cuda_fail(e, "pack down");
   if (c.n_shared) {
     if ((e = cudaMalloc(&L.sh_gate_up, 2 * Is * H * wb)) != cudaSuccess) return cuda_fail(e, "cudaMalloc shared");
-    if ((e = asap::launch_pack_gate_up(wts->sh_gate, wts->sh_up, 1, static_cast<int>(Is),
-                                       static_cast<long long>(H * wb), L.sh_gate_up, st)) != cudaSuccess)
+    if ((e = asap::launch_retile(wts->sh_gate, wts->sh_up, 1, static_cast<int>(2 * Is), static_cast<long long>(H * wb),
+                                 true, L.sh_gate_up, st)) != cudaSuccess)
       return cuda_fail(e, "pack shared");
     if ((e = cudaMalloc(&L.sh_down, H * Is * wb)) != cudaSuccess) return cuda_fail(e, "cudaMalloc shared down");
-    if ((e = cudaMemcpyAsync(L.sh_down, wts->sh_down, H * Is * wb, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
-      return cuda_fail(e, "copy shared down");
+    if ((e = asap::launch_retile(wts->sh_down, nullptr, 1, static_cast<int>(H), static_cast<long long>(Is * wb), false,
+                                 L.sh_down, st)) != cudaSuccess)
+      return cuda_fail(e, "pack shared down");
   }
   if (h->fp8) {
     // scale rows interleaved like the weight rows: gate block b -> 2b, up block b -> 2b+1
@@ -675,9 +683,13 @@ int encode_layer(asap_moe_t h, const LayerWeights& L, asap::LayerEntry* out) {
   std::string err;
   if (h->tc_router && !asap::encode_tmap_bf16(&out->map[asap::MAP_ROUTER], L.router_w, E, H, asap::kGemmBN, &err))
     return fail(ASAP_ERR_CUDA, "router map: " + err);
+  // tile-contiguous expert weights (launch_retile): 128-byte rows, boxes of
+  // 256 consecutive rows
+  const uint64_t wb = h->fp8 ? 1 : 2;
   auto enc = [&](int which, const void* p, uint64_t rows, uint64_t cols) {
-    return h->fp8 ? asap::encode_tmap_u8(&out->map[which], p, rows, cols, asap::kGemmBN, &err)
-                  : asap::encode_tmap_bf16(&out->map[which], p, rows, cols, asap::kGemmBN, &err);
+    const uint64_t rows128 = rows * cols * wb / 128;
+    return h->fp8 ? asap::encode_tmap_u8(&out->map[which], p, rows128, 128, asap::kGemmBN, &err)
+                  : asap::encode_tmap_bf16(&out->map[which], p, rows128, 64, asap::kGemmBN, &err);
   };
   if (!enc(asap::MAP_GATE_UP, L.gate_up, E * 2 * I, H)) return fail(ASAP_ERR_CUDA, "gate/up map: " + err);
   if (!enc(asap::MAP_DOWN, L.down, E * H, I)) return fail(ASAP_ERR_CUDA, "down map: " + err);

@@ -251,6 +251,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       decode_tile(cur, sch, G, total0, args, T);
       const CUtensorMap* m = isB ? (T.p1 ? tmB1 : tmB0) : (T.p1 ? &tmA1 : &tmA0);
       const int row = isB ? T.b_row : T.a_row;
+      // tile-contiguous weights: box (b_row / BN, kb) is rows ((b_row / BN) k_iters + kb) BN
+      const bool tiled = isB && args.b_tiled;
+      const long long tile_row0 = static_cast<long long>(row / BN) * (T.p1 ? args.k_iters1 : args.k_iters0);
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
         const uint32_t full = isB ? fullB(stage) : fullA(stage);
         if (!mbar_wait(isB ? emptyB(stage) : emptyA(stage), phase ^ 1u, abort_flag)) {
@@ -258,7 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         mbar_arrive_expect_tx(full, bytes);
-        tma_load_2d(ring + stage * bytes, m, full, kb * BK, row, pol);
+        if (tiled)
+          tma_load_2d(ring + stage * bytes, m, full, 0, static_cast<int>((tile_row0 + kb) * BN), pol);
+        else
+          tma_load_2d(ring + stage * bytes, m, full, kb * BK, row, pol);
         pending |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
         if (++stage == nst) {

@@ -63,6 +63,7 @@ struct GemmArgs {
   LayerRef lref;           // B of problem p is lref.table[layer].map[bmap_p]
   int bmap0, bmap1;
   int* tile_counter;       // zero at launch: tiles are claimed dynamically; nullptr: static order
+  int b_tiled;             // B in tile-contiguous order (launch_retile): box row ((b_row/256) k_iters + kb) 256
 };
 
 constexpr int kTileCounters = 2;  // per call: gate/up GEMM, down GEMM
@@ -213,10 +214,14 @@ cudaError_t launch_dispatch_fp8_seg(const void* x, int n, int H, int k, int E, c
                                     const int32_t* chunk_base, void* xq, float* xs, void* xq_sh, float* xs_sh,
                                     int32_t* perm_src, int32_t* perm_dst, uint32_t* status, const DispatchSeg& seg,
                                     cudaStream_t s);
-// packed[e][b*256 + r] = gate[e][b*128 + r] (r < 128), up[...] for r >= 128
-// Rows are row_bytes wide (H * element size).
-cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, long long row_bytes, void* packed,
-                                cudaStream_t s);
+// Expert weights in tile-contiguous order for the grouped GEMMs' weight
+// boxes: box (e, nt, kb) = rows nt*256 .. nt*256+255 of expert e's packed
+// matrix ([E][R] rows of row_bytes; gate_up: packed row nt*256 + r is gate
+// row nt*128 + r for r < 128, else up row nt*128 + r - 128, a = gate, b = up),
+// bytes [kb*128, kb*128+128) of each row, stored as 256 consecutive 128-byte
+// rows.  R % 256 == 0 and row_bytes % 128 == 0.
+cudaError_t launch_retile(const void* a, const void* b, int E, int R, long long row_bytes, bool gate_up, void* dst,
+                          cudaStream_t s);
 
 inline int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
 

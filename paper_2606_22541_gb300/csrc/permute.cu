@@ -272,19 +272,32 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
 // packed[e][b*256 + r] = gate[e][b*128 + r] for r < 128, up[e][b*128 + r - 128]
 // otherwise, so one 256-row weight tile holds 128 gate rows and the matching
 // 128 up rows.
-__global__ void pack_gate_up_kernel(const uint4* __restrict__ gate, const uint4* __restrict__ up, int E,
-                                    int I, int V, uint4* __restrict__ packed) {
-  const long long total = static_cast<long long>(E) * 2 * I * V;
+// Tile-contiguous weights: 128-byte row pieces grouped per GEMM box.
+// dst box (e, nt, kb) = 256 consecutive rows of 128 B: rows nt*256 .. of
+// expert e's packed matrix, bytes [kb*128, kb*128 + 128) of each row; one box
+// is one contiguous 32 KB read from HBM.  gate_up: packed row r of tile nt is
+// gate row nt*128 + r (r < 128) or up row nt*128 + r - 128; else row nt*256 + r
+// of a.  R: packed rows per expert; V: 16-byte units per row.
+__global__ void retile_kernel(const uint4* __restrict__ a, const uint4* __restrict__ b, int E, int R, int V,
+                              bool gate_up, uint4* __restrict__ dst) {
+  const int KB = V / 8, NT = R / 256;
+  const long long total = static_cast<long long>(E) * R * V;
   for (long long q = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; q < total;
        q += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int v = static_cast<int>(q % V);
-    const long long rowq = q / V;
-    const int r = static_cast<int>(rowq % (2 * I));
-    const long long e = rowq / (2 * I);
-    const int b = r / 256, rr = r % 256;
-    const int src_row = b * 128 + (rr & 127);
-    const uint4* src = rr < 128 ? gate : up;
-    packed[q] = src[(e * I + src_row) * V + v];
+    const int v8 = static_cast<int>(q & 7);
+    long long t = q >> 3;
+    const int r = static_cast<int>(t & 255);
+    t >>= 8;
+    const int kb = static_cast<int>(t % KB);
+    t /= KB;
+    const int nt = static_cast<int>(t % NT);
+    const long long e = t / NT;
+    const uint4* src;
+    if (gate_up)
+      src = (r < 128 ? a : b) + (e * (R / 2) + nt * 128 + (r & 127)) * V;
+    else
+      src = a + (e * R + nt * 256 + r) * V;
+    dst[q] = src[kb * 8 + v8];
   }
 }
 
@@ -353,11 +366,13 @@ cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_pack_gate_up(const void* gate, const void* up, int E, int I, long long row_bytes, void* packed,
-                                cudaStream_t s) {
-  pack_gate_up_kernel<<<4096, 256, 0, s>>>(static_cast<const uint4*>(gate), static_cast<const uint4*>(up), E, I,
-                                           static_cast<int>(row_bytes / 16), static_cast<uint4*>(packed));
+cudaError_t launch_retile(const void* a, const void* b, int E, int R, long long row_bytes, bool gate_up, void* dst,
+                          cudaStream_t s) {
+  if (R % 256 != 0 || row_bytes % 128 != 0) return cudaErrorInvalidValue;
+  retile_kernel<<<4096, 256, 0, s>>>(static_cast<const uint4*>(a), static_cast<const uint4*>(b), E, R,
+                                     static_cast<int>(row_bytes / 16), gate_up, static_cast<uint4*>(dst));
   return cudaGetLastError();
 }
+
 
 }  // namespace asap
