@@ -200,7 +200,11 @@ int asap_moe_router_logits(asap_moe_t h, const void* x, int32_t n, float* logits
 
 /* Routing (Table 1: top-K of E_total experts; Section 3.2.1: per-expert token
  * counts): logits, gating, idx/w, counts, offsets.  counts and offsets are
- * deterministic. */
+ * deterministic.  For E = 256 with grouped sigmoid gating (1, 2, 4 or 8
+ * groups) this is one kernel launch (router GEMM over a thread-block cluster,
+ * gating and scan) after a 260-byte memset of the workspace's counters; the
+ * logits are not written.  Other configurations launch the router, gate and
+ * scan kernels in turn. */
 int asap_moe_route(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
                    int32_t* counts, int32_t* offsets, void* ws, size_t ws_bytes,
                    void* stream);
@@ -301,7 +305,10 @@ int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int
  *    GPU (for example on two streams without ordering between them) race and
  *    may return wrong routing; order them on one stream or with events.
  *  - The array keeps the last call's contents; every element a call reads is
- *    written earlier by the same call.                                      */
+ *    written earlier by the same call (the counter by a 4-byte memset on the
+ *    stream, which allocates nothing).
+ *  - For E = 256 with grouped sigmoid gating it runs the same single launch as
+ *    asap_moe_route and returns the same bits.                             */
 int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
                            int32_t* counts, int32_t* offsets, void* stream);
 

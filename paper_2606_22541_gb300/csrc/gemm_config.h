@@ -5,11 +5,12 @@
 
 // Ring depths (stages of A [128 x 64] and B [256 x 64] bf16 boxes).  A k-step
 // needs both boxes, so the pipeline depth that counts is that of the
-// shallowest ring whose operand comes from HBM.  gate/up (GU): both operands
-// from HBM, 4 + 4.  down (DN): its activations h are still in L2 from the
-// gate/up launch, 3 + 5 (1.84 -> 1.73 ms at 4096 DeepSeek-V3 tokens).  router
-// (RT): activations from HBM, the 256 x H router weights from L2, 6 + 3
-// (70.5 -> 64.5 us at 16384 tokens).
+// shallowest ring whose operand comes from HBM.  Measured at 4096 DeepSeek-V3
+// tokens with the weights in tile-contiguous order (one 32 KB read per box):
+// gate/up (GU) 4 + 4 (2.45 ms; 3 + 5: 2.58, 5 + 3: 2.69, 2 + 6: 3.23); down
+// (DN) 4 + 4 (1.34 ms; 3 + 5: 1.36, 2 + 6: 1.64, 3 + 4: 1.37).  router (RT):
+// activations from HBM, the 256 x H router weights from L2, 6 + 3 (70.5 ->
+// 64.5 us at 16384 tokens).
 #ifndef ASAP_RING_GU_A
 #define ASAP_RING_GU_A 4
 #endif
@@ -17,10 +18,10 @@
 #define ASAP_RING_GU_B 4
 #endif
 #ifndef ASAP_RING_DN_A
-#define ASAP_RING_DN_A 3
+#define ASAP_RING_DN_A 4
 #endif
 #ifndef ASAP_RING_DN_B
-#define ASAP_RING_DN_B 5
+#define ASAP_RING_DN_B 4
 #endif
 #ifndef ASAP_RING_RT_A
 #define ASAP_RING_RT_A 6

@@ -10,8 +10,9 @@
 // Design (one CTA per SM, persistent, warp-specialised, 224 threads):
 //   warps 0,6: TMA producers.  Weight boxes B [256 rows, 64 K] (warp 0) and
 //              activation boxes A [128 rows, 64 K] (warp 6) into separate
-//              shared-memory rings (4 + 4 stages, or 5 + 3 when the
-//              activations are L2-resident), 128-byte swizzle.
+//              shared-memory rings (depths per launch kind in
+//              gemm_config.h), 128-byte swizzle.  The weights are stored
+//              tile-contiguous (one 32 KB read per box).
 //   warp 1   : TMEM allocator and MMA issuer (one thread): 4 x
 //              tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) per stage,
 //              fp32 accumulator in TMEM, two accumulators (2 x 256 columns) so
