@@ -23,6 +23,8 @@ DS_ROUTE = inputs.small_variant(DSV3, name="dsv3_route", hidden=2048, inter=128,
                                 microbatches=[700, 10000])
 DS_ROUTE_G4 = inputs.small_variant(DS_ROUTE, name="dsv3_route_g4", n_groups=4, topk_groups=2, top_k=6)
 DS_ROUTE_G1 = inputs.small_variant(DS_ROUTE, name="dsv3_route_g1", n_groups=1, topk_groups=1)
+# a selection bias (it moves the selection keys and group scores, not the weights)
+DS_ROUTE_BIAS = inputs.small_variant(DS_ROUTE, name="dsv3_route_bias")
 SIZES = [1, 33, 130, 700, 5000, 10000]
 
 
@@ -38,8 +40,16 @@ _cache = {}
 def case(cfg):
     if cfg.name not in _cache:
         w = inputs.make_weights(cfg, DEV)
+        if cfg is DS_ROUTE_BIAS:
+            g = torch.Generator(device=DEV).manual_seed(4242)
+            w["router_bias"] = 0.05 * torch.randn(cfg.n_experts, generator=g, device=DEV)
         _cache[cfg.name] = (w, api.asap_moe_create(cfg, w, max(SIZES)), weights_f64(w))
     return _cache[cfg.name]
+
+
+def bias_of(w):
+    b = w.get("router_bias")
+    return None if b is None else b.cpu().numpy().astype(np.float32).astype(np.float64)
 
 
 def outputs(n, cfg):
@@ -50,7 +60,7 @@ def outputs(n, cfg):
             torch.full((E + 1,), -7, dtype=torch.int32, device=DEV))
 
 
-@pytest.mark.parametrize("cfg", [DS_ROUTE, DS_ROUTE_G4, DS_ROUTE_G1], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", [DS_ROUTE, DS_ROUTE_G4, DS_ROUTE_G1, DS_ROUTE_BIAS], ids=lambda c: c.name)
 @pytest.mark.parametrize("n", SIZES)
 def test_fused_route_against_oracle_and_composed_route(cfg, n):
     w, h, wf = case(cfg)
@@ -70,9 +80,10 @@ def test_fused_route_against_oracle_and_composed_route(cfg, n):
     L = oracle.router_logits(xf, wf["router_w"])
     eps = oracle.logit_error_bound(xf, wf["router_w"])
     ocfg = cfg.oracle_cfg()
-    idx_ref, w_ref = oracle.route(L, ocfg)
+    bias = bias_of(w)
+    idx_ref, w_ref = oracle.route(L, ocfg, bias)
     ig = idx.astype(np.int64)
-    decided = routing_check(L, eps, ocfg, ig, wt.astype(np.float64), w_ref, idx_ref)
+    decided = routing_check(L, eps, ocfg, ig, wt.astype(np.float64), w_ref, idx_ref, bias=bias)
     assert np.array_equal(counts, np.bincount(ig.reshape(-1), minlength=cfg.n_experts))
     assert offsets[0] == 0 and np.array_equal(np.diff(offsets), counts) and offsets[-1] == ig.size
     if decided.all():
