@@ -64,7 +64,7 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 constexpr int kMaxBatch = 64;  // micro-batches one asap_moe_layer_batched call may serve
 
-constexpr int kHintA = ASAP_HINT_BF16_A, kHintB = ASAP_HINT_BF16_B;
+constexpr int kHintA = ASAP_HINT_BF16_A, kHintB = ASAP_HINT_BF16_B, kHintDnA = ASAP_HINT_BF16_DN_A;
 constexpr int kHintF8A = ASAP_HINT_FP8_A, kHintF8B = ASAP_HINT_FP8_B;
 
 struct Layout {
@@ -393,7 +393,7 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.out1 = y_sh;
   a.ldo1 = c.hidden;
   a.status = h->status;
-  a.hint_a = kHintA;
+  a.hint_a = kHintDnA;
   a.hint_b = kHintB;
   a.k_splits = 1;
   a.tile_counter = counter;

@@ -43,6 +43,11 @@
 #ifndef ASAP_HINT_BF16_B
 #define ASAP_HINT_BF16_B 0
 #endif
+// the down GEMM's activations (h), re-read by every n-tile of their expert:
+// evict-last as for gate/up (measured: 1.33 ms; normal 1.35, evict-first 1.42)
+#ifndef ASAP_HINT_BF16_DN_A
+#define ASAP_HINT_BF16_DN_A ASAP_HINT_BF16_A
+#endif
 #ifndef ASAP_HINT_FP8_A
 #define ASAP_HINT_FP8_A 2
 #endif

@@ -374,5 +374,4 @@ cudaError_t launch_retile(const void* a, const void* b, int E, int R, long long 
   return cudaGetLastError();
 }
 
-
 }  // namespace asap
