@@ -215,7 +215,7 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
     a.k_splits = splits;
     a.split_rows0 = n;
     const int tiles = asap::ceil_div(n, asap::kGemmBM) * splits;
-    CU_TRY(asap::gemm_launch(asap::EPI_F32, maps, a, std::min(tiles, h->num_sms), st), "router GEMM launch");
+    CU_TRY(asap::gemm_launch(asap::EPI_F32, false, maps, a, std::min(tiles, h->num_sms), st), "router GEMM launch");
   } else {
     CU_TRY(asap::launch_router_small(x, lref(h, layer), n, c.hidden, c.n_experts, logits, h->status, st),
            "router launch");
@@ -307,8 +307,17 @@ int run_route(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_
   return run_gate_scan(h, logits, splits, n, idx, w, counts, offsets, ws, layer, st);
 }
 
-int ub_mtiles(const asap_moe_config& c, long long nk) {
-  return asap::ceil_div(nk, asap::kGemmBM) + static_cast<int>(std::min<long long>(c.n_experts, nk));
+// Paired m-tiles (two 128-row m-tiles per GEMM tile sharing the weight
+// boxes) when the routed segments hold at least ASAP_PAIR_ROWS rows per
+// expert on average: the grouped GEMMs are then bound by the tensor core
+// rather than by streaming the weights.
+bool use_pair(const asap_moe_config& c, long long nk) {
+  return nk >= static_cast<long long>(ASAP_PAIR_ROWS) * c.n_experts;
+}
+
+// Upper bound of the m-tiles of bm rows over the routed segments.
+int ub_mtiles(const asap_moe_config& c, long long nk, int bm = asap::kGemmBM) {
+  return asap::ceil_div(nk, bm) + static_cast<int>(std::min<long long>(c.n_experts, nk));
 }
 
 // GEMM1: h = silu(X Wg^T) * (X Wu^T) on the routed segments, plus the shared
@@ -319,12 +328,14 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
+  const bool pair = use_pair(c, nk);
+  const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
   CUtensorMap maps[2];
-  if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
+  if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, bm, &err))
     return fail(ASAP_ERR_INVALID, "x_perm: " + err);
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, bm, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
   } else {
     maps[1] = maps[0];
@@ -352,9 +363,10 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   a.k_splits = 1;
   a.tile_counter = counter;
   a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
-  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
-                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
-  CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk, bm)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, bm)) * a.n_tiles1 : 0);
+  CU_TRY(asap::gemm_launch(asap::EPI_SWIGLU, pair, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)),
+                           st),
          "gate/up GEMM launch");
   return ASAP_OK;
 }
@@ -365,12 +377,14 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
+  const bool pair = ASAP_PAIR_DOWN && use_pair(c, nk);
+  const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
   CUtensorMap maps[2];
-  if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
+  if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, bm, &err))
     return fail(ASAP_ERR_INVALID, "h: " + err);
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, asap::kGemmBM, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, bm, &err))
       return fail(ASAP_ERR_INVALID, "h_shared: " + err);
   } else {
     maps[1] = maps[0];
@@ -398,9 +412,9 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.k_splits = 1;
   a.tile_counter = counter;
   a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
-  const long long tiles = static_cast<long long>(ub_mtiles(c, nk)) * a.n_tiles0 +
-                          (sh ? static_cast<long long>(asap::ceil_div(n, asap::kGemmBM)) * a.n_tiles1 : 0);
-  CU_TRY(asap::gemm_launch(asap::EPI_BF16, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
+  const long long tiles = static_cast<long long>(ub_mtiles(c, nk, bm)) * a.n_tiles0 +
+                          (sh ? static_cast<long long>(asap::ceil_div(n, bm)) * a.n_tiles1 : 0);
+  CU_TRY(asap::gemm_launch(asap::EPI_BF16, pair, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
          "down GEMM launch");
   return ASAP_OK;
 }

@@ -23,6 +23,21 @@
 #ifndef ASAP_RING_DN_B
 #define ASAP_RING_DN_B 4
 #endif
+// paired m-tiles (two 128-row m-tiles per tile sharing the weight boxes, for
+// segments of at least ASAP_PAIR_ROWS rows on average): A boxes of 256 rows
+// (32 KB) and B boxes of 32 KB, 3 + 3 stages.
+#ifndef ASAP_RING_PAIR_A
+#define ASAP_RING_PAIR_A 3
+#endif
+#ifndef ASAP_RING_PAIR_B
+#define ASAP_RING_PAIR_B 3
+#endif
+#ifndef ASAP_PAIR_ROWS
+#define ASAP_PAIR_ROWS 256
+#endif
+#ifndef ASAP_PAIR_DOWN
+#define ASAP_PAIR_DOWN 1
+#endif
 #ifndef ASAP_RING_RT_A
 #define ASAP_RING_RT_A 6
 #endif

@@ -78,6 +78,8 @@ __device__ __forceinline__ int next_tile(const GemmArgs& a, int t) {
 
 // Tile t of the launch: problem 0 groups in order (inside a group: K slice,
 // then n-tile, then m-tile innermost), then problem 1 (n-tile, m-tile).
+// Tiles are BMT rows high.
+template <int BMT = kGemmBM>
 __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int total0,
                                             const GemmArgs& a, Tile& T) {
   if (t < total0) {
@@ -90,14 +92,14 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
     int local = t - s->tile_start[g];
     const int r0 = s->row_base[g];
     const int mrows = s->row_base[g + 1] - r0;
-    const int mt = (mrows + kGemmBM - 1) / kGemmBM;
+    const int mt = (mrows + BMT - 1) / BMT;
     const int per_split = mt * a.n_tiles0;
     const int split = local / per_split;   // K slice (split-K of problem 0)
     local -= split * per_split;
     const int nt = local / mt;
     const int mi = local - nt * mt;
-    T.a_row = r0 + mi * kGemmBM;
-    T.rows = min(kGemmBM, mrows - mi * kGemmBM);
+    T.a_row = r0 + mi * BMT;
+    T.rows = min(BMT, mrows - mi * BMT);
     T.b_row = g * a.b_stride0 + nt * kGemmBN;
     T.n_tile = nt;
     T.split = split;
@@ -107,11 +109,11 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
     T.p1 = false;
   } else {
     const int u = t - total0;
-    const int mt = (a.m1 + kGemmBM - 1) / kGemmBM;
+    const int mt = (a.m1 + BMT - 1) / BMT;
     const int nt = u / mt;
     const int mi = u - nt * mt;
-    T.a_row = mi * kGemmBM;
-    T.rows = min(kGemmBM, a.m1 - mi * kGemmBM);
+    T.a_row = mi * BMT;
+    T.rows = min(BMT, a.m1 - mi * BMT);
     T.b_row = nt * kGemmBN;
     T.n_tile = nt;
     T.split = 0;
@@ -123,9 +125,10 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
 }
 
 // Warp-level construction of the schedule table (called by one full warp):
-// per-group m-tile counts and their exclusive prefix; each lane owns up to 8
+// per-group counts of BMT-row m-tiles and their exclusive prefix; each lane owns up to 8
 // consecutive groups.  Offsets that are negative, not monotone or run past
 // the rows are reported in the status word and leave problem 0 empty.
+template <int BMT = kGemmBM>
 __device__ __forceinline__ void build_schedule(const GemmArgs& args, Sched* sch, int G, int lane) {
   int local = 0;
   int cnt[8];
@@ -144,7 +147,7 @@ __device__ __forceinline__ void build_schedule(const GemmArgs& args, Sched* sch,
         m = hi - lo[i];
         bad |= lo[i] < 0 || m < 0 || hi > args.m0;
       }
-      cnt[i] = (max(m, 0) + kGemmBM - 1) / kGemmBM;
+      cnt[i] = (max(m, 0) + BMT - 1) / BMT;
       local += cnt[i] * args.n_tiles0 * args.k_splits;
     }
   }

@@ -38,29 +38,39 @@ namespace asap {
 
 namespace {
 
-// Separate rings for the two operands, depths per launch kind (gemm_config.h).
-template <int EPI>
-struct Rings {
-  static constexpr int A = EPI == EPI_BF16 ? ASAP_RING_DN_A : EPI == EPI_SWIGLU ? ASAP_RING_GU_A : ASAP_RING_RT_A;
-  static constexpr int B = EPI == EPI_BF16 ? ASAP_RING_DN_B : EPI == EPI_SWIGLU ? ASAP_RING_GU_B : ASAP_RING_RT_B;
+// Shape of one launch kind.  PAIR: a tile is two 128-row m-tiles of the same
+// expert and n-tile that share every weight box (two M = 128 MMAs per K
+// step into the two halves of TMEM), for segments of at least 256 rows; each
+// weight box then feeds twice the MMA work, so the same ring bytes cover
+// twice the load latency.  Without PAIR a tile is one 128-row m-tile and the
+// two TMEM halves are ping-pong accumulators (the epilogue of one tile
+// overlaps the main loop of the next).  Ring depths per launch kind in
+// gemm_config.h.
+template <int EPI, bool PAIR>
+struct Gemm {
+  static constexpr int BMT = PAIR ? 2 * kGemmBM : kGemmBM;  // rows per tile
+  static constexpr int SA = PAIR ? ASAP_RING_PAIR_A
+                                 : EPI == EPI_BF16 ? ASAP_RING_DN_A : EPI == EPI_SWIGLU ? ASAP_RING_GU_A : ASAP_RING_RT_A;
+  static constexpr int SB = PAIR ? ASAP_RING_PAIR_B
+                                 : EPI == EPI_BF16 ? ASAP_RING_DN_B : EPI == EPI_SWIGLU ? ASAP_RING_GU_B : ASAP_RING_RT_B;
+  static constexpr int A_BYTES = BMT * kGemmBK * 2;
+  static constexpr int EPI_WARPS = PAIR ? 8 : 4;        // two per TMEM lane quarter with PAIR (one per half)
+  static constexpr int kThreads = 32 * (3 + EPI_WARPS);  // warp 0 B producer, 1 MMA, epilogue, last A producer
+  static constexpr int kAProdWarp = 2 + EPI_WARPS;
 };
 constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK;
 
-constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
-constexpr int kThreads = 224;  // warp 0 B producer, 1 MMA, 2-5 epilogue, 6 A producer
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
-
 
 constexpr int kBarBytes = 384;  // 2*SA + 2*SB + 5 + 2*kTileQ mbarriers, tmem slot, abort flag, tile ids
 // Dynamic shared memory: rings (1024-byte aligned for the 128-byte swizzle,
 // the alignment the kernel declares and checks), barriers, schedule table.
-template <int EPI>
+template <int EPI, bool PAIR>
 __host__ __device__ constexpr size_t smem_bytes() {
-  return Rings<EPI>::A * A_BYTES + Rings<EPI>::B * B_BYTES + kBarBytes + sizeof(Sched);
+  return Gemm<EPI, PAIR>::SA * Gemm<EPI, PAIR>::A_BYTES + Gemm<EPI, PAIR>::SB * B_BYTES + kBarBytes + sizeof(Sched);
 }
-
 
 
 template <int EPI>
@@ -134,13 +144,14 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
   }
 }
 
-template <int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int EPI, bool PAIR>
+__global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                         const __grid_constant__ CUtensorMap tmA1, const GemmArgs args) {
-  constexpr int SA = Rings<EPI>::A, SB = Rings<EPI>::B;
+  using C = Gemm<EPI, PAIR>;
+  constexpr int SA = C::SA, SB = C::SB, A_BYTES = C::A_BYTES, BMT = C::BMT;
   static_assert(8 * (2 * SA + 2 * SB + 5) + kTileQBytes + 8 <= kBarBytes, "barrier area");
-  static_assert(smem_bytes<EPI>() <= 227 * 1024, "shared memory budget");
+  static_assert(smem_bytes<EPI, PAIR>() <= 227 * 1024, "shared memory budget");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t base = smem_u32(smem_raw);
   if (base & 1023u) {  // uniform for the CTA: nothing is initialised yet
@@ -165,8 +176,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
-  // consumers of each queued tile id: A producer, MMA issuer, 4 epilogue warps
-  constexpr int kTileQConsumers = 6;
+  // consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
+  constexpr int kTileQConsumers = 2 + C::EPI_WARPS;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -193,7 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (int a = 0; a < 2; ++a) {
         mbar_init(tfull_bar(a), 1);
-        mbar_init(tempty_bar(a), 128);
+        mbar_init(tempty_bar(a), 32 * C::EPI_WARPS);
       }
       mbar_init(drain_bar, 1);
       TileQueue{tq_base}.init(kTileQConsumers);
@@ -206,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(tmB1);
       }
     }
-    build_schedule(args, sch, G, lane);
+    build_schedule<BMT>(args, sch, G, lane);
   } else if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
@@ -216,10 +227,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int total0 = sch->tile_start[G];
-  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BMT - 1) / BMT) * args.n_tiles1 : 0);
   TileQueue tq{tq_base};
 
-  if ((warp == 0 || warp == 6) && lane == 0) {
+  if ((warp == 0 || warp == C::kAProdWarp) && lane == 0) {
     // ------------------------------------------------------------ producers
     // warp 0 claims the tiles and streams their weight boxes (B) into its
     // ring, warp 6 the activation boxes (A) into its own; the MMA issuer joins
@@ -249,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (cur < 0) break;
       Tile T;
-      decode_tile(cur, sch, G, total0, args, T);
+      decode_tile<BMT>(cur, sch, G, total0, args, T);
       const CUtensorMap* m = isB ? (T.p1 ? tmB1 : tmB0) : (T.p1 ? &tmA1 : &tmA0);
       const int row = isB ? T.b_row : T.a_row;
       // tile-contiguous weights: box (b_row / BN, kb) is rows ((b_row / BN) k_iters + kb) BN
@@ -295,9 +306,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (t < 0) break;
       Tile T;
-      decode_tile(t, sch, G, total0, args, T);
-      const int acc = it & 1;
-      const uint32_t acc_phase = (it >> 1) & 1;
+      decode_tile<BMT>(t, sch, G, total0, args, T);
+      // PAIR: one tile accumulator (both TMEM halves); else ping-pong halves
+      const int acc = PAIR ? 0 : (it & 1);
+      const uint32_t acc_phase = PAIR ? (it & 1) : ((it >> 1) & 1);
       if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) {
         ok = false;
         break;
@@ -317,6 +329,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t adesc = BK == 64 ? smem_desc_sw128(a_addr + kk * 32) : smem_desc_sw64(a_addr + kk * 32);
           const uint64_t bdesc = BK == 64 ? smem_desc_sw128(b_addr + kk * 32) : smem_desc_sw64(b_addr + kk * 32);
           tc_mma_bf16(d, adesc, bdesc, kIdesc, (kb > T.kb0 || kk > 0) ? 1u : 0u);
+          if constexpr (PAIR) {
+            // rows 128 .. 255 of the A box (128 rows x 128 bytes further) into the other half
+            const uint32_t a_hi = a_addr + kGemmBM * BK * 2;
+            const uint64_t adesc_hi = BK == 64 ? smem_desc_sw128(a_hi + kk * 32) : smem_desc_sw64(a_hi + kk * 32);
+            tc_mma_bf16(tmem_base + BN, adesc_hi, bdesc, kIdesc, (kb > T.kb0 || kk > 0) ? 1u : 0u);
+          }
         }
         issued = true;
         tc_commit(emptyA(sa));
@@ -341,10 +359,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(drain_bar, 0, &dummy);
       }
     }
-  } else if (warp >= 2 && warp <= 5) {
+  } else if (warp >= 2 && warp < 2 + C::EPI_WARPS) {
     // ------------------------------------------------------------ epilogue
+    // warp w reads TMEM lanes 32 (w % 4) ..; with PAIR warps 2-5 take the
+    // tile's first 128 rows (TMEM columns 0 ..), warps 6-9 the next 128
+    // (columns 256 ..)
     const int q = warp & 3;
-    const int row = q * 32 + lane;
+    const int half = PAIR ? (warp - 2) >> 2 : 0;
+    const int row = half * kGemmBM + q * 32 + lane;
     for (int it = 0;; ++it) {
       int t = -1;
       const uint32_t qslot = tq.slot();
@@ -359,9 +381,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(tq.empty(qslot));
       if (t < 0) break;
       Tile T;
-      decode_tile(t, sch, G, total0, args, T);
-      const int acc = it & 1;
-      const uint32_t acc_phase = (it >> 1) & 1;
+      decode_tile<BMT>(t, sch, G, total0, args, T);
+      const int acc = PAIR ? 0 : (it & 1);
+      const uint32_t acc_phase = PAIR ? (it & 1) : ((it >> 1) & 1);
       const bool ok = __all_sync(0xffffffffu, mbar_wait(tfull_bar(acc), acc_phase, abort_flag));
       if (!ok) {
         if (lane == 0) {
@@ -371,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (PAIR ? half : acc) * BN;
       epilogue_tile<EPI>(T, args, taddr, row);
       tc_fence_before();
       mbar_arrive(tempty_bar(acc));
@@ -386,10 +408,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int EPI>
+template <int EPI, bool PAIR>
 cudaError_t set_attr() {
-  return cudaFuncSetAttribute(grouped_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(smem_bytes<EPI>()));
+  return cudaFuncSetAttribute(grouped_gemm_kernel<EPI, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(smem_bytes<EPI, PAIR>()));
+}
+
+template <int EPI, bool PAIR>
+void launch(const CUtensorMap* maps, const GemmArgs& args, int grid, cudaStream_t stream) {
+  grouped_gemm_kernel<EPI, PAIR><<<dim3(grid), dim3(Gemm<EPI, PAIR>::kThreads), smem_bytes<EPI, PAIR>(), stream>>>(
+      maps[0], maps[1], args);
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -416,26 +444,26 @@ EncodeFn get_encode_fn() {
 static_assert(sizeof(Sched) + 0 <= 8192, "schedule table");
 
 cudaError_t gemm_set_attributes() {
-  cudaError_t e = set_attr<EPI_SWIGLU>();
-  if (e == cudaSuccess) e = set_attr<EPI_BF16>();
-  if (e == cudaSuccess) e = set_attr<EPI_F32>();
+  cudaError_t e = set_attr<EPI_SWIGLU, false>();
+  if (e == cudaSuccess) e = set_attr<EPI_SWIGLU, true>();
+  if (e == cudaSuccess) e = set_attr<EPI_BF16, false>();
+  if (e == cudaSuccess) e = set_attr<EPI_BF16, true>();
+  if (e == cudaSuccess) e = set_attr<EPI_F32, false>();
   return e;
 }
 
-cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, int grid,
+cudaError_t gemm_launch(int epi, bool pair, const CUtensorMap* maps, const GemmArgs& args, int grid,
                         cudaStream_t stream) {
   if (grid <= 0) return cudaSuccess;
-  const dim3 g(grid), b(kThreads);
-  switch (epi) {
-    case EPI_SWIGLU:
-      grouped_gemm_kernel<EPI_SWIGLU><<<g, b, smem_bytes<EPI_SWIGLU>(), stream>>>(maps[0], maps[1], args);
-      break;
-    case EPI_BF16:
-      grouped_gemm_kernel<EPI_BF16><<<g, b, smem_bytes<EPI_BF16>(), stream>>>(maps[0], maps[1], args);
-      break;
-    default:
-      grouped_gemm_kernel<EPI_F32><<<g, b, smem_bytes<EPI_F32>(), stream>>>(maps[0], maps[1], args);
-      break;
+  if (epi == EPI_SWIGLU) {
+    if (pair) launch<EPI_SWIGLU, true>(maps, args, grid, stream);
+    else launch<EPI_SWIGLU, false>(maps, args, grid, stream);
+  } else if (epi == EPI_BF16) {
+    if (pair) launch<EPI_BF16, true>(maps, args, grid, stream);
+    else launch<EPI_BF16, false>(maps, args, grid, stream);
+  } else {
+    if (pair) return cudaErrorInvalidValue;
+    launch<EPI_F32, false>(maps, args, grid, stream);
   }
   return cudaGetLastError();
 }

@@ -75,9 +75,10 @@ constexpr int kGemmBN = 256;
 constexpr int kGemmBK = ASAP_GEMM_BK;  // 64 (128-byte swizzle) or 32 (64-byte swizzle)
 
 cudaError_t gemm_set_attributes();
-// maps: A0, A1 (A1 may repeat A0 when m1 == 0); the B maps come from the
-// layer table.
-cudaError_t gemm_launch(int epi, const CUtensorMap* maps, const GemmArgs& args, int grid,
+// maps: A0, A1 (A1 may repeat A0 when m1 == 0), encoded for boxes of 128 rows,
+// or 256 rows with pair; the B maps come from the layer table.  pair: tiles of
+// two 128-row m-tiles sharing the weight boxes (EPI_SWIGLU and EPI_BF16).
+cudaError_t gemm_launch(int epi, bool pair, const CUtensorMap* maps, const GemmArgs& args, int grid,
                         cudaStream_t stream);
 // Encode a 2-D row-major bf16 tensor [rows, cols] for 128-byte-swizzled
 // boxes of [box_rows, 64].  Returns false and fills *err on failure.

@@ -393,6 +393,33 @@ def test_streams_concurrent_equals_serial_and_token_independent(cfg):
     assert_clean(c)
 
 
+# 8 experts, top-2: 1100 tokens give 2200 >= 256 x 8 routed rows, so the grouped
+# GEMMs take tiles of two 128-row m-tiles sharing their weight boxes; 900
+# tokens (1800 rows) take single m-tiles.
+MX_PAIR = inputs.small_variant(MIXTRAL, name="mixtral_pair", hidden=512, inter=512, microbatches=[1100])
+
+
+def test_paired_m_tiles_match_oracle_and_single_tiles():
+    """The paired-tile GEMMs (large segments) against the oracle, and bit for
+    bit against the single-tile GEMMs on the tokens both calls share."""
+    c = Case.get(MX_PAIR)
+    x = c.tokens(0)
+    n = x.shape[0]
+    out = torch.empty_like(x)
+    api.asap_moe_layer(c.h, x, out, c.ws(n))
+    x9 = x[:900].contiguous()
+    out9 = torch.empty_like(x9)
+    api.asap_moe_layer(c.h, x9, out9, c.ws(900))
+    torch.cuda.synchronize()
+    assert torch.equal(out[:900].view(torch.int16), out9.view(torch.int16))
+    xf = bf16_to_f64(x)
+    r = oracle.moe_layer(xf, c.wf["router_w"], c.wf["w_gate"], c.wf["w_up"], c.wf["w_down"], c.ocfg)
+    eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+    decided = np.array([oracle.token_decided(r["logits"][t], eps[t], c.ocfg) for t in range(n)])
+    compare_rows(bf16_to_f64(out)[decided], r["y"][decided])
+    assert_clean(c)
+
+
 def test_edge_sizes():
     c = Case.get(DS_SMALL)
     H = DS_SMALL.hidden
