@@ -178,6 +178,25 @@ int asap_moe_create_layers(const asap_moe_config* cfg, const asap_moe_weights* w
 /* Number of layers of the handle (1 for asap_moe_create). */
 int asap_moe_n_layers(asap_moe_t h, int32_t* n_layers);
 
+/* Tile shape of the BF16 grouped expert GEMMs (gate/up and down) of the
+ * calls that follow on this handle (the FP8 GEMMs have one shape):
+ *  - ASAP_TILING_AUTO (the default): per launch, paired tiles when the
+ *    launch has at least three waves of them (estimated from n, top_k and
+ *    the expert count; one tile per SM per wave), else single tiles.
+ *  - ASAP_TILING_SINGLE: 128-row m-tiles.
+ *  - ASAP_TILING_PAIRED: two 128-row m-tiles of one expert per tile, sharing
+ *    every weight box; a segment's last <= 128 rows form a half tile.
+ * Every mode computes each output element with the same products in the same
+ * order, so the results are bit-identical; only the speed differs.  Another
+ * mode returns ASAP_ERR_INVALID.  Host state only (nothing is enqueued); do
+ * not call it while another thread enqueues on the same handle. */
+enum {
+  ASAP_TILING_AUTO = 0,
+  ASAP_TILING_SINGLE = 1,
+  ASAP_TILING_PAIRED = 2
+};
+int asap_moe_set_tiling(asap_moe_t h, int32_t mode);
+
 /* Free everything create allocated.  Synchronises the device first.  NULL is
  * accepted. */
 int asap_moe_destroy(asap_moe_t h);

@@ -59,6 +59,7 @@ SIGNATURES = {
     "asap_moe_layer_dyn": [_P, _P, _P, _I, _P, _P, _SZ, _P],
     "asap_moe_layer_batched_dyn": [_P, _P, _I, ctypes.POINTER(_P), ctypes.POINTER(_I), ctypes.POINTER(_P), _P, _SZ,
                                    _P],
+    "asap_moe_set_tiling": [_P, _I],
     "asap_moe_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "asap_moe_last_error": [],
 }

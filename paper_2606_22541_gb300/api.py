@@ -214,6 +214,15 @@ def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
                                        _ptr(offsets), _stream(stream)))
 
 
+TILING_AUTO, TILING_SINGLE, TILING_PAIRED = 0, 1, 2
+
+
+def asap_moe_set_tiling(h, mode):
+    """Tile shape of the BF16 grouped expert GEMMs: TILING_AUTO, _SINGLE or
+    _PAIRED (bit-identical results; only the speed differs)."""
+    check("asap_moe_set_tiling", lib().asap_moe_set_tiling(h.ptr, int(mode)))
+
+
 def asap_moe_status(h):
     """(code, raw status word); code is ASAP_OK or ASAP_ERR_DEVICE_STATUS."""
     word = ctypes.c_uint32()

@@ -39,6 +39,7 @@ struct asap_moe_s {
   uint32_t* status = nullptr;         // device status word
   bool tc_router = false;             // router GEMM on the tensor core (E == 256)
   bool fp8 = false;                   // e4m3 experts with fp32 128 x 128 block scales
+  int tiling = ASAP_TILING_AUTO;       // BF16 grouped GEMM tile shape (asap_moe_set_tiling)
 };
 
 namespace {
@@ -308,11 +309,18 @@ int run_route(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_
 }
 
 // Paired m-tiles (two 128-row m-tiles per GEMM tile sharing the weight
-// boxes) when the routed segments hold at least ASAP_PAIR_ROWS rows per
-// expert on average: the grouped GEMMs are then bound by the tensor core
-// rather than by streaming the weights.
-bool use_pair(const asap_moe_config& c, long long nk) {
-  return nk >= static_cast<long long>(ASAP_PAIR_ROWS) * c.n_experts;
+// boxes, a half tile for a segment's last <= 128 rows) unless the launch has
+// fewer than ASAP_PAIR_MIN_WAVES waves of paired tiles: the estimate takes
+// nk / 256 full tiles plus half a tile of rounding per non-empty segment.
+// With few tiles the larger tile rounds the launch to whole waves more
+// coarsely than it saves.
+bool use_pair(asap_moe_t h, long long nk, int n_tiles0, long long m1, int n_tiles1) {
+  if (h->tiling != ASAP_TILING_AUTO) return h->tiling == ASAP_TILING_PAIRED;
+  const asap_moe_config& c = h->cfg;
+  const long long seg = std::min<long long>(c.n_experts, nk);
+  const long long est = (asap::ceil_div(nk, 2 * asap::kGemmBM) + seg / 2) * n_tiles0 +
+                        asap::ceil_div(m1, 2 * asap::kGemmBM) * n_tiles1;
+  return est >= static_cast<long long>(ASAP_PAIR_MIN_WAVES) * h->num_sms;
 }
 
 // Upper bound of the m-tiles of bm rows over the routed segments.
@@ -328,14 +336,14 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
-  const bool pair = use_pair(c, nk);
+  const bool pair = use_pair(h, nk, c.inter / 128, sh ? n : 0, c.shared_inter / 128);
   const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
   CUtensorMap maps[2];
-  if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, bm, &err))
+  if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "x_perm: " + err);
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, bm, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
   } else {
     maps[1] = maps[0];
@@ -377,14 +385,14 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
-  const bool pair = ASAP_PAIR_DOWN && use_pair(c, nk);
+  const bool pair = use_pair(h, nk, c.hidden / asap::kGemmBN, sh ? n : 0, c.hidden / asap::kGemmBN);
   const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
   CUtensorMap maps[2];
-  if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, bm, &err))
+  if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "h: " + err);
   if (sh) {
-    if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, bm, &err))
+    if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "h_shared: " + err);
   } else {
     maps[1] = maps[0];
@@ -1174,6 +1182,14 @@ ASAP_API int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, i
 ASAP_API int asap_moe_n_layers(asap_moe_t h, int32_t* n_layers) {
   if (!h || !n_layers) return fail(ASAP_ERR_INVALID, "NULL handle or output");
   *n_layers = static_cast<int32_t>(h->layers.size());
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_set_tiling(asap_moe_t h, int32_t mode) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  if (mode != ASAP_TILING_AUTO && mode != ASAP_TILING_SINGLE && mode != ASAP_TILING_PAIRED)
+    return fail(ASAP_ERR_INVALID, "tiling mode must be ASAP_TILING_AUTO, _SINGLE or _PAIRED");
+  h->tiling = mode;
   return ASAP_OK;
 }
 

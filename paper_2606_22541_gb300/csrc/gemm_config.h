@@ -23,20 +23,23 @@
 #ifndef ASAP_RING_DN_B
 #define ASAP_RING_DN_B 4
 #endif
-// paired m-tiles (two 128-row m-tiles per tile sharing the weight boxes, for
-// segments of at least ASAP_PAIR_ROWS rows on average): A boxes of 256 rows
-// (32 KB) and B boxes of 32 KB, 3 + 3 stages.
+// paired m-tiles (two 128-row m-tiles per tile sharing the weight boxes): A
+// stages of 2 x 128 rows (32 KB) and B boxes of 32 KB, 3 + 3 stages.
 #ifndef ASAP_RING_PAIR_A
 #define ASAP_RING_PAIR_A 3
 #endif
 #ifndef ASAP_RING_PAIR_B
 #define ASAP_RING_PAIR_B 3
 #endif
-#ifndef ASAP_PAIR_ROWS
-#define ASAP_PAIR_ROWS 256
-#endif
-#ifndef ASAP_PAIR_DOWN
-#define ASAP_PAIR_DOWN 1
+// A launch runs paired m-tiles when it has at least this many waves of them
+// (estimated, one tile per SM per wave).  Measured on a GB300 against single
+// m-tiles: paired tiles (with half tiles for segment tails) win the gate/up
+// GEMM at every measured size (DeepSeek-V3 4096 tokens 2.40 vs 2.45 ms,
+// Mixtral 1024 tokens 0.44 vs 0.46 ms) and the down GEMM from about three
+// waves (Mixtral 4096 tokens, 3.8 waves: 0.61 vs 0.71 ms), but lose the
+// Mixtral down GEMM at 2.9 waves and below (3072 tokens 0.56 vs 0.53 ms).
+#ifndef ASAP_PAIR_MIN_WAVES
+#define ASAP_PAIR_MIN_WAVES 3
 #endif
 #ifndef ASAP_RING_RT_A
 #define ASAP_RING_RT_A 6

@@ -9,7 +9,7 @@
 //
 // Design (one CTA per SM, persistent, warp-specialised, 224 threads):
 //   warps 0,6: TMA producers.  Weight boxes B [256 rows, 64 K] (warp 0) and
-//              activation boxes A [128 rows, 64 K] (warp 6) into separate
+//              activation boxes A [128 rows, 64 K] (the last warp) into separate
 //              shared-memory rings (depths per launch kind in
 //              gemm_config.h), 128-byte swizzle.  The weights are stored
 //              tile-contiguous (one 32 KB read per box).
@@ -40,12 +40,13 @@ namespace {
 
 // Shape of one launch kind.  PAIR: a tile is two 128-row m-tiles of the same
 // expert and n-tile that share every weight box (two M = 128 MMAs per K
-// step into the two halves of TMEM), for segments of at least 256 rows; each
-// weight box then feeds twice the MMA work, so the same ring bytes cover
-// twice the load latency.  Without PAIR a tile is one 128-row m-tile and the
-// two TMEM halves are ping-pong accumulators (the epilogue of one tile
-// overlaps the main loop of the next).  Ring depths per launch kind in
-// gemm_config.h.
+// step into the two halves of TMEM); each weight box then feeds twice the MMA
+// work, so the same ring bytes cover twice the load latency.  The last tile
+// of a segment whose remaining rows fit one m-tile is a half tile: one A box
+// and one MMA per K step, so a segment pays for at most 127 padding rows, as
+// without PAIR.  Without PAIR a tile is one 128-row m-tile and the two TMEM
+// halves are ping-pong accumulators (the epilogue of one tile overlaps the
+// main loop of the next).  Ring depths per launch kind in gemm_config.h.
 template <int EPI, bool PAIR>
 struct Gemm {
   static constexpr int BMT = PAIR ? 2 * kGemmBM : kGemmBM;  // rows per tile
@@ -239,7 +240,7 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
     // them per k-step.
     const bool isB = warp == 0;
     const int nst = isB ? SB : SA;
-    const uint32_t bytes = isB ? B_BYTES : A_BYTES;
+    const uint32_t bytes = isB ? B_BYTES : A_BYTES;  // stage stride
     const uint32_t ring = isB ? sB : sA;
     const uint64_t pol = l2_policy(isB ? args.hint_b : args.hint_a);
     int stage = 0;
@@ -268,17 +269,22 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
       // tile-contiguous weights: box (b_row / BN, kb) is rows ((b_row / BN) k_iters + kb) BN
       const bool tiled = isB && args.b_tiled;
       const long long tile_row0 = static_cast<long long>(row / BN) * (T.p1 ? args.k_iters1 : args.k_iters0);
+      // A boxes are 128 rows: a paired tile loads two (rows 128 .. 255 land
+      // 128 x 128 bytes further, the layout of one 256-row box), a half tile one
+      const bool two = PAIR && !isB && T.rows > BM;
+      const uint32_t tx = isB ? B_BYTES : two ? A_BYTES : static_cast<uint32_t>(BM * BK * 2);
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
         const uint32_t full = isB ? fullB(stage) : fullA(stage);
         if (!mbar_wait(isB ? emptyB(stage) : emptyA(stage), phase ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(full, bytes);
+        mbar_arrive_expect_tx(full, tx);
         if (tiled)
           tma_load_2d(ring + stage * bytes, m, full, 0, static_cast<int>((tile_row0 + kb) * BN), pol);
         else
           tma_load_2d(ring + stage * bytes, m, full, kb * BK, row, pol);
+        if (two) tma_load_2d(ring + stage * bytes + BM * BK * 2, m, full, kb * BK, row + BM, pol);
         pending |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
         if (++stage == nst) {
@@ -318,6 +324,7 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
       }
       tc_fence_after();
       const uint32_t d = tmem_base + acc * BN;
+      const bool two = PAIR && T.rows > BM;  // else a half tile: the upper MMA is skipped
       for (int kb = T.kb0; kb < T.kb1; ++kb) {
         if (!mbar_wait(fullA(sa), pa, abort_flag) || !mbar_wait(fullB(sb), pb, abort_flag)) {
           ok = false;
@@ -331,8 +338,8 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
           const uint64_t adesc = BK == 64 ? smem_desc_sw128(a_addr + kk * 32) : smem_desc_sw64(a_addr + kk * 32);
           const uint64_t bdesc = BK == 64 ? smem_desc_sw128(b_addr + kk * 32) : smem_desc_sw64(b_addr + kk * 32);
           tc_mma_bf16(d, adesc, bdesc, kIdesc, (kb > T.kb0 || kk > 0) ? 1u : 0u);
-          if constexpr (PAIR) {
-            // rows 128 .. 255 of the A box (128 rows x 128 bytes further) into the other half
+          if (two) {
+            // rows 128 .. 255 of the A stage (128 rows x 128 bytes further) into the other half
             const uint32_t a_hi = a_addr + kGemmBM * BK * 2;
             const uint64_t adesc_hi = BK == 64 ? smem_desc_sw128(a_hi + kk * 32) : smem_desc_sw64(a_hi + kk * 32);
             tc_mma_bf16(tmem_base + BN, adesc_hi, bdesc, kIdesc, (kb > T.kb0 || kk > 0) ? 1u : 0u);
@@ -396,7 +403,8 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
       }
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (PAIR ? half : acc) * BN;
-      epilogue_tile<EPI>(T, args, taddr, row);
+      // the upper half of a half tile holds no rows (and no result)
+      if (half == 0 || T.rows > BM) epilogue_tile<EPI>(T, args, taddr, row);
       tc_fence_before();
       mbar_arrive(tempty_bar(acc));
     }

@@ -102,3 +102,11 @@ def test_create_layers_rejects_bad_layer_counts_before_touching_cuda(L):
     assert L.asap_moe_layer_batched_dyn(None, None, 1, None, None, None, None, 0, None) == _native.ASAP_ERR_INVALID
     n = ctypes.c_int32(0)
     assert L.asap_moe_n_layers(None, ctypes.byref(n)) == _native.ASAP_ERR_INVALID
+
+
+def test_tiling_modes_match_the_header(L):
+    text = open(HEADER).read()
+    vals = {m: int(v) for m, v in re.findall(r"ASAP_TILING_(\w+)\s*=\s*(\d+)", text)}
+    assert vals == {"AUTO": api.TILING_AUTO, "SINGLE": api.TILING_SINGLE, "PAIRED": api.TILING_PAIRED}
+    # a NULL handle is rejected on the host
+    assert L.asap_moe_set_tiling(None, api.TILING_AUTO) == _native.ASAP_ERR_INVALID

@@ -393,28 +393,33 @@ def test_streams_concurrent_equals_serial_and_token_independent(cfg):
     assert_clean(c)
 
 
-# 8 experts, top-2: 1100 tokens give 2200 >= 256 x 8 routed rows, so the grouped
-# GEMMs take tiles of two 128-row m-tiles sharing their weight boxes; 900
-# tokens (1800 rows) take single m-tiles.
+# 8 experts, top-2, 1100 tokens: about 275 routed rows per expert, so with
+# paired tiles every segment takes one full paired tile and one half tile.
 MX_PAIR = inputs.small_variant(MIXTRAL, name="mixtral_pair", hidden=512, inter=512, microbatches=[1100])
 
 
-def test_paired_m_tiles_match_oracle_and_single_tiles():
-    """The paired-tile GEMMs (large segments) against the oracle, and bit for
-    bit against the single-tile GEMMs on the tokens both calls share."""
-    c = Case.get(MX_PAIR)
+@pytest.mark.parametrize("cfg", [MX_PAIR, DS_SMALL], ids=lambda c: c.name)
+def test_paired_m_tiles_match_oracle_and_single_tiles(cfg):
+    """The paired-tile GEMMs (with half tiles at the segment tails, and on
+    the shared expert's rows) against the oracle, and bit for bit against the
+    single-tile GEMMs and the automatic choice."""
+    c = Case.get(cfg)
     x = c.tokens(0)
     n = x.shape[0]
-    out = torch.empty_like(x)
-    api.asap_moe_layer(c.h, x, out, c.ws(n))
-    x9 = x[:900].contiguous()
-    out9 = torch.empty_like(x9)
-    api.asap_moe_layer(c.h, x9, out9, c.ws(900))
+    outs = {}
+    try:
+        for mode in (api.TILING_SINGLE, api.TILING_PAIRED, api.TILING_AUTO):
+            api.asap_moe_set_tiling(c.h, mode)
+            outs[mode] = torch.empty_like(x)
+            api.asap_moe_layer(c.h, x, outs[mode], c.ws(n))
+    finally:
+        api.asap_moe_set_tiling(c.h, api.TILING_AUTO)
     torch.cuda.synchronize()
-    assert torch.equal(out[:900].view(torch.int16), out9.view(torch.int16))
-    xf = bf16_to_f64(x)
-    r = oracle.moe_layer(xf, c.wf["router_w"], c.wf["w_gate"], c.wf["w_up"], c.wf["w_down"], c.ocfg)
-    eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+    out = outs[api.TILING_PAIRED]
+    assert torch.equal(out.view(torch.int16), outs[api.TILING_SINGLE].view(torch.int16))
+    assert torch.equal(out.view(torch.int16), outs[api.TILING_AUTO].view(torch.int16))
+    r = oracle_layer(c, x)
+    eps = oracle.logit_error_bound(bf16_to_f64(x), c.wf["router_w"])
     decided = np.array([oracle.token_decided(r["logits"][t], eps[t], c.ocfg) for t in range(n)])
     compare_rows(bf16_to_f64(out)[decided], r["y"][decided])
     assert_clean(c)

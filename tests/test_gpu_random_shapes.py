@@ -2,8 +2,9 @@
 counts from 8 to 256, top-k 1..8, the three gating rules with random group
 counts, hidden sizes that do and do not split the router's K, with and
 without a shared expert, ragged token counts (some large enough for the
-paired-m-tile GEMMs).  Each case is drawn from its own seed, so a failure
-names a reproducible shape."""
+paired-m-tile GEMMs).  Each case also runs with single and with paired
+m-tiles forced, which must give the same bits.  Each case is drawn from its
+own seed, so a failure names a reproducible shape."""
 import numpy as np
 import pytest
 import torch
@@ -45,7 +46,8 @@ def random_config(i):
 # fixed shapes the draws may miss: E = 256 with grouped gating through the
 # one-launch route (8 groups, K split over a cluster) and through the gate
 # kernels (16 groups), E = 256 softmax-renorm with a shared expert, and a
-# Mixtral-like shape large enough for paired m-tiles
+# Mixtral-like shape with segments of about 275 rows (a paired and a half tile
+# each with paired m-tiles)
 FIXED = [
     LayerConfig("fixed_g8", hidden=2048, n_experts=256, top_k=8, inter=128, n_shared=1, shared_inter=128,
                 gating="sigmoid_grouped", n_groups=8, topk_groups=4, route_scale=2.5, microbatches=[777], seed=7101),
@@ -74,6 +76,12 @@ def test_random_shape_layer_matches_oracle(cfg):
         x = inputs.make_tokens(cfg, n, 0, DEV)
         out = torch.empty_like(x)
         api.asap_moe_layer(h, x, out, api.workspace(h, n))
+        forced = {}
+        for mode in (api.TILING_SINGLE, api.TILING_PAIRED):
+            api.asap_moe_set_tiling(h, mode)
+            forced[mode] = torch.empty_like(x)
+            api.asap_moe_layer(h, x, forced[mode], api.workspace(h, n))
+        api.asap_moe_set_tiling(h, api.TILING_AUTO)
         k, E = cfg.top_k, cfg.n_experts
         idx = torch.empty((n, k), dtype=torch.int32, device=DEV)
         wt = torch.empty((n, k), dtype=torch.float32, device=DEV)
@@ -81,6 +89,8 @@ def test_random_shape_layer_matches_oracle(cfg):
         offsets = torch.empty(E + 1, dtype=torch.int32, device=DEV)
         api.asap_moe_route(h, x, idx, wt, counts, offsets, api.workspace(h, n))
         torch.cuda.synchronize()
+        for mode, o in forced.items():
+            assert torch.equal(o.view(torch.int16), out.view(torch.int16)), f"tiling mode {mode}"
         wf = weights_f64(w)
         xf = bf16_to_f64(x)
         ocfg = cfg.oracle_cfg()
