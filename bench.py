@@ -221,7 +221,7 @@ def profile_traffic(name, source_files):
         return None, None
     if h.group(1) != sources_sha256(source_files):
         return None, "stale"
-    return float(m.group(1)), path
+    return float(m.group(1)), os.path.relpath(path, ROOT)
 
 
 def sources_sha256(files):

@@ -181,8 +181,9 @@ int asap_moe_n_layers(asap_moe_t h, int32_t* n_layers);
 /* Tile shape of the BF16 grouped expert GEMMs (gate/up and down) of the
  * calls that follow on this handle (the FP8 GEMMs have one shape):
  *  - ASAP_TILING_AUTO (the default): per launch, paired tiles when the
- *    launch has at least three waves of them (estimated from n, top_k and
- *    the expert count; one tile per SM per wave), else single tiles.
+ *    routed rows average at least 128 per expert and the launch has at least
+ *    three waves of paired tiles (estimated from n, top_k and the expert
+ *    count; one tile per SM per wave), else single tiles.
  *  - ASAP_TILING_SINGLE: 128-row m-tiles.
  *  - ASAP_TILING_PAIRED: two 128-row m-tiles of one expert per tile, sharing
  *    every weight box; a segment's last <= 128 rows form a half tile.

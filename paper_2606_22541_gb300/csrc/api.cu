@@ -309,14 +309,21 @@ int run_route(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_
 }
 
 // Paired m-tiles (two 128-row m-tiles per GEMM tile sharing the weight
-// boxes, a half tile for a segment's last <= 128 rows) unless the launch has
-// fewer than ASAP_PAIR_MIN_WAVES waves of paired tiles: the estimate takes
-// nk / 256 full tiles plus half a tile of rounding per non-empty segment.
-// With few tiles the larger tile rounds the launch to whole waves more
-// coarsely than it saves.
+// boxes, a half tile for a segment's last <= 128 rows) when
+//  - the segments hold at least one m-tile (128 rows) per expert on average:
+//    below that nearly every paired tile is a half tile, and the paired rings
+//    (3 + 3 stages) keep fewer weight bytes in flight than the single-tile
+//    rings (4 + 4).  Measured on a GB300 at the DeepSeek-V3 shape (gate/up |
+//    down ms, paired vs single): 3072 tokens (96 rows per expert) 2.26 |
+//    1.23 vs 2.19 | 1.16; 4096 tokens (128) 2.35 | 1.31 vs 2.39 | 1.33;
+//  - and the launch has at least ASAP_PAIR_MIN_WAVES waves of paired tiles
+//    (estimate: nk / 256 full tiles plus half a tile of rounding per
+//    non-empty segment).  With few tiles the larger tile rounds the launch to
+//    whole waves more coarsely than it saves.
 bool use_pair(asap_moe_t h, long long nk, int n_tiles0, long long m1, int n_tiles1) {
   if (h->tiling != ASAP_TILING_AUTO) return h->tiling == ASAP_TILING_PAIRED;
   const asap_moe_config& c = h->cfg;
+  if (nk < static_cast<long long>(asap::kGemmBM) * c.n_experts) return false;
   const long long seg = std::min<long long>(c.n_experts, nk);
   const long long est = (asap::ceil_div(nk, 2 * asap::kGemmBM) + seg / 2) * n_tiles0 +
                         asap::ceil_div(m1, 2 * asap::kGemmBM) * n_tiles1;
