@@ -250,6 +250,63 @@ def test_certified_comparison():
     assert n_decided > 40
 
 
+def _bf16_values(a):
+    """Round float64 values to bf16 (torch's round-to-nearest-even) and return them as float64."""
+    return torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).to(torch.float64).numpy()
+
+
+def _fp32_truncating_block_sums(prods, block=16):
+    """fp32 accumulation as a tensor-core MMA does it: each step adds a block
+    of ``block`` products (K of one bf16 MMA) to the accumulator in one
+    operation whose result is rounded toward zero (truncated) to fp32."""
+    n_blk = prods.shape[-1] // block
+    blocks = prods.reshape(*prods.shape[:-1], n_blk, block).astype(np.float64).sum(axis=-1)
+    acc = np.zeros(prods.shape[:-1], np.float32)
+    for i in range(n_blk):
+        t = acc.astype(np.float64) + blocks[..., i]
+        f = t.astype(np.float32)
+        over = np.abs(f.astype(np.float64)) > np.abs(t)
+        f[over] = np.nextafter(f[over], np.float32(0))
+        acc = f
+    return acc
+
+
+@pytest.mark.parametrize("case", ["configs", "cancelling"])
+def test_logit_error_bound_covers_fp32_accumulation_orders(case):
+    """The bound on |fp32 logit - exact logit| that the certified routing
+    comparison relies on holds, on inputs drawn like the configs' (x ~ N(0,1),
+    router weights ~ N(0, 0.02), bf16) and on rows whose logit nearly cancels,
+    for fp32 accumulation of the (exact) bf16 products in every order a router
+    kernel may use: sequential, reversed, blocked by the MMA's K = 16, split-K
+    slices added in slice order, and MMA steps of 16 products whose sums are
+    truncated instead of rounded."""
+    rng = np.random.default_rng({"configs": 31, "cancelling": 33}[case])
+    n, E, H = 24, 48, 7168
+    x, wr = rng.normal(0, 1, (n, H)), rng.normal(0, 0.02, (E, H))
+    if case == "cancelling":
+        # second half of every weight row cancels the first half's dot with x[0]
+        ratio = x[0, :H // 2] / np.where(np.abs(x[0, H // 2:]) < 1e-3, 1.0, x[0, H // 2:])
+        wr[:, H // 2:] = np.clip(-wr[:, :H // 2] * ratio[None, :], -0.1, 0.1)
+    x, wr = _bf16_values(x), _bf16_values(wr)
+    exact = x @ wr.T
+    eps = gating.logit_error_bound(x, wr)
+    prods = (x[:, None, :] * wr[None, :, :]).astype(np.float32)   # bf16 x bf16 is exact in fp32
+    assert np.array_equal(prods.astype(np.float64), x[:, None, :] * wr[None, :, :])
+    sums = {
+        "sequential": np.cumsum(prods, axis=2, dtype=np.float32)[..., -1],
+        "reversed": np.cumsum(prods[..., ::-1], axis=2, dtype=np.float32)[..., -1],
+        "k16_blocks": np.cumsum(prods.reshape(n, E, H // 16, 16).sum(axis=3, dtype=np.float32), axis=2,
+                                dtype=np.float32)[..., -1],
+        "split_k4": np.cumsum(np.stack([np.cumsum(q, axis=2, dtype=np.float32)[..., -1]
+                                        for q in np.split(prods, 4, axis=2)], axis=2), axis=2,
+                              dtype=np.float32)[..., -1],
+        "k16_truncating": _fp32_truncating_block_sums(prods),
+    }
+    for name, got in sums.items():
+        err = np.abs(got.astype(np.float64) - exact)
+        assert np.all(err <= eps), (case, name, float((err / eps).max()))
+
+
 # ---------------------------------------------------------------- counts / permutation
 
 def _random_idx(rng, n, E, k):
