@@ -66,73 +66,93 @@ constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
 constexpr int kBarBytes = 384;  // 2*SA + 2*SB + 5 + 2*kTileQ mbarriers, tmem slot, abort flag, tile ids
+// bf16 epilogues stage their stores through 4 KB of shared memory per warp
+// (32 rows x 8 chunks of 16 bytes)
+constexpr int kStageWarpBytes = 32 * 8 * 16;
+template <int EPI, bool PAIR>
+__host__ __device__ constexpr int stage_bytes() {
+  return EPI == EPI_F32 ? 0 : Gemm<EPI, PAIR>::EPI_WARPS * kStageWarpBytes;
+}
 // Dynamic shared memory: rings (1024-byte aligned for the 128-byte swizzle,
-// the alignment the kernel declares and checks), barriers, schedule table.
+// the alignment the kernel declares and checks), barriers, store staging,
+// schedule table.
 template <int EPI, bool PAIR>
 __host__ __device__ constexpr size_t smem_bytes() {
-  return Gemm<EPI, PAIR>::SA * Gemm<EPI, PAIR>::A_BYTES + Gemm<EPI, PAIR>::SB * B_BYTES + kBarBytes + sizeof(Sched);
+  return Gemm<EPI, PAIR>::SA * Gemm<EPI, PAIR>::A_BYTES + Gemm<EPI, PAIR>::SB * B_BYTES + kBarBytes +
+         stage_bytes<EPI, PAIR>() + sizeof(Sched);
 }
 
 
+// One round of a warp's coalesced stores: lane l holds 8 chunks of 16 bytes
+// (pk, 32 words) of its row l.  Every lane writes them to the warp's 4 KB
+// staging buffer (chunk j of row r at slot j ^ (r % 8), so neither side of
+// the exchange has bank conflicts), then lanes 8u .. 8u+7 store the 8 chunks
+// of rows u, u + 4, ...: each store instruction writes four rows x 128
+// contiguous bytes instead of 32 rows x 16 bytes.  Rows from ``valid_rows``
+// on are not stored.  out: the warp's first row at the round's first column.
+__device__ __forceinline__ void store_round(const uint32_t* pk, uint4* stage, int lane, uint16_t* out, long long ldo,
+                                            int valid_rows) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    stage[lane * 8 + (j ^ (lane & 7))] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+  __syncwarp();
+  const int ru = lane >> 3, cu = lane & 7;
+  uint16_t* dst = out + ru * ldo + cu * 8;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int r = ru + 4 * k;
+    const uint4 v = stage[r * 8 + (cu ^ (r & 7))];
+    if (r < valid_rows) *reinterpret_cast<uint4*>(dst + 4 * k * ldo) = v;
+  }
+  __syncwarp();
+}
+
+// TMEM -> packed bf16 for 64 output columns starting at output column c0:
+// SwiGLU tiles read gate columns c0 .. c0 + 63 and the matching up columns
+// BN / 2 further and form silu(g) u; plain tiles read columns c0 .. c0 + 63.
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr,
-                                              int row) {
-  const bool valid = row < T.rows;
-  // split-K slices of problem 0 write separate output planes
-  const long long orow = static_cast<long long>(T.a_row) + row + (T.p1 ? 0 : T.split * a.split_rows0);
-  if constexpr (EPI == EPI_SWIGLU) {
-    uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
-    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
-    uint16_t* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * (BN / 2);
-#pragma unroll 1
-    for (int c = 0; c < BN / 2; c += 16) {
-      uint32_t g[16], u[16];
-      tmem_ld16(taddr + c, g);
-      tmem_ld16(taddr + BN / 2 + c, u);
+__device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t* pk) {
+#pragma unroll
+  for (int c = 0; c < 64; c += 16) {
+    uint32_t g[16];
+    tmem_ld16(taddr + c0 + c, g);
+    if constexpr (EPI == EPI_SWIGLU) {
+      uint32_t u[16];
+      tmem_ld16(taddr + BN / 2 + c0 + c, u);
       tmem_ld_wait();
-      if (valid) {
-        uint32_t pk[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
-          const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
-          // silu(g) u with the fast exponential and divide (within a few
-          // fp32 ulp, far below h's bf16 rounding)
-          const float h0 = __fdividef(g0, 1.0f + __expf(-g0)) * u0;
-          const float h1 = __fdividef(g1, 1.0f + __expf(-g1)) * u1;
-          pk[i] = pack_bf16x2(h0, h1);
-        }
-        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
-        d4[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        d4[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      for (int i = 0; i < 8; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        // silu(g) u with the fast exponential and divide (within a few
+        // fp32 ulp, far below h's bf16 rounding)
+        pk[c / 2 + i] = pack_bf16x2(__fdividef(g0, 1.0f + __expf(-g0)) * u0, __fdividef(g1, 1.0f + __expf(-g1)) * u1);
       }
-    }
-  } else if constexpr (EPI == EPI_BF16) {
-    uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
-    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
-    uint16_t* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * BN;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t v0[16], v1[16];
-      tmem_ld16(taddr + c, v0);
-      tmem_ld16(taddr + c + 16, v1);
+    } else {
       tmem_ld_wait();
-      if (valid) {
-        uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          pk[i] = pack_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
-          pk[8 + i] = pack_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
-        }
-        uint4* d4 = reinterpret_cast<uint4*>(dst + c);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) d4[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-      }
+      for (int i = 0; i < 8; ++i) pk[c / 2 + i] = pack_bf16x2(__uint_as_float(g[2 * i]), __uint_as_float(g[2 * i + 1]));
     }
-  } else {
+  }
+}
+
+// Epilogue of one tile for the thread owning TMEM lane ``row`` (taddr: that
+// lane, the accumulator's first column); it arrives on ``tempty`` once the
+// accumulator has been read.  bf16 outputs (SwiGLU: BN / 2 columns, plain: BN)
+// are read and stored in rounds of 64 columns through the warp's staging
+// buffer.  (Reading the whole row into registers and handing the accumulator
+// back before storing measured no faster once the stores were coalesced.)
+// The fp32 epilogue (router logits) stores as it reads.
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr, int row,
+                                              uint32_t tempty, uint4* stage, int lane) {
+  // output row of the tile's row 0; split-K slices of problem 0 write separate planes
+  const long long orow_t = static_cast<long long>(T.a_row) + (T.p1 ? 0 : T.split * a.split_rows0);
+  if constexpr (EPI == EPI_F32) {
+    const bool valid = row < T.rows;
     float* out = static_cast<float*>(T.p1 ? a.out1 : a.out0);
     const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
-    float* dst = out + orow * ldo + static_cast<long long>(T.n_tile) * BN;
+    float* dst = out + (orow_t + row) * ldo + static_cast<long long>(T.n_tile) * BN;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
       uint32_t v[16];
@@ -144,6 +164,24 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
         for (int i = 0; i < 4; ++i) d4[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
       }
     }
+    tc_fence_before();
+    mbar_arrive(tempty);
+  } else {
+    constexpr int kOutCols = EPI == EPI_SWIGLU ? BN / 2 : BN;
+    constexpr int kRounds = kOutCols / 64;
+    const int wrow0 = row - lane;           // the warp's first row in the tile
+    const int valid_rows = T.rows - wrow0;  // rows of the warp that are stored
+    uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
+    const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
+    uint16_t* out_w = out + (orow_t + wrow0) * ldo + static_cast<long long>(T.n_tile) * kOutCols;
+#pragma unroll 1
+    for (int rd = 0; rd < kRounds; ++rd) {
+      uint32_t pk[32];
+      tmem_to_bf16_64<EPI>(taddr, 64 * rd, pk);
+      store_round(pk, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+    }
+    tc_fence_before();
+    mbar_arrive(tempty);
   }
 }
 
@@ -178,7 +216,9 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
   const uint32_t tq_base = bar0 + 8u * (2 * SA + 2 * SB + 5);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
+  // bf16 store staging, kStageWarpBytes per epilogue warp (16-byte aligned)
+  uint4* stage_all = reinterpret_cast<uint4*>(bar_area + kBarBytes);
+  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes + stage_bytes<EPI, PAIR>());
   // consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
   constexpr int kTileQConsumers = 2 + C::EPI_WARPS;
 
@@ -404,9 +444,13 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (PAIR ? half : acc) * BN;
       // the upper half of a half tile holds no rows (and no result)
-      if (half == 0 || T.rows > BM) epilogue_tile<EPI>(T, args, taddr, row);
-      tc_fence_before();
-      mbar_arrive(tempty_bar(acc));
+      if (half == 0 || T.rows > BM) {
+        epilogue_tile<EPI>(T, args, taddr, row, tempty_bar(acc),  // arrives on tempty itself
+                           stage_all + (warp - 2) * (kStageWarpBytes / 16), lane);
+      } else {
+        tc_fence_before();
+        mbar_arrive(tempty_bar(acc));
+      }
     }
   }
 
