@@ -49,8 +49,12 @@ constexpr uint32_t kTmemCols = 2 * BN;          // two partial buffers
 constexpr uint32_t kIdescF8 = (1u << 4) | (static_cast<uint32_t>(BN >> 3) << 17) | (static_cast<uint32_t>(BM >> 4) << 24);
 
 constexpr int kBarBytes = 384;
-// rings first (1024-byte aligned, declared and checked), then barriers, schedule, amax exchange
-constexpr size_t kSmemBytes = SA * A_BYTES + SB * B_BYTES + kBarBytes + sizeof(Sched) + 2 * 4 * BM * sizeof(float);
+// outputs are stored through 2 KB of shared memory per epilogue warp (32 rows x 4 chunks of 16 bytes)
+constexpr int kStageWarpBytes = 32 * 4 * 16;
+// rings first (1024-byte aligned, declared and checked), then barriers, store
+// staging, schedule, amax exchange
+constexpr size_t kSmemBytes = SA * A_BYTES + SB * B_BYTES + kBarBytes + kEpiWarps * kStageWarpBytes + sizeof(Sched) +
+                              2 * 4 * BM * sizeof(float);
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(8 * (2 * SA + 2 * SB + 7) + kTileQBytes + 12 <= kBarBytes, "barrier area");
 // consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
@@ -88,6 +92,29 @@ __device__ __forceinline__ void promote32(float* acc, uint32_t taddr, float s) {
   }
 }
 
+// One round of a warp's coalesced stores: lane l holds 4 chunks of 16 bytes
+// (w, 16 words) of its row l.  Every lane writes them to the warp's 2 KB
+// staging buffer (chunk j of row r at slot j ^ ((r / 2) % 4), so neither side
+// of the exchange has bank conflicts), then lanes 4u .. 4u+3 store the 4
+// chunks of rows u, u + 8, ...: each store instruction writes eight rows x 64
+// contiguous bytes instead of 32 rows x 16 bytes.  Rows from ``valid_rows`` on
+// are not stored.  out: the warp's first row at the round's first byte.
+__device__ __forceinline__ void store_round4(const uint32_t* w, uint4* stage, int lane, uint8_t* out,
+                                             long long ldo_bytes, int valid_rows) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    stage[lane * 4 + (j ^ ((lane >> 1) & 3))] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+  __syncwarp();
+  const int ru = lane >> 2, cu = lane & 3;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int r = ru + 8 * k;
+    const uint4 v = stage[r * 4 + (cu ^ ((r >> 1) & 3))];
+    if (r < valid_rows) *reinterpret_cast<uint4*>(out + r * ldo_bytes + cu * 16) = v;
+  }
+  __syncwarp();
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     grouped_gemm_fp8_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
@@ -117,7 +144,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 7) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* layer_slot = reinterpret_cast<int*>(tmem_slot + 2);  // layer id, shared with the epilogue
-  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
+  uint4* stage_all = reinterpret_cast<uint4*>(bar_area + kBarBytes);  // 16-byte aligned
+  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes + kEpiWarps * kStageWarpBytes);
   float* amax_x = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sch) + sizeof(Sched));  // [2][4][BM]
 
   const int warp = threadIdx.x >> 5;
@@ -370,6 +398,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
       const bool valid = r < T.rows;
+      uint4* stage = stage_all + (warp - 2) * (kStageWarpBytes / 16);
+      const int valid_rows = T.rows - q * 32;  // rows of this warp (rows q*32 .. q*32+31) that are stored
+      const long long wrow0 = static_cast<long long>(T.a_row) + q * 32;
       if constexpr (EPI == EPI_SWIGLU) {
         // h = silu(gate) * up for 32 channels, then e4m3 with one scale per
         // row per 128 channels (this tile's 128 h columns): the four column
@@ -394,40 +425,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int u = 0; u < kColGroups; ++u) amax = fmaxf(amax, xs[u * BM + r]);
         const float scale = amax > 0.f ? amax / 448.0f : 1.0f;
         const float inv = 1.0f / scale;  // one division; the quotients below are products
-        if (valid) {
-          uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
-          const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
-          uint8_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * (BN / 2) + cq * kH;
+        // kH = 64 e4m3 values: 4 chunks of 16 bytes, one staged round
+        static_assert(kH == 64, "one store round of e4m3 h per thread");
+        uint32_t w[16];
 #pragma unroll
-          for (int j = 0; j < kH; j += 16) {
-            uint32_t w4[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const __nv_fp8x2_storage_t lo = __nv_cvt_float2_to_fp8x2(
-                  make_float2(acc[j + 4 * u] * inv, acc[j + 4 * u + 1] * inv), __NV_SATFINITE, __NV_E4M3);
-              const __nv_fp8x2_storage_t hi = __nv_cvt_float2_to_fp8x2(
-                  make_float2(acc[j + 4 * u + 2] * inv, acc[j + 4 * u + 3] * inv), __NV_SATFINITE, __NV_E4M3);
-              w4[u] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
-            }
-            *reinterpret_cast<uint4*>(dst + j) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-          }
-          if (cq == 0) {
-            float* os = T.p1 ? fa.out_scale1 : fa.out_scale0;
-            const int osld = T.p1 ? fa.o_sld1 : fa.o_sld0;
-            os[row * osld + T.n_tile] = scale;
-          }
+        for (int j = 0; j < kH; j += 4) {
+          const __nv_fp8x2_storage_t lo = __nv_cvt_float2_to_fp8x2(make_float2(acc[j] * inv, acc[j + 1] * inv),
+                                                                    __NV_SATFINITE, __NV_E4M3);
+          const __nv_fp8x2_storage_t hi = __nv_cvt_float2_to_fp8x2(make_float2(acc[j + 2] * inv, acc[j + 3] * inv),
+                                                                    __NV_SATFINITE, __NV_E4M3);
+          w[j / 4] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+        }
+        uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
+        const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
+        store_round4(w, stage, lane, out + wrow0 * ldo + static_cast<long long>(T.n_tile) * (BN / 2) + cq * kH, ldo,
+                     valid_rows);
+        if (valid && cq == 0) {
+          float* os = T.p1 ? fa.out_scale1 : fa.out_scale0;
+          const int osld = T.p1 ? fa.o_sld1 : fa.o_sld0;
+          os[row * osld + T.n_tile] = scale;
         }
       } else {
-        if (valid) {
-          uint16_t* out = static_cast<uint16_t*>(T.p1 ? args.out1 : args.out0);
-          const long long ldo = T.p1 ? args.ldo1 : args.ldo0;
-          uint16_t* dst = out + row * ldo + static_cast<long long>(T.n_tile) * BN + cq * kCols;
+        // kCols = 128 bf16 values: 16 chunks, four staged rounds of 64 bytes
+        uint8_t* out = static_cast<uint8_t*>(T.p1 ? args.out1 : args.out0);
+        const long long ldo_b = 2 * (T.p1 ? args.ldo1 : args.ldo0);
+        uint8_t* out_w = out + wrow0 * ldo_b + 2 * (static_cast<long long>(T.n_tile) * BN + cq * kCols);
 #pragma unroll
-          for (int j = 0; j < kCols; j += 8) {
-            *reinterpret_cast<uint4*>(dst + j) =
-                make_uint4(pack_bf16x2(acc[j], acc[j + 1]), pack_bf16x2(acc[j + 2], acc[j + 3]),
-                           pack_bf16x2(acc[j + 4], acc[j + 5]), pack_bf16x2(acc[j + 6], acc[j + 7]));
-          }
+        for (int rd = 0; rd < kCols / 32; ++rd) {
+          uint32_t w[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(acc[32 * rd + 2 * i], acc[32 * rd + 2 * i + 1]);
+          store_round4(w, stage, lane, out_w + 64 * rd, ldo_b, valid_rows);
         }
       }
     }
