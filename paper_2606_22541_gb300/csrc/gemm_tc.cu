@@ -7,19 +7,23 @@
 // list is derived on the device from those offsets, so the host never reads
 // the per-expert counts back (the bubble-free principle of Section 3.4.2).
 //
-// Design (one CTA per SM, persistent, warp-specialised, 224 threads):
-//   warps 0,6: TMA producers.  Weight boxes B [256 rows, 64 K] (warp 0) and
-//              activation boxes A [128 rows, 64 K] (the last warp) into separate
-//              shared-memory rings (depths per launch kind in
-//              gemm_config.h), 128-byte swizzle.  The weights are stored
-//              tile-contiguous (one 32 KB read per box).
-//   warp 1   : TMEM allocator and MMA issuer (one thread): 4 x
-//              tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) per stage,
-//              fp32 accumulator in TMEM, two accumulators (2 x 256 columns) so
-//              the epilogue of one tile overlaps the main loop of the next.
-//   warps 2-5: epilogue.  tcgen05.ld 32x32b (warp w reads TMEM lanes
-//              32*(w%4) ...), fused SwiGLU (gate and up columns of a tile are
-//              the two 128-column halves), bf16 or fp32 store.
+// Design (one CTA per SM, persistent, warp-specialised; 224 threads, 352 with
+// paired m-tiles):
+//   warp 0   : weight producer.  B boxes [256 rows, 64 K] into its ring; the
+//              weights are stored tile-contiguous (one 32 KB read per box).
+//   last warp: activation producer.  A boxes [128 rows, 64 K] (two per stage
+//              for a paired tile) into its ring.  Ring depths per launch kind
+//              in gemm_config.h; 128-byte swizzle.
+//   warp 1   : TMEM allocator and MMA issuer (one thread): per stage 4 x
+//              tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16), twice
+//              for a paired tile; fp32 accumulators in TMEM (2 x 256 columns:
+//              ping-pong accumulators for single m-tiles, the two halves of a
+//              paired tile).
+//   epilogue : warps 2-5 (2-9 paired).  tcgen05.ld 32x32b (warp w reads TMEM
+//              lanes 32*(w%4) ...), fused SwiGLU (gate and up columns of a
+//              tile are the two 128-column halves), bf16 stores staged through
+//              shared memory so each store writes whole 128-byte row pieces
+//              (fp32 router logits are stored directly).
 // Weights: the B descriptors come from the layer table (one entry per layer,
 // in global memory) at the layer id the kernel loads when it starts, so one
 // launch sequence serves any layer (the MoE Super Kernel of Section 3.4.2).
