@@ -1,4 +1,5 @@
-// Routing kernels: router logits on CUDA cores (small expert counts), top-k
+// Routing kernels: router logits for expert counts below 256 (mma.sync, or
+// CUDA cores for shapes it does not cover), top-k
 // gating with a fixed tie-break, per-chunk expert histograms and their
 // deterministic prefix scan into per-expert counts and offsets.
 //
@@ -79,6 +80,82 @@ __global__ void __launch_bounds__(256) router_small_kernel(const uint4* __restri
     for (int i = 0; i < kRouterEB; ++i)
       if (lane == i) mine = acc[i];
     if (lane < kRouterEB && e0 + lane < E) logits[static_cast<long long>(t) * E + e0 + lane] = mine;
+  }
+}
+
+// Router logits on the tensor core for 8, 16, 32 or 64 experts (mma.sync
+// m16n8k16, bf16 in, fp32 accumulate; the partials of 64 experts fill 32 KB
+// of shared memory, the static limit is 48 KB): the contraction
+// has only E columns, too narrow for a 128 x 256 tcgen05 tile.  A CTA takes
+// 16 tokens; its 8 warps split K, warp w taking the 32-wide K chunks w, w + 8,
+// ...; the partial sums are added in warp order in shared memory.
+//
+// Fragments are loaded straight from global memory with a permutation of K
+// that A and B share (the dot product does not depend on the order of K):
+// thread (g = lane / 4, q = lane % 4) loads 16 bytes (8 bf16) of token rows g
+// and g + 8 and of expert rows 8 j + g at K offset 8 q of the chunk, and feeds
+// bf16 pairs 0, 1 to the chunk's first MMA and pairs 2, 3 to the second: in
+// the first MMA, K slots 2q, 2q+1 are K offsets 8q, 8q+1 and slots 2q+8,
+// 2q+9 are 8q+2, 8q+3, for A and for B alike.
+constexpr int kRmmaWarps = 8;
+constexpr int kRmmaTokens = 16;
+
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+template <int NB>  // E = 8 NB experts
+__global__ void __launch_bounds__(kRmmaWarps * 32) router_mma_kernel(const uint4* __restrict__ x, LayerRef lref,
+                                                                     uint32_t* status, int n, int V,
+                                                                     float* __restrict__ logits) {
+  constexpr int E = 8 * NB;
+  __shared__ float part[kRmmaWarps][kRmmaTokens][E];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, q = lane & 3;
+  const int t0 = blockIdx.x * kRmmaTokens;
+  const uint4* __restrict__ wr = static_cast<const uint4*>(
+      lref.table[load_layer(lref.layer, lref.n_layers, status, blockIdx.x == 0 && threadIdx.x == 0)].router_w);
+  // token rows g and g + 8 (rows past n read as zero and are not stored)
+  const bool in0 = t0 + g < n, in1 = t0 + g + 8 < n;
+  const uint4* x0 = x + static_cast<long long>(in0 ? t0 + g : 0) * V;
+  const uint4* x1 = x + static_cast<long long>(in1 ? t0 + g + 8 : 0) * V;
+  float c[NB][4];
+#pragma unroll
+  for (int j = 0; j < NB; ++j) c[j][0] = c[j][1] = c[j][2] = c[j][3] = 0.f;
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  // chunk ch covers 16-byte vectors 4 ch .. 4 ch + 3 of every row
+  for (int ch = warp; ch < V / 4; ch += kRmmaWarps) {
+    const int v = 4 * ch + q;
+    const uint4 a = in0 ? __ldg(x0 + v) : zero;
+    const uint4 b = in1 ? __ldg(x1 + v) : zero;
+#pragma unroll
+    for (int j = 0; j < NB; ++j) {
+      const uint4 w = __ldg(wr + static_cast<long long>(8 * j + g) * V + v);
+      mma_bf16_16816(c[j], a.x, b.x, a.y, b.y, w.x, w.y);
+      mma_bf16_16816(c[j], a.z, b.z, a.w, b.w, w.z, w.w);
+    }
+  }
+  // c[j]: (token g, experts 8j + 2q, 8j + 2q + 1) and (token g + 8, the same experts)
+#pragma unroll
+  for (int j = 0; j < NB; ++j) {
+    part[warp][g][8 * j + 2 * q] = c[j][0];
+    part[warp][g][8 * j + 2 * q + 1] = c[j][1];
+    part[warp][g + 8][8 * j + 2 * q] = c[j][2];
+    part[warp][g + 8][8 * j + 2 * q + 1] = c[j][3];
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < kRmmaTokens * E; i += blockDim.x) {
+    const int tl = i / E, e = i % E;
+    if (t0 + tl >= n) continue;
+    float sum = part[0][tl][e];
+#pragma unroll
+    for (int w = 1; w < kRmmaWarps; ++w) sum += part[w][tl][e];
+    logits[static_cast<long long>(t0 + tl) * E + e] = sum;
   }
 }
 
@@ -615,6 +692,20 @@ __global__ void reduce_splits_kernel(const float* __restrict__ parts, int splits
 cudaError_t launch_router_small(const void* x, const LayerRef& lref, int n, int H, int E, float* logits,
                                 uint32_t* status, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
+  if (H % 32 == 0) {
+    const int grid = ceil_div(n, kRmmaTokens);
+    const uint4* xv = static_cast<const uint4*>(x);
+#define ASAP_ROUTER_MMA(NBV)                                                                                  \
+  if (E == 8 * NBV) {                                                                                         \
+    router_mma_kernel<NBV><<<grid, kRmmaWarps * 32, 0, s>>>(xv, lref, status, n, H / 8, logits);              \
+    return cudaGetLastError();                                                                                \
+  }
+    ASAP_ROUTER_MMA(1)
+    ASAP_ROUTER_MMA(2)
+    ASAP_ROUTER_MMA(4)
+    ASAP_ROUTER_MMA(8)
+#undef ASAP_ROUTER_MMA
+  }
   router_small_kernel<<<ceil_div(n, 8), 256, 0, s>>>(static_cast<const uint4*>(x), lref, status, n, H / 8, E,
                                                        logits);
   return cudaGetLastError();
