@@ -65,6 +65,7 @@ struct Gemm {
 };
 constexpr int BM = kGemmBM, BN = kGemmBN, BK = kGemmBK;
 
+
 constexpr int B_BYTES = BN * BK * 2;
 constexpr uint32_t kTmemCols = 2 * BN;
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
@@ -114,6 +115,7 @@ __device__ __forceinline__ void store_round(const uint32_t* pk, uint4* stage, in
 // TMEM -> packed bf16 for 64 output columns starting at output column c0:
 // SwiGLU tiles read gate columns c0 .. c0 + 63 and the matching up columns
 // BN / 2 further and form silu(g) u; plain tiles read columns c0 .. c0 + 63.
+// (16 columns per TMEM wait: 32 or 64 per wait measured the same.)
 template <int EPI>
 __device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t* pk) {
 #pragma unroll
@@ -143,11 +145,15 @@ __device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t
 // Epilogue of one tile for the thread owning TMEM lane ``row`` (taddr: that
 // lane, the accumulator's first column); it arrives on ``tempty`` once the
 // accumulator has been read.  bf16 outputs (SwiGLU: BN / 2 columns, plain: BN)
-// are read and stored in rounds of 64 columns through the warp's staging
-// buffer.  (Reading the whole row into registers and handing the accumulator
-// back before storing measured no faster once the stores were coalesced.)
-// The fp32 epilogue (router logits) stores as it reads.
-template <int EPI>
+// are stored in rounds of 64 columns through the warp's staging buffer.
+// EARLY (down GEMM with paired tiles, whose accumulator is all of TMEM): the
+// whole row is read into registers (packed bf16) and the accumulator handed
+// back before any store, so the stores overlap the next tile's main loop
+// (measured 1-2 % faster; for the gate/up GEMM it measured no faster and
+// spilled).  Otherwise rows are read and stored round by round (single
+// m-tiles' two accumulators already overlap the epilogue with the next main
+// loop).  The fp32 epilogue (router logits) stores as it reads.
+template <int EPI, bool EARLY>
 __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr, int row,
                                               uint32_t tempty, uint4* stage, int lane) {
   // output row of the tile's row 0; split-K slices of problem 0 write separate planes
@@ -178,14 +184,24 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
     uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
     const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
     uint16_t* out_w = out + (orow_t + wrow0) * ldo + static_cast<long long>(T.n_tile) * kOutCols;
+    if constexpr (EARLY) {
+      uint32_t pk[kRounds * 32];
+#pragma unroll
+      for (int rd = 0; rd < kRounds; ++rd) tmem_to_bf16_64<EPI>(taddr, 64 * rd, pk + 32 * rd);
+      tc_fence_before();
+      mbar_arrive(tempty);
+#pragma unroll
+      for (int rd = 0; rd < kRounds; ++rd) store_round(pk + 32 * rd, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+    } else {
 #pragma unroll 1
-    for (int rd = 0; rd < kRounds; ++rd) {
-      uint32_t pk[32];
-      tmem_to_bf16_64<EPI>(taddr, 64 * rd, pk);
-      store_round(pk, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+      for (int rd = 0; rd < kRounds; ++rd) {
+        uint32_t pk[32];
+        tmem_to_bf16_64<EPI>(taddr, 64 * rd, pk);
+        store_round(pk, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+      }
+      tc_fence_before();
+      mbar_arrive(tempty);
     }
-    tc_fence_before();
-    mbar_arrive(tempty);
   }
 }
 
@@ -449,8 +465,9 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (PAIR ? half : acc) * BN;
       // the upper half of a half tile holds no rows (and no result)
       if (half == 0 || T.rows > BM) {
-        epilogue_tile<EPI>(T, args, taddr, row, tempty_bar(acc),  // arrives on tempty itself
-                           stage_all + (warp - 2) * (kStageWarpBytes / 16), lane);
+        // arrives on tempty itself
+        epilogue_tile<EPI, PAIR && EPI == EPI_BF16>(T, args, taddr, row, tempty_bar(acc),
+                                                    stage_all + (warp - 2) * (kStageWarpBytes / 16), lane);
       } else {
         tc_fence_before();
         mbar_arrive(tempty_bar(acc));
