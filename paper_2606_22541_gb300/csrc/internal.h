@@ -69,10 +69,9 @@ struct GemmArgs {
 constexpr int kTileCounters = 2;  // per call: gate/up GEMM, down GEMM
 constexpr int kGemmBM = 128;
 constexpr int kGemmBN = 256;
-#ifndef ASAP_GEMM_BK
-#define ASAP_GEMM_BK 64
-#endif
-constexpr int kGemmBK = ASAP_GEMM_BK;  // 64 (128-byte swizzle) or 32 (64-byte swizzle)
+// K per stage: 64 bf16, one 128-byte swizzled row per box row (the weight
+// packing of launch_retile and the tile-contiguous addressing assume it)
+constexpr int kGemmBK = 64;
 
 cudaError_t gemm_set_attributes();
 // maps: A0, A1 (A1 may repeat A0 when m1 == 0), encoded for boxes of 128 rows,
