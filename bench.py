@@ -47,7 +47,7 @@ def parse_args():
     ap.add_argument("--workload", default="dsv3_bf16")
     ap.add_argument("--kernel-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample-tokens", type=int, default=6)
+    ap.add_argument("--cpu-sample-tokens", type=int, default=12)
     ap.add_argument("--microbatches", default=None,
                     help="comma-separated micro-batch sizes overriding the workload's")
     ap.add_argument("--measure-fp8-peak", action="store_true",
