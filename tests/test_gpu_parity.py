@@ -99,6 +99,37 @@ def test_router_logits_within_bound(cfg):
     assert_clean(c)
 
 
+# router widths: E = 8, 16, 32, 64 run the mma.sync router (16 tokens per CTA,
+# K split over 8 warps), E = 24 and 128 the CUDA-core one; ragged token counts
+# cover the CTA's 16-token tail
+ROUTER_E = [inputs.small_variant(MIXTRAL, name=f"router_e{E}", hidden=768, n_experts=E, top_k=2, inter=128,
+                                 microbatches=[1000]) for E in (8, 16, 24, 32, 64, 128)]
+
+
+@pytest.mark.parametrize("cfg", ROUTER_E, ids=lambda c: c.name)
+def test_router_logits_widths_within_bound(cfg):
+    c = Case.get(cfg)
+    for n in (1, 15, 17, 100, 1000):
+        x = c.tokens(0, n)
+        logits = torch.full((n, cfg.n_experts), float("nan"), dtype=torch.float32, device=DEV)
+        api.asap_moe_router_logits(c.h, x, logits, c.ws(n))
+        torch.cuda.synchronize()
+        xf = bf16_to_f64(x)
+        L = oracle.router_logits(xf, c.wf["router_w"])
+        eps = oracle.logit_error_bound(xf, c.wf["router_w"])
+        err = np.abs(logits.cpu().numpy().astype(np.float64) - L)
+        assert (err <= eps).all(), f"n={n}: max err/bound {float(np.nanmax(err / eps)):.3f}"
+    assert_clean(c)
+
+
+def test_set_tiling_rejects_unknown_mode():
+    from paper_2606_22541_gb300._native import AsapError
+    c = Case.get(TINY)
+    with pytest.raises(AsapError):
+        api.asap_moe_set_tiling(c.h, 3)
+    api.asap_moe_set_tiling(c.h, api.TILING_AUTO)
+
+
 @pytest.mark.parametrize("cfg", SMALL + ODD, ids=lambda c: c.name)
 def test_route_matches_oracle(cfg):
     c = Case.get(cfg)
