@@ -328,6 +328,39 @@ def test_expert_ffn_matches_oracle(cfg):
     assert_clean(c)
 
 
+@pytest.mark.parametrize("hot", ["first", "middle", "last"])
+def test_expert_ffn_all_rows_in_one_expert(hot):
+    """Every routed row in one expert, every other segment empty, with single
+    and with paired m-tiles: the same bits both ways and the oracle's values."""
+    cfg = DS_SMALL
+    c = Case.get(cfg)
+    n, k, E, H = max(cfg.microbatches), cfg.top_k, cfg.n_experts, cfg.hidden
+    e_hot = {"first": 0, "middle": E // 2, "last": E - 1}[hot]
+    counts = np.zeros(E, np.int64)
+    counts[e_hot] = n * k
+    offsets_np = oracle.expert_offsets(counts)
+    x = c.tokens(0, n)
+    x_perm = inputs.randn_bf16((n * k, H), 1.0, 91, DEV)
+    offsets = torch.tensor(offsets_np, dtype=torch.int32, device=DEV)
+    outs = []
+    try:
+        for mode in (api.TILING_SINGLE, api.TILING_PAIRED):
+            api.asap_moe_set_tiling(c.h, mode)
+            y_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+            y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+            api.asap_moe_expert_ffn(c.h, x_perm, offsets, x, y_perm, y_sh, c.ws(n))
+            outs.append((y_perm, y_sh))
+    finally:
+        api.asap_moe_set_tiling(c.h, api.TILING_AUTO)
+    torch.cuda.synchronize()
+    for a, b in zip(outs[0], outs[1]):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    ref = oracle.expert_ffn(bf16_to_f64(x_perm), offsets_np, c.wf["w_gate"], c.wf["w_up"], c.wf["w_down"])
+    compare_rows(bf16_to_f64(outs[1][0]), ref)
+    compare_rows(bf16_to_f64(outs[1][1]), oracle.swiglu(bf16_to_f64(x), *c.shared))
+    assert_clean(c)
+
+
 # ---------------------------------------------------------------- whole layer
 
 def oracle_layer(c, x):
