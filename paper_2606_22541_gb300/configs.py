@@ -99,6 +99,14 @@ DSV3_FP8_E32 = LayerConfig("dsv3_fp8_e32_profile", hidden=7168, n_experts=32, to
                            shared_inter=2048, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
                            route_scale=2.5, dtype="fp8_e4m3_block128", microbatches=[512], seed=1004)
 
+# Profiling case of the grouped GEMMs where they are bound by the tensor core:
+# the DeepSeek-V3 expert shape with 32 experts and 4096 tokens, i.e. ~1024 rows
+# per expert (the regime of several micro-batches aggregated into one GEMM);
+# 2.8 GB of weights and ~0.9 GB of activations on the device.
+DSV3_E32_COMPUTE = LayerConfig("dsv3_e32_compute_profile", hidden=7168, n_experts=32, top_k=8, inter=2048,
+                               n_shared=1, shared_inter=2048, gating="sigmoid_grouped", n_groups=8,
+                               topk_groups=4, route_scale=2.5, microbatches=[4096], seed=1005)
+
 # Profiling case of route, dispatch and combine: the DeepSeek-V3 routing shape
 # (H = 7168, 256 experts, top-8, grouped sigmoid, 4096 tokens), whose bytes do
 # not depend on the expert FFN width, with a narrow FFN (I = 256) so the device
@@ -107,4 +115,5 @@ DSV3_ROUTING = LayerConfig("dsv3_routing_profile", hidden=7168, n_experts=256, t
                            shared_inter=256, gating="sigmoid_grouped", n_groups=8, topk_groups=4,
                            route_scale=2.5, microbatches=[4096], seed=1002)
 
-CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32, DSV3_FP8_E32, DSV3_ROUTING)}
+CONFIGS = {c.name: c for c in (TINY, MIXTRAL, DSV3, STRESS, DSV3_FP8, DSV3_E32, DSV3_E32_COMPUTE, DSV3_FP8_E32,
+                               DSV3_ROUTING)}
