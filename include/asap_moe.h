@@ -159,7 +159,7 @@ int asap_moe_create(const asap_moe_config* cfg, const asap_moe_weights* weights,
                     asap_moe_t* out);
 
 /* One handle over n_layers MoE layers of the same shape: the layer-oblivious
- * MoE Super Kernel of Section 3.4.2 (Section 4.1 describes it as a layer-ID
+ * MoE Super Kernel of Section 3.4.2 (Section 4.3 describes it as a layer-ID
  * input plus a pre-computed list of weight addresses).
  *  - weights points to n_layers structs; layer l is copied and packed as
  *    asap_moe_create does, and occupies that much HBM (all layers stay

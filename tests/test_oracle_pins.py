@@ -462,7 +462,9 @@ def test_dequant_blocks_layout():
     assert w[0, 0] == 0 and w[127, 383] == 2 and w[128, 0] == 3 and w[255, 383] == 5
 
 
-def test_fp8_swiglu_is_close_to_exact_and_exact_on_representable_input():
+def test_fp8_swiglu_within_e4m3_error_of_unquantised():
+    """Two e4m3 roundings (x, then h) of about 2^-4 relative each keep the
+    result within a few per cent of the unquantised SwiGLU."""
     rng = np.random.default_rng(42)
     H, I = 256, 128
     x = rng.normal(0, 1, (3, H))
@@ -473,6 +475,190 @@ def test_fp8_swiglu_is_close_to_exact_and_exact_on_representable_input():
     assert np.linalg.norm(a - b) / np.linalg.norm(b) < 0.08
 
 
+# Pins of the FP8 emulation (activation quantisation per token per 128
+# channels, s = amax / 448, round to nearest even e4m3, for x before the
+# gate/up product and for h before the down product).  Each pin returns
+# True when it holds, so the planted-mistake test below can show that a
+# missing h quantisation, a 64-channel block or a scale taken over the wrong
+# axis fails at least one of them.
+
+def _representable_block(rng, c, width=128):
+    """One block of ``width`` values that are e4m3 values times 2^c; the
+    first half holds the block maximum 448 * 2^c, the second half peaks at
+    320 * 2^c, so only a 128-wide block has a power-of-two scale."""
+    e4 = formats.e4m3_bits_to_f64(np.arange(0, 0x7F, dtype=np.uint8))   # finite, >= 0
+    e4 = e4[e4 <= 320.0]
+    v = rng.choice(e4, width) * rng.choice([-1.0, 1.0], width)
+    v[rng.integers(0, width // 2)] = 448.0
+    v[width // 2 + rng.integers(0, width // 2)] = -320.0
+    return np.ldexp(v, c)
+
+
+def _fp8_exact_weights(x0, h_target):
+    """Gate/up weights that read only channel 0 of x (x0 = x[0], a power of
+    two): g = 64 in every channel, where silu(64) == 64 in float64, and
+    u = h_target / 64, so silu(g) * u == h_target exactly."""
+    I = len(h_target)
+    H = 256
+    wg = np.zeros((I, H))
+    wu = np.zeros((I, H))
+    wg[:, 0] = 64.0 / x0
+    wu[:, 0] = h_target / 64.0 / x0
+    return wg, wu
+
+
+def _pin_fp8_exact_on_representable_input():
+    """x and h whose 128-channel blocks are e4m3 values times power-of-two
+    scales equal to amax / 448 quantise without error, so the emulation
+    must return the unquantised SwiGLU bit for bit."""
+    rng = np.random.default_rng(61)
+    x = np.concatenate([_representable_block(rng, -3), _representable_block(rng, 2)])
+    x[0] = 256.0 * 2.0 ** -3            # channel 0 is a power of two below the block max
+    h = np.concatenate([_representable_block(rng, -5), _representable_block(rng, 1)])
+    wg, wu = _fp8_exact_weights(x[0], h)
+    wd = rng.normal(0, 0.1, (256, 256))
+    a = layer.swiglu_fp8(x[None], wg, wu, wd)
+    b = layer.swiglu(x[None], wg, wu, wd)
+    return np.array_equal(a, b)
+
+
+def _pin_fp8_hand_worked_rounding():
+    """One token, hand-worked.  x is representable (quantises exactly), g = 64
+    everywhere and the down projection is the identity, so the output is
+    the quantised h itself.  h has two 128-channel blocks with maxima 448 * 2
+    and 448 / 4 (scales 2 and 1/4); the other values, divided by the scale,
+    sit on rounding ties or off the grid:
+        17 -> 16, 19 -> 20 (ties to the even neighbour, binade [16, 32) step 2),
+        1.5 * 2^-9 -> 2^-8 (subnormal tie), 0.3 -> 0.3125 (nearest, step 2^-5),
+        -100 -> -96 (step 8: 96 and 104, 100 is a tie -> 96, even),
+    and the rest are zero."""
+    x = np.zeros(256)
+    x[0] = 1.0
+    x[1] = 448.0
+    x[128] = 448.0 * 2.0 ** -6
+    s0, s1 = 2.0, 0.25
+    scaled = {0: 448.0, 1: 17.0, 2: 19.0, 3: 1.5 * 2.0 ** -9, 4: 0.3, 5: -100.0,
+              64: -19.0, 65: 17.0, 100: -0.3}
+    expect_q = {0: 448.0, 1: 16.0, 2: 20.0, 3: 2.0 ** -8, 4: 0.3125, 5: -96.0,
+                64: -20.0, 65: 16.0, 100: -0.3125}
+    h = np.zeros(256)
+    want = np.zeros(256)
+    for ch, v in scaled.items():
+        h[ch] = v * s0
+        want[ch] = expect_q[ch] * s0
+        h[128 + ch] = v * s1
+        want[128 + ch] = expect_q[ch] * s1
+    wg, wu = _fp8_exact_weights(x[0], h)
+    y = layer.moe_layer_tokens_fp8(x[None], np.array([[0]]), np.array([[1.0]]),
+                                   wg[None], wu[None], np.eye(256)[None])
+    return np.array_equal(y[0], want)
+
+
+_E4M3_TABLE = torch.arange(0, 0x7F, dtype=torch.uint8).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+
+
+def _nearest_e4m3(v):
+    """Round to e4m3 by search over the table of finite non-negative codes
+    (decoded by torch): nearest value, a tie going to the even code; magnitudes
+    above 448 saturate."""
+    a = np.minimum(np.abs(v), 448.0)
+    i = np.clip(np.searchsorted(_E4M3_TABLE, a), 1, len(_E4M3_TABLE) - 1)
+    lo, hi = _E4M3_TABLE[i - 1], _E4M3_TABLE[i]
+    pick_hi = (hi - a < a - lo) | ((hi - a == a - lo) & (i % 2 == 0))
+    return np.copysign(np.where(pick_hi, hi, lo), v)
+
+
+def _quantize_blocks_by_search(v):
+    n, c = v.shape
+    blocks = v.reshape(n, c // 128, 128)
+    amax = np.abs(blocks).max(axis=2, keepdims=True)
+    s = np.where(amax > 0, amax / 448.0, 1.0)
+    return (_nearest_e4m3(blocks / s) * s).reshape(n, c)
+
+
+def _pin_fp8_equals_search_composition():
+    """Random inputs: the emulation equals quantise (by table search) ->
+    product -> quantise -> product, composed here without the oracle."""
+    rng = np.random.default_rng(62)
+    n, H, I = 5, 384, 256
+    x = rng.normal(0, 1, (n, H))
+    x[1, 130:140] *= 40.0                      # one block with a large maximum
+    wg, wu = rng.normal(0, 1 / 19.6, (2, I, H))
+    wd = rng.normal(0, 1 / 16, (H, I))
+    xd = _quantize_blocks_by_search(x)
+    g = xd @ wg.T
+    hd = _quantize_blocks_by_search(g / (1.0 + np.exp(-g)) * (xd @ wu.T))
+    ref = hd @ wd.T
+    got = layer.swiglu_fp8(x, wg, wu, wd)
+    return np.allclose(got, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+
+
+def test_fp8_swiglu_exact_on_representable_input():
+    assert _pin_fp8_exact_on_representable_input()
+
+
+def test_fp8_hand_worked_rounding_of_h():
+    assert _pin_fp8_hand_worked_rounding()
+
+
+def test_fp8_swiglu_equals_composition_by_table_search():
+    assert _pin_fp8_equals_search_composition()
+
+
+def test_fp8_layer_tokens_weights_and_shared_expert():
+    """moe_layer_tokens_fp8: two experts with equal weights and routing
+    weights summing to 1 give one expert's output; the shared expert adds
+    its own quantised SwiGLU."""
+    rng = np.random.default_rng(63)
+    n, H, I = 4, 256, 128
+    x = rng.normal(0, 1, (n, H))
+    wg, wu = rng.normal(0, 1 / 16, (2, 1, I, H))
+    wd = rng.normal(0, 1 / 11.3, (1, H, I))
+    two = lambda a: np.concatenate([a, a])
+    idx = np.tile([[0, 1]], (n, 1))
+    w = np.tile([[0.25, 0.75]], (n, 1))
+    one = layer.swiglu_fp8(x, wg[0], wu[0], wd[0])
+    y = layer.moe_layer_tokens_fp8(x, idx, w, two(wg), two(wu), two(wd))
+    assert np.allclose(y, one, rtol=1e-14, atol=1e-14 * np.abs(one).max())
+    sh = (rng.normal(0, 1 / 16, (I, H)), rng.normal(0, 1 / 16, (I, H)), rng.normal(0, 1 / 11.3, (H, I)))
+    ys = layer.moe_layer_tokens_fp8(x, idx, w, two(wg), two(wu), two(wd), shared=sh)
+    assert np.allclose(ys - y, layer.swiglu_fp8(x, *sh), rtol=1e-12, atol=1e-12 * np.abs(ys).max())
+
+
+def test_fp8_pins_catch_planted_mistakes(monkeypatch):
+    """Plant each plausible mistake in the oracle's FP8 emulation and check
+    that at least one FP8 pin fails."""
+    pins = (_pin_fp8_exact_on_representable_input, _pin_fp8_hand_worked_rounding,
+            _pin_fp8_equals_search_composition)
+    assert all(p() for p in pins)
+    real = layer.quantize_rows_e4m3
+
+    def skip_h(v, block=128):                 # the second call (h) is not quantised
+        skip_h.calls += 1
+        if skip_h.calls % 2 == 0:
+            v = np.asarray(v, np.float64)
+            return v.copy(), np.ones((v.shape[0], (v.shape[1] + block - 1) // block))
+        return real(v, block)
+    skip_h.calls = 0
+
+    # the mistakes below return dequantised values with unit scales, which
+    # the emulation multiplies back unchanged
+    def block64(v, block=128):                # 64-channel blocks
+        q, s = real(v, 64)
+        v = np.asarray(v, np.float64)
+        return q * np.repeat(s, 64, 1)[:, :v.shape[1]], np.ones((v.shape[0], (v.shape[1] + block - 1) // block))
+
+    def column_scale(v, block=128):           # amax over tokens instead of channels
+        v = np.asarray(v, np.float64)
+        amax = np.abs(v).max(axis=0, keepdims=True)
+        sc = np.where(amax > 0, amax / 448.0, 1.0)
+        q = formats.round_to_e4m3_sat(v / sc)
+        return q * sc, np.ones((v.shape[0], (v.shape[1] + block - 1) // block))
+
+    for mistake in (skip_h, block64, column_scale):
+        monkeypatch.setattr(layer, "quantize_rows_e4m3", mistake)
+        assert not all(p() for p in pins), mistake.__name__
+        monkeypatch.setattr(layer, "quantize_rows_e4m3", real)
 # ---------------------------------------------------------------- paper constants
 
 def test_table1_shapes_are_the_dsv3_configs():
