@@ -314,9 +314,10 @@ int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int
  * or would synchronise the device.  This call takes the same inputs and
  * outputs as asap_moe_route but keeps its scratch (router logits, per-chunk
  * histograms, chunk bases and a counter) in one static device array of the
- * library: 4096 tokens x 256 experts, 4 MiB + 256 KiB + 256 B, held by every
- * GPU that loads libasap_moe until the process exits.  It calls no cudaMalloc, cudaFree or
- * other allocating routine.
+ * library: 4096 tokens x 256 experts x up to 4 router K-slice planes,
+ * 16 MiB + 256 KiB + 256 B, held by every GPU that loads libasap_moe until
+ * the process exits.  It calls no cudaMalloc, cudaFree or other allocating
+ * routine.
  *  - n > 4096 (or n > max_tokens) returns ASAP_ERR_INVALID with a message.
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
@@ -327,8 +328,10 @@ int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int
  *  - The array keeps the last call's contents; every element a call reads is
  *    written earlier by the same call (the counter by a 4-byte memset on the
  *    stream, which allocates nothing).
- *  - For E = 256 with grouped sigmoid gating it runs the same single launch as
- *    asap_moe_route and returns the same bits.                             */
+ *  - It returns the same bits as asap_moe_route for every configuration:
+ *    for E = 256 with grouped sigmoid gating it runs the same single launch;
+ *    otherwise the same router kernels with the same K slices, the same gate
+ *    and the same scan.                                                    */
 int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int32_t* idx, float* w,
                            int32_t* counts, int32_t* offsets, void* stream);
 

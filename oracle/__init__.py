@@ -22,4 +22,4 @@ from .layer import (expert_counts, expert_offsets, permutation, dispatch, silu,
                     swiglu, expert_ffn, combine, moe_layer, moe_layer_tokens,
                     moe_layer_tokens_by_expert,
                     quantize_rows_e4m3, dequant_blocks, swiglu_fp8,
-                    moe_layer_tokens_fp8)
+                    moe_layer_tokens_fp8, moe_layer_tokens_fp8_by_expert)

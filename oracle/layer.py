@@ -228,3 +228,22 @@ def moe_layer_tokens_fp8(x_tok, idx, w, wg, wu, wd, shared=None, block=128):
         if shared is not None:
             out[t] += swiglu_fp8(x_tok[t:t + 1], *shared, block=block)[0]
     return out
+
+
+def moe_layer_tokens_fp8_by_expert(x_tok, idx, w, get_expert, shared=None, block=128):
+    """``moe_layer_tokens_fp8`` looping over experts instead of tokens, so a
+    large weight set is fetched (decoded) once per expert: get_expert(e)
+    returns the dequantised (Wg_e, Wu_e, Wd_e).  Same definition (the
+    activation quantisation is per row, so an expert's rows are quantised
+    together); the terms of a token are added in expert order, then the
+    shared expert."""
+    x_tok = np.asarray(x_tok, np.float64)
+    idx = np.asarray(idx, np.int64)
+    out = np.zeros_like(x_tok)
+    for e in np.unique(idx):
+        rows, slots = np.nonzero(idx == e)
+        wg, wu, wd = get_expert(int(e))
+        out[rows] += w[rows, slots][:, None] * swiglu_fp8(x_tok[rows], wg, wu, wd, block)
+    if shared is not None:
+        out += swiglu_fp8(x_tok, *shared, block=block)
+    return out

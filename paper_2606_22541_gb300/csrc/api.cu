@@ -1224,15 +1224,18 @@ ASAP_API int asap_moe_status(asap_moe_t h, uint32_t* word) {
 // a path where a cudaMalloc would implicitly synchronise the device or is not
 // permitted at all.  asap_moe_route_noalloc gives them the routing step with
 // its scratch (router logits, per-chunk histograms, chunk bases) in a
-// file-scope device array instead of a caller workspace.  The array is
-// kStaticRouteMaxTokens tokens x 256 experts and is held by every GPU that
-// loads this library until the process exits.
+// file-scope device array instead of a caller workspace.  The array holds
+// kStaticRouteMaxTokens tokens x 256 experts of up to kMaxRouterSplits logit
+// planes and is held by every GPU that loads this library until the process
+// exits.
 
 namespace {
 
 constexpr int kStaticRouteMaxTokens = 4096;
-constexpr size_t kStaticLogitsBytes =
-    static_cast<size_t>(kStaticRouteMaxTokens) * ASAP_MOE_MAX_EXPERTS * sizeof(float);   // 4 MiB
+// the router's K-slice planes: up to kMaxRouterSplits partial-logit planes of
+// [n, E] fp32, as asap_moe_route keeps them in its workspace
+constexpr size_t kStaticLogitsBytes = static_cast<size_t>(asap::kMaxRouterSplits) * kStaticRouteMaxTokens *
+                                      ASAP_MOE_MAX_EXPERTS * sizeof(float);  // 16 MiB
 constexpr size_t kStaticChunkBytes = static_cast<size_t>(kStaticRouteMaxTokens / asap::kChunkTokens) *
                                      ASAP_MOE_MAX_EXPERTS * sizeof(int32_t);                  // 128 KiB
 constexpr size_t kStaticRouteBytes = kStaticLogitsBytes + 2 * kStaticChunkBytes + 256;  // + the scan's ticket
@@ -1295,12 +1298,15 @@ ASAP_API int asap_moe_route_noalloc(asap_moe_t h, const void* x, int32_t n, int3
     return run_route_fused(h, x, n, idx, w, hist, 0, asap::ceil_div(n, asap::kChunkTokens), ticket, counts, offsets,
                            base, nullptr, h->layer_ids, st);
   }
-  // every scratch element read below is written earlier on the same stream
-  // (logits by the router, all E entries of each chunk's histogram and the
-  // scan's ticket by the gate kernel), so nothing has to be cleared between
-  // calls
-  if ((r = run_router_logits(h, x, n, logits, 1, h->layer_ids, st)) != ASAP_OK) return r;
-  CU_TRY(asap::launch_gate(logits, 1, n, gate_params(h, h->layer_ids, ticket), idx, w, hist, st), "gate launch");
+  // the router's K slices and their order of addition are those of
+  // asap_moe_route, so the bits are the same.  Every scratch element read
+  // below is written earlier on the same stream (the logit planes by the
+  // router, all E entries of each chunk's histogram and the scan's ticket by
+  // the gate kernel), so nothing has to be cleared between calls.
+  const int splits = router_splits(h, n);
+  if ((r = run_router_logits(h, x, n, logits, splits, h->layer_ids, st)) != ASAP_OK) return r;
+  CU_TRY(asap::launch_gate(logits, splits, n, gate_params(h, h->layer_ids, ticket), idx, w, hist, st),
+         "gate launch");
   CU_TRY(asap::launch_scan(hist, asap::ceil_div(n, asap::kChunkTokens), h->cfg.n_experts, counts, offsets, base,
                            ticket, st),
          "scan launch");

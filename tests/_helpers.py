@@ -57,3 +57,20 @@ def routing_check(L_ref, eps, cfg, idx_gpu, w_gpu, w_ref, idx_ref, bias=None):
     for t in np.nonzero(~d)[0]:
         assert oracle.token_feasible(L_ref[t], eps[t], cfg, idx_gpu[t], bias), f"token {t} infeasible"
     return decided
+
+
+def sample_tokens(idx_ref, decided, E, rng, count):
+    """Decided tokens to compare: the last token, the first and last token
+    of the hottest and of the coldest non-empty expert, then random ones."""
+    n = idx_ref.shape[0]
+    cnt = np.bincount(idx_ref.reshape(-1), minlength=E)
+    hot = int(cnt.argmax())
+    cold = int(np.where(cnt > 0, cnt, cnt.max() + 1).argmin())
+    must = [n - 1]
+    for e in (hot, cold):
+        toks = np.nonzero((idx_ref == e).any(axis=1))[0]
+        must += [int(toks[0]), int(toks[-1])]
+    must = sorted({t for t in must if decided[t]})
+    rest = np.setdiff1d(np.nonzero(decided)[0], must)
+    extra = rng.choice(rest, max(0, min(count - len(must), len(rest))), replace=False)
+    return np.unique(np.r_[must, extra]).astype(np.int64)

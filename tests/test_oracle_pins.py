@@ -625,6 +625,20 @@ def test_fp8_layer_tokens_weights_and_shared_expert():
     assert np.allclose(ys - y, layer.swiglu_fp8(x, *sh), rtol=1e-12, atol=1e-12 * np.abs(ys).max())
 
 
+def test_fp8_expert_major_equals_token_major():
+    rng = np.random.default_rng(64)
+    n, H, E, k, I = 9, 256, 5, 3, 128
+    x = rng.normal(0, 1, (n, H))
+    wg, wu = rng.normal(0, 1 / 16, (2, E, I, H))
+    wd = rng.normal(0, 1 / 11.3, (E, H, I))
+    sh = (rng.normal(0, 1 / 16, (I, H)), rng.normal(0, 1 / 16, (I, H)), rng.normal(0, 1 / 11.3, (H, I)))
+    idx = _random_idx(rng, n, E, k)
+    w = rng.uniform(0, 1, (n, k))
+    a = layer.moe_layer_tokens_fp8(x, idx, w, wg, wu, wd, sh)
+    b = layer.moe_layer_tokens_fp8_by_expert(x, idx, w, lambda e: (wg[e], wu[e], wd[e]), sh)
+    assert np.allclose(a, b, rtol=1e-12, atol=1e-12 * np.abs(a).max())
+
+
 def test_fp8_pins_catch_planted_mistakes(monkeypatch):
     """Plant each plausible mistake in the oracle's FP8 emulation and check
     that at least one FP8 pin fails."""
