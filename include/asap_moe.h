@@ -357,12 +357,99 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
                                const void* const* xs, const int32_t* ns, void* const* outs,
                                void* ws, size_t ws_bytes, void* stream);
 
+/* ------------------------------------------------------------------------
+ * Mailbox: the device decides which micro-batches one grouped GEMM pass
+ * serves.  The single-GPU form of the asynchronous primitives of Sections
+ * 3.2.1 and 3.2.2 (Table 2: a payload region, a metadata region and a ready
+ * bitmap per DP group; the receiver polls the bitmaps, migrates the payload
+ * into its private memory, clears the flags, and returns results with a
+ * completion bitmap), with the MoE side serving DP groups out of order
+ * (Section 3.3).
+ *
+ *  - A DP group's stream POSTS a micro-batch into its slot: the post routes
+ *    it (exactly as asap_moe_route) into the slot's region and then sets the
+ *    slot's ready flag, an epoch, with a release store.
+ *  - The MoE stream SERVES: a service round claims, on the device, every
+ *    post whose flag is set and that has not been served when the round
+ *    starts; dispatches all claimed posts into one expert-major buffer (the
+ *    migration); runs one gate/up and one down grouped GEMM over all of them,
+ *    so each expert's weights stream from HBM once per round, not once per
+ *    micro-batch; combines each post into its own out; then sets each claimed
+ *    slot's completion flag (an epoch in device memory and in host-mapped
+ *    memory).
+ *  - out of every post is bit-identical to asap_moe_layer on the same x,
+ *    whichever other posts share its round.
+ *
+ * Ordering (no kernel waits for a kernel that may be queued behind it):
+ *  - asap_moe_mailbox_serve(slot, epoch) makes the MoE stream wait, with a
+ *    CUDA event, for the last post made to that slot; call it after the post
+ *    that returned epoch.  The round then claims that post and every other
+ *    ready one.  The round's claim kernel also checks the slot's flag and,
+ *    if epoch has not been published (a post that was announced but never
+ *    made), waits at most wait_ns, records status bit 128 and serves the
+ *    posts that are ready.
+ *  - A post to a slot waits (on its own stream, with an event) for the round
+ *    that served the slot's previous post; posting again before a serve call
+ *    was made for the previous post returns ASAP_ERR_INVALID (the sender's
+ *    backpressure of Section 3.2.1).
+ *  - x and out of a post must stay valid until the post is served.
+ *
+ * One mailbox serves one layer (layer_id, or layer 0) of its handle and owns
+ * its memory: a server workspace for n_slots * slot_tokens tokens
+ * (asap_moe_workspace_size of that many tokens) and a few KB of state.
+ * Calls are thread-safe with respect to each other (one lock per mailbox).
+ * ------------------------------------------------------------------------ */
+typedef struct asap_moe_mailbox_s* asap_moe_mailbox_t;
+
+/* Create a mailbox of n_slots slots (1..64) of up to slot_tokens tokens
+ * (<= max_tokens) each on h's device.  layer_id: NULL (layer 0) or a 4-byte
+ * aligned device int32 read by the kernels when they run.  wait_ns > 0:
+ * the limit of a round's wait for a post that has not been published.
+ * Allocates; synchronous. */
+int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot_tokens,
+                            const int32_t* layer_id, int64_t wait_ns, asap_moe_mailbox_t* out);
+
+/* Free the mailbox (synchronises the device first).  NULL is accepted. */
+int asap_moe_mailbox_destroy(asap_moe_mailbox_t m);
+
+/* Post n tokens of x (0 <= n <= slot_tokens) into slot on stream: waits on
+ * the stream for the slot's previous round, routes, publishes.  *epoch
+ * (nullable) receives the post's epoch (1, 2, ... per slot), the value to
+ * serve it with.  Enqueues only. */
+int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int32_t n,
+                          void* out, void* stream, uint64_t* epoch);
+
+/* One service round on stream for post epoch of slot, as described above.
+ * Enqueues only. */
+int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream);
+
+/* Make stream wait until the round of the serve call for slot's last post
+ * has finished (its out is then complete).  ASAP_ERR_INVALID when no serve
+ * call has been made for that post. */
+int asap_moe_mailbox_wait(asap_moe_mailbox_t m, int32_t slot, void* stream);
+
+/* The slot's completion epoch as the device last released it to host-mapped
+ * memory (0 = none yet).  Non-blocking: for a host thread that polls. */
+int asap_moe_mailbox_served(asap_moe_mailbox_t m, int32_t slot, uint64_t* epoch);
+
+/* Record ev_before / ev_after (cudaEvent_t) on the stream right before the
+ * first and right after the last grouped GEMM of the next serve call (for
+ * timing the GEMMs of a round).  NULL events clear the request. */
+int asap_moe_mailbox_time_gemms(asap_moe_mailbox_t m, void* ev_before, void* ev_after);
+
+/* Synchronise the device; *rounds = service rounds run so far; claimed
+ * (nullable) receives the number of posts each of the first min(cap,
+ * rounds, 4096) rounds claimed. */
+int asap_moe_mailbox_rounds(asap_moe_mailbox_t m, int32_t* rounds, int32_t* claimed, int32_t cap);
+
 /* Synchronise the device, return ASAP_OK or ASAP_ERR_DEVICE_STATUS, write the
  * raw status word (0 = clean) to *word if non-NULL, then clear it.  Bits:
  * 1 expert index outside [0, E); 2 permutation position out of range;
  * 4 a wait passed its time limit; 8 offsets not monotone or past the rows;
  * 16 layer id outside [0, n_layers); 32 a grouped GEMM found its dynamic
- * shared memory misaligned and did nothing. */
+ * shared memory misaligned and did nothing; 64 a mailbox slot was published
+ * again before its previous post was served; 128 a mailbox round's wait for
+ * the post it was started for ran out. */
 int asap_moe_status(asap_moe_t h, uint32_t* word);
 
 /* Thread-local text of this thread's last failure ("" if none). */

@@ -214,6 +214,83 @@ def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
                                        _ptr(offsets), _stream(stream)))
 
 
+class Mailbox:
+    """Owns an asap_moe_mailbox_t (slots that DP-group streams post routed
+    micro-batches into and that service rounds on the MoE stream claim on the
+    device); destroyed on close() or garbage collection.  Keeps the tensors
+    of every post alive until the mailbox is closed or the slot is reposted."""
+
+    def __init__(self, ptr, handle, n_slots, slot_tokens):
+        self.ptr = ptr
+        self.handle = handle          # the weights must outlive the mailbox
+        self.n_slots = n_slots
+        self.slot_tokens = slot_tokens
+        self._keep = {}
+
+    def close(self):
+        if self.ptr:
+            lib().asap_moe_mailbox_destroy(self.ptr)
+            self.ptr = None
+            self._keep.clear()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def asap_moe_mailbox_create(h, n_slots, slot_tokens, layer_id=None, wait_ns=2_000_000_000):
+    """A mailbox of n_slots slots of up to slot_tokens tokens on h (layer_id:
+    None for layer 0, or a one-element int32 CUDA tensor)."""
+    out = ctypes.c_void_p()
+    check("asap_moe_mailbox_create",
+          lib().asap_moe_mailbox_create(h.ptr, int(n_slots), int(slot_tokens), _ptr(layer_id), int(wait_ns),
+                                        ctypes.byref(out)))
+    m = Mailbox(out, h, n_slots, slot_tokens)
+    m._layer = layer_id
+    return m
+
+
+def asap_moe_mailbox_post(m, slot, x, out, stream=None):
+    """Post x (n tokens) into slot; returns the post's epoch."""
+    ep = ctypes.c_uint64()
+    check("asap_moe_mailbox_post",
+          lib().asap_moe_mailbox_post(m.ptr, int(slot), _ptr(x), x.shape[0], _ptr(out), _stream(stream),
+                                      ctypes.byref(ep)))
+    m._keep[int(slot)] = (x, out)
+    return ep.value
+
+
+def asap_moe_mailbox_serve(m, slot, epoch, stream=None):
+    check("asap_moe_mailbox_serve", lib().asap_moe_mailbox_serve(m.ptr, int(slot), int(epoch), _stream(stream)))
+
+
+def asap_moe_mailbox_wait(m, slot, stream=None):
+    check("asap_moe_mailbox_wait", lib().asap_moe_mailbox_wait(m.ptr, int(slot), _stream(stream)))
+
+
+def asap_moe_mailbox_served(m, slot):
+    ep = ctypes.c_uint64()
+    check("asap_moe_mailbox_served", lib().asap_moe_mailbox_served(m.ptr, int(slot), ctypes.byref(ep)))
+    return ep.value
+
+
+def asap_moe_mailbox_time_gemms(m, ev_before, ev_after):
+    """torch.cuda.Event pair recorded around the next serve call's GEMMs."""
+    check("asap_moe_mailbox_time_gemms",
+          lib().asap_moe_mailbox_time_gemms(m.ptr, ctypes.c_void_p(ev_before.cuda_event),
+                                            ctypes.c_void_p(ev_after.cuda_event)))
+
+
+def asap_moe_mailbox_rounds(m, cap=4096):
+    """(rounds run so far, list of the posts each round claimed); synchronises."""
+    n = ctypes.c_int32()
+    buf = (ctypes.c_int32 * cap)()
+    check("asap_moe_mailbox_rounds", lib().asap_moe_mailbox_rounds(m.ptr, ctypes.byref(n), buf, cap))
+    return n.value, list(buf[:min(cap, n.value)])
+
+
 TILING_AUTO, TILING_SINGLE, TILING_PAIRED = 0, 1, 2
 
 

@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libasap_moe.so")
-SOURCES = ["api.cu", "gemm_tc.cu", "gemm_fp8.cu", "route.cu", "route_tc.cu", "permute.cu"]
+SOURCES = ["api.cu", "gemm_tc.cu", "gemm_fp8.cu", "route.cu", "route_tc.cu", "permute.cu", "mailbox.cu"]
 HEADERS = [os.path.join(CSRC, "common.cuh"), os.path.join(CSRC, "internal.h"), os.path.join(CSRC, "gemm_sched.cuh"), os.path.join(CSRC, "gemm_config.h"),
            os.path.join(INCLUDE, "asap_moe.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -338,8 +338,11 @@ int ub_mtiles(const asap_moe_config& c, long long nk, int bm = asap::kGemmBM) {
 // GEMM1: h = silu(X Wg^T) * (X Wu^T) on the routed segments, plus the shared
 // expert on x (problem 1 of the same launch).
 // counter: a zeroed int the launch claims its tiles from (nullptr: static order).
+// m1_dev (nullable): the shared expert's row count read when the launch runs
+// (at most n); the tile count and the maps are sized for n.
 int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const void* x, int n, void* hbuf,
-                void* hsh, const int32_t* layer, int32_t* counter, cudaStream_t st) {
+                void* hsh, const int32_t* layer, int32_t* counter, cudaStream_t st,
+                const int32_t* m1_dev = nullptr) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
@@ -368,6 +371,7 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   a.out0 = hbuf;
   a.ldo0 = c.inter;
   a.m1 = sh ? n : 0;
+  a.m1_dev = sh ? m1_dev : nullptr;
   a.n_tiles1 = sh ? c.shared_inter / 128 : 0;
   a.k_iters1 = c.hidden / asap::kGemmBK;
   a.out1 = hsh;
@@ -388,7 +392,7 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
 
 // GEMM2: y = h Wd^T on the routed segments, plus the shared expert.
 int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void* hsh, int n, void* y_perm,
-             void* y_sh, const int32_t* layer, int32_t* counter, cudaStream_t st) {
+             void* y_sh, const int32_t* layer, int32_t* counter, cudaStream_t st, const int32_t* m1_dev = nullptr) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
@@ -417,6 +421,7 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.out0 = y_perm;
   a.ldo0 = c.hidden;
   a.m1 = sh ? n : 0;
+  a.m1_dev = sh ? m1_dev : nullptr;
   a.n_tiles1 = sh ? c.hidden / asap::kGemmBN : 0;
   a.k_iters1 = sh ? c.shared_inter / asap::kGemmBK : 0;
   a.out1 = y_sh;
@@ -447,7 +452,7 @@ int run_expert_ffn(asap_moe_t h, const void* x_perm, const int32_t* offsets, con
 // segments plus the shared expert on the quantised x.
 int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t* offsets, const void* xq_sh,
                     const float* xs_sh, int n, void* hq, float* hs, void* hq_sh, float* hs_sh, const int32_t* layer,
-                    int32_t* counter, cudaStream_t st) {
+                    int32_t* counter, cudaStream_t st, const int32_t* m1_dev = nullptr) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
@@ -474,6 +479,7 @@ int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t
   a.out0 = hq;
   a.ldo0 = c.inter;
   a.m1 = sh ? n : 0;
+  a.m1_dev = sh ? m1_dev : nullptr;
   a.n_tiles1 = sh ? c.shared_inter / 128 : 0;
   a.k_iters1 = c.hidden / asap::kFp8BK;
   a.out1 = hq_sh;
@@ -504,7 +510,7 @@ int run_gate_up_fp8(asap_moe_t h, const void* xq, const float* xs, const int32_t
 // FP8 GEMM2: y = (hq * hs) (Wd * sd)^T, bf16 out.
 int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* offsets, const void* hq_sh,
                  const float* hs_sh, int n, void* y_perm, void* y_sh, const int32_t* layer, int32_t* counter,
-                 cudaStream_t st) {
+                 cudaStream_t st, const int32_t* m1_dev = nullptr) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
@@ -531,6 +537,7 @@ int run_down_fp8(asap_moe_t h, const void* hq, const float* hs, const int32_t* o
   a.out0 = y_perm;
   a.ldo0 = c.hidden;
   a.m1 = sh ? n : 0;
+  a.m1_dev = sh ? m1_dev : nullptr;
   a.n_tiles1 = sh ? c.hidden / asap::kGemmBN : 0;
   a.k_iters1 = sh ? c.shared_inter / asap::kFp8BK : 0;
   a.out1 = y_sh;
@@ -1213,6 +1220,290 @@ ASAP_API int asap_moe_status(asap_moe_t h, uint32_t* word) {
   if (e != cudaSuccess) return cuda_fail(e, "status read");
   if (word) *word = v;
   if (v != 0) return fail(ASAP_ERR_DEVICE_STATUS, "device status word " + std::to_string(v));
+  return ASAP_OK;
+}
+
+// ============================================================ mailbox (device-side ready set)
+//
+// The single-GPU form of ASAP's asynchronous dispatch and combine (Sections
+// 3.2.1 and 3.2.2) with ready-set aggregation: DP groups post routed
+// micro-batches into slots on their own streams; a service round on the MoE
+// stream claims every post that is ready when the round starts (decided on
+// the device) and serves all of them with one grouped GEMM pass, so each
+// expert's weights stream from HBM once per round instead of once per
+// micro-batch.  Host state is only bookkeeping (epochs, events); nothing here
+// reads device memory back.
+
+struct asap_moe_mailbox_s {
+  asap_moe_t h = nullptr;
+  asap::MboxGeom g{};
+  const int32_t* layer = nullptr;  // device layer id of the posts
+  unsigned long long wait_ns = 0;
+  Layout L{};                      // server workspace: layout for n_slots * slot_tokens tokens
+  void* ws = nullptr;
+  asap::MboxSlot* slots = nullptr;
+  asap::MboxRound* round = nullptr;
+  int32_t* rowmap = nullptr;
+  int32_t* log = nullptr;
+  unsigned long long* served_host = nullptr;      // host-mapped completion epochs
+  unsigned long long* served_host_dev = nullptr;  // its device address
+  std::vector<cudaEvent_t> post_ev, served_ev;
+  std::vector<unsigned long long> posted, serve_called;  // host view: last post, last serve call per slot
+  cudaEvent_t gemm_ev0 = nullptr, gemm_ev1 = nullptr;   // recorded around the next round's GEMMs
+  std::mutex mu;
+};
+
+namespace {
+
+int mbox_free(asap_moe_mailbox_t m) {
+  if (!m) return ASAP_OK;
+  int prev = 0;
+  cudaGetDevice(&prev);
+  if (m->h) cudaSetDevice(m->h->device);
+  cudaDeviceSynchronize();
+  cudaFree(m->ws);
+  cudaFree(m->slots);
+  cudaFree(m->round);
+  cudaFree(m->rowmap);
+  cudaFree(m->log);
+  if (m->served_host) cudaFreeHost(m->served_host);
+  for (cudaEvent_t e : m->post_ev) cudaEventDestroy(e);
+  for (cudaEvent_t e : m->served_ev) cudaEventDestroy(e);
+  cudaSetDevice(prev);
+  delete m;
+  return ASAP_OK;
+}
+
+}  // namespace
+
+ASAP_API int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot_tokens, const int32_t* layer_id,
+                                     int64_t wait_ns, asap_moe_mailbox_t* out) {
+  if (!out) return fail(ASAP_ERR_INVALID, "NULL out");
+  *out = nullptr;
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  const asap_moe_config& c = h->cfg;
+  if (n_slots < 1 || n_slots > asap::kMboxMaxSlots)
+    return fail(ASAP_ERR_INVALID, "n_slots must be in [1, " + std::to_string(asap::kMboxMaxSlots) + "]");
+  if (slot_tokens < 1 || slot_tokens > c.max_tokens)
+    return fail(ASAP_ERR_INVALID, "slot_tokens must be in [1, max_tokens]");
+  const long long total = static_cast<long long>(n_slots) * slot_tokens;
+  if (total * c.top_k >= (1ll << 31)) return fail(ASAP_ERR_INVALID, "n_slots * slot_tokens * top_k must be < 2^31");
+  if (layer_id && !valid_layer_ptr(layer_id))
+    return fail(ASAP_ERR_INVALID, "layer_id must be NULL or a 4-byte aligned device pointer");
+  if (wait_ns <= 0) return fail(ASAP_ERR_INVALID, "wait_ns must be positive");
+  asap_moe_mailbox_s* m = new asap_moe_mailbox_s();
+  m->h = h;
+  m->g.n_slots = n_slots;
+  m->g.slot_tokens = slot_tokens;
+  m->g.slot_chunks = asap::ceil_div(slot_tokens, asap::kChunkTokens);
+  m->g.k = c.top_k;
+  m->g.E = c.n_experts;
+  m->g.H = c.hidden;
+  m->layer = layer_id ? layer_id : h->layer_ids;
+  m->wait_ns = static_cast<unsigned long long>(wait_ns);
+  m->L = layout(c, total);
+  auto bail = [&](int code) {
+    mbox_free(m);
+    return code;
+  };
+  int prev = 0;
+  cudaGetDevice(&prev);
+  cudaError_t e = cudaSetDevice(h->device);
+  if (e != cudaSuccess) return bail(cuda_fail(e, "cudaSetDevice"));
+  auto restore = [&](int code) {
+    cudaSetDevice(prev);
+    return code;
+  };
+  if ((e = cudaMalloc(&m->ws, m->L.total)) != cudaSuccess) return restore(bail(cuda_fail(e, "cudaMalloc mailbox workspace")));
+  if ((e = cudaMalloc(&m->slots, sizeof(asap::MboxSlot) * n_slots)) != cudaSuccess ||
+      (e = cudaMalloc(&m->round, sizeof(asap::MboxRound))) != cudaSuccess ||
+      (e = cudaMalloc(&m->rowmap, sizeof(int32_t) * n_slots * m->g.slot_chunks)) != cudaSuccess ||
+      (e = cudaMalloc(&m->log, sizeof(int32_t) * asap::kMboxLog)) != cudaSuccess)
+    return restore(bail(cuda_fail(e, "cudaMalloc mailbox state")));
+  if ((e = cudaHostAlloc(reinterpret_cast<void**>(&m->served_host), sizeof(unsigned long long) * n_slots,
+                         cudaHostAllocMapped)) != cudaSuccess ||
+      (e = cudaHostGetDevicePointer(reinterpret_cast<void**>(&m->served_host_dev), m->served_host, 0)) != cudaSuccess)
+    return restore(bail(cuda_fail(e, "mapped completion flags")));
+  std::memset(m->served_host, 0, sizeof(unsigned long long) * n_slots);
+  if ((e = cudaMemset(m->slots, 0, sizeof(asap::MboxSlot) * n_slots)) != cudaSuccess ||
+      (e = cudaMemset(m->round, 0, sizeof(asap::MboxRound))) != cudaSuccess ||
+      (e = cudaMemset(m->log, 0, sizeof(int32_t) * asap::kMboxLog)) != cudaSuccess)
+    return restore(bail(cuda_fail(e, "clear mailbox state")));
+  m->post_ev.assign(n_slots, nullptr);
+  m->served_ev.assign(n_slots, nullptr);
+  for (int i = 0; i < n_slots; ++i)
+    if ((e = cudaEventCreateWithFlags(&m->post_ev[i], cudaEventDisableTiming)) != cudaSuccess ||
+        (e = cudaEventCreateWithFlags(&m->served_ev[i], cudaEventDisableTiming)) != cudaSuccess)
+      return restore(bail(cuda_fail(e, "mailbox events")));
+  m->posted.assign(n_slots, 0);
+  m->serve_called.assign(n_slots, 0);
+  if ((e = cudaDeviceSynchronize()) != cudaSuccess) return restore(bail(cuda_fail(e, "mailbox create sync")));
+  *out = m;
+  return restore(ASAP_OK);
+}
+
+ASAP_API int asap_moe_mailbox_destroy(asap_moe_mailbox_t m) { return mbox_free(m); }
+
+ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int32_t n, void* out,
+                                   void* stream, uint64_t* epoch) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  asap_moe_t h = m->h;
+  const asap_moe_config& c = h->cfg;
+  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+  if (n < 0 || n > m->g.slot_tokens) return fail(ASAP_ERR_INVALID, "n outside [0, slot_tokens]");
+  if (n > 0 && (!x || !out || !aligned16(x) || !aligned16(out)))
+    return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
+  std::lock_guard<std::mutex> lock(m->mu);
+  if (m->posted[slot] > m->serve_called[slot])
+    return fail(ASAP_ERR_INVALID, "slot " + std::to_string(slot) + " still holds post " +
+                                      std::to_string(m->posted[slot]) + ", for which no serve call has been made");
+  cudaStream_t st = S(stream);
+  const unsigned long long ep = m->posted[slot] + 1;
+  // backpressure (Section 3.2.1): the round that served the slot's previous
+  // post must be done with the slot's region before it is written again
+  CU_TRY(cudaStreamWaitEvent(st, m->served_ev[slot], 0), "wait for the slot's previous round");
+  const asap::MboxGeom& g = m->g;
+  const long long sk = static_cast<long long>(slot) * g.slot_tokens * c.top_k;
+  int32_t* idx = at<int32_t>(m->ws, m->L.idx) + sk;
+  float* w = at<float>(m->ws, m->L.w) + sk;
+  int32_t* hist = at<int32_t>(m->ws, m->L.hist);
+  const int chunk0 = slot * g.slot_chunks, chunks_total = g.n_slots * g.slot_chunks;
+  int r;
+  if (n > 0) {
+    // routing exactly as asap_moe_route routes n tokens; the histogram rows
+    // are the slot's, scanned later together with the other claimed posts
+    if (fused_route(h)) {
+      if ((r = run_route_fused(h, x, n, idx, w, hist, chunk0, chunks_total, nullptr, nullptr, nullptr, nullptr,
+                               nullptr, m->layer, st)) != ASAP_OK)
+        return r;
+    } else {
+      const int splits = router_splits(h, n);
+      float* lg = at<float>(m->ws, m->L.logits) +
+                  static_cast<long long>(slot) * asap::kMaxRouterSplits * g.slot_tokens * c.n_experts;
+      if ((r = run_router_logits(h, x, n, lg, splits, m->layer, st)) != ASAP_OK) return r;
+      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, m->layer, nullptr), idx, w, hist, chunk0,
+                                   chunks_total, st),
+             "gate launch");
+    }
+  }
+  CU_TRY(asap::launch_mbox_publish(m->slots, slot, x, n, out, ep, h->status, st), "publish launch");
+  CU_TRY(cudaEventRecord(m->post_ev[slot], st), "post event");
+  m->posted[slot] = ep;
+  if (epoch) *epoch = ep;
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  asap_moe_t h = m->h;
+  const asap_moe_config& c = h->cfg;
+  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+  if (epoch < 1) return fail(ASAP_ERR_INVALID, "epoch must be >= 1 (the value asap_moe_mailbox_post returned)");
+  std::lock_guard<std::mutex> lock(m->mu);
+  cudaStream_t st = S(stream);
+  const asap::MboxGeom& g = m->g;
+  const Layout& L = m->L;
+  void* ws = m->ws;
+  const int N = g.n_slots * g.slot_tokens;  // upper bound of the round's tokens
+  const bool sh = c.n_shared != 0;
+  int32_t* offsets = at<int32_t>(ws, L.offsets);
+  int32_t* counters = at<int32_t>(ws, L.tile_counters);
+  const int32_t* n_total = &m->round->n_total;
+  int r;
+  // the post this round is for was published before the round starts
+  CU_TRY(cudaStreamWaitEvent(st, m->post_ev[slot], 0), "wait for the post");
+  CU_TRY(asap::launch_mbox_claim(m->slots, g, slot, epoch, m->wait_ns, m->round, m->rowmap, at<int32_t>(ws, L.ticket),
+                                 h->status, st),
+         "claim launch");
+  CU_TRY(asap::launch_scan_mapped(at<int32_t>(ws, L.hist), m->rowmap, &m->round->chunks_total,
+                                  g.n_slots * g.slot_chunks, c.n_experts, at<int32_t>(ws, L.counts), offsets,
+                                  at<int32_t>(ws, L.chunk_base), at<int32_t>(ws, L.ticket), counters, st),
+         "scan launch");
+  const int32_t* idx = at<int32_t>(ws, L.idx);
+  int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
+  void* y_sh = sh ? at<void>(ws, L.y_sh) : nullptr;
+  void* y_perm;
+  if (h->fp8) {
+    void* xq_sh = sh ? at<void>(ws, L.xq_sh) : nullptr;
+    float* xs_sh = sh ? at<float>(ws, L.xs_sh) : nullptr;
+    CU_TRY(asap::launch_dispatch_fp8_mbox(m->round, g, idx, at<int32_t>(ws, L.chunk_base), offsets, at<void>(ws, L.xq),
+                                          at<float>(ws, L.xs), xq_sh, xs_sh, at<int32_t>(ws, L.perm_src), perm_dst,
+                                          h->status, st),
+           "dispatch launch");
+    if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
+    if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, N, at<void>(ws, L.hq),
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), m->layer, counters,
+                             st, n_total)) != ASAP_OK)
+      return r;
+    y_perm = at<void>(ws, L.y_perm);
+    if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
+                          at<float>(ws, L.hs_sh), N, y_perm, y_sh, m->layer, counters + 1, st, n_total)) != ASAP_OK)
+      return r;
+  } else {
+    // the shared expert reads the gathered rows from y_sh's region, which its
+    // own output overwrites only after the gate/up GEMM
+    y_perm = at<void>(ws, L.x_perm);
+    CU_TRY(asap::launch_dispatch_mbox(m->round, g, idx, at<int32_t>(ws, L.chunk_base), offsets, y_perm,
+                                      at<int32_t>(ws, L.perm_src), perm_dst, y_sh, h->status, st),
+           "dispatch launch");
+    if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
+    if ((r = run_gate_up(h, y_perm, offsets, y_sh, N, at<void>(ws, L.h), at<void>(ws, L.h_sh), m->layer, counters, st,
+                         n_total)) != ASAP_OK)
+      return r;
+    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), N, y_perm, y_sh, m->layer, counters + 1,
+                      st, n_total)) != ASAP_OK)
+      return r;
+  }
+  if (m->gemm_ev1) CU_TRY(cudaEventRecord(m->gemm_ev1, st), "timing event");
+  m->gemm_ev0 = m->gemm_ev1 = nullptr;
+  CU_TRY(asap::launch_combine_mbox(m->round, g, y_perm, y_sh, at<float>(ws, L.w), perm_dst, h->status, st),
+         "combine launch");
+  CU_TRY(asap::launch_mbox_finish(m->slots, m->round, m->log, m->served_host_dev, st), "finish launch");
+  CU_TRY(cudaEventRecord(m->served_ev[slot], st), "served event");
+  if (epoch > m->serve_called[slot]) m->serve_called[slot] = epoch;
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_mailbox_wait(asap_moe_mailbox_t m, int32_t slot, void* stream) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+  std::lock_guard<std::mutex> lock(m->mu);
+  if (m->serve_called[slot] < m->posted[slot])
+    return fail(ASAP_ERR_INVALID, "no serve call has been made for the slot's last post");
+  CU_TRY(cudaStreamWaitEvent(S(stream), m->served_ev[slot], 0), "wait for the slot's round");
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_mailbox_served(asap_moe_mailbox_t m, int32_t slot, uint64_t* epoch) {
+  if (!m || !epoch) return fail(ASAP_ERR_INVALID, "NULL mailbox or output");
+  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+  *epoch = *reinterpret_cast<volatile unsigned long long*>(m->served_host + slot);
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_mailbox_time_gemms(asap_moe_mailbox_t m, void* ev_before, void* ev_after) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  std::lock_guard<std::mutex> lock(m->mu);
+  m->gemm_ev0 = static_cast<cudaEvent_t>(ev_before);
+  m->gemm_ev1 = static_cast<cudaEvent_t>(ev_after);
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_mailbox_rounds(asap_moe_mailbox_t m, int32_t* rounds, int32_t* claimed, int32_t cap) {
+  if (!m || !rounds) return fail(ASAP_ERR_INVALID, "NULL mailbox or output");
+  int prev = 0;
+  cudaGetDevice(&prev);
+  cudaSetDevice(m->h->device);
+  cudaError_t e = cudaDeviceSynchronize();
+  int32_t cnt = 0;
+  if (e == cudaSuccess)
+    e = cudaMemcpy(&cnt, &m->round->rounds, sizeof(int32_t), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && claimed && cap > 0)
+    e = cudaMemcpy(claimed, m->log, sizeof(int32_t) * std::min(std::min(cap, cnt), asap::kMboxLog),
+                   cudaMemcpyDeviceToHost);
+  cudaSetDevice(prev);
+  if (e != cudaSuccess) return cuda_fail(e, "mailbox rounds read");
+  *rounds = cnt;
   return ASAP_OK;
 }
 

@@ -20,6 +20,8 @@ enum : uint32_t {
   ST_BAD_OFFSETS = 1u << 3,       // offsets not monotone or past the rows
   ST_BAD_LAYER = 1u << 4,         // layer id outside [0, n_layers); layer 0 was used
   ST_SMEM_ALIGN = 1u << 5,        // dynamic shared memory not 1024-byte aligned; the GEMM did nothing
+  ST_MBOX_OVERRUN = 1u << 6,      // a mailbox slot was posted again before its previous post was served
+  ST_MBOX_WAIT = 1u << 7,         // a mailbox round's wait for the post it serves ran out
 };
 
 __device__ __forceinline__ void record_status(uint32_t* st, uint32_t bits) {

@@ -198,7 +198,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int total0 = sch->tile_start[G];
-  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BM - 1) / BM) * args.n_tiles1 : 0);
+  const int total = total0 + (sch->m1 > 0 ? ((sch->m1 + BM - 1) / BM) * args.n_tiles1 : 0);
   TileQueue tq{tq_base};
 
   if ((warp == 0 || warp == kAProdWarp) && lane == 0) {
@@ -339,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (t < 0) break;
       Tile T;
       decode_tile(t, sch, G, total0, args, T);
-      const int mrows = T.p1 ? args.m1 : args.m0;
+      const int mrows = T.p1 ? sch->m1 : args.m0;
       const long long row = static_cast<long long>(T.a_row) + r;
       const long long srow = row < mrows ? row : mrows - 1;  // in-bounds scale row for masked rows
       const int asld = T.p1 ? fa.a_sld1 : fa.a_sld0;

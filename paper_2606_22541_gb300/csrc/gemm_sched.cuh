@@ -13,6 +13,7 @@ namespace asap {
 struct Sched {
   int tile_start[kMaxExperts + 1];
   int row_base[kMaxExperts + 1];
+  int m1;  // rows of problem 1 in this launch (args.m1, or *args.m1_dev clamped to [0, args.m1])
 };
 
 struct Tile {
@@ -109,11 +110,11 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
     T.p1 = false;
   } else {
     const int u = t - total0;
-    const int mt = (a.m1 + BMT - 1) / BMT;
+    const int mt = (s->m1 + BMT - 1) / BMT;
     const int nt = u / mt;
     const int mi = u - nt * mt;
     T.a_row = mi * BMT;
-    T.rows = min(BMT, a.m1 - mi * BMT);
+    T.rows = min(BMT, s->m1 - mi * BMT);
     T.b_row = nt * kGemmBN;
     T.n_tile = nt;
     T.split = 0;
@@ -130,6 +131,7 @@ __device__ __forceinline__ void decode_tile(int t, const Sched* s, int G, int to
 // the rows are reported in the status word and leave problem 0 empty.
 template <int BMT = kGemmBM>
 __device__ __forceinline__ void build_schedule(const GemmArgs& args, Sched* sch, int G, int lane) {
+  if (lane == 0) sch->m1 = args.m1_dev ? min(max(__ldg(args.m1_dev), 0), args.m1) : args.m1;
   int local = 0;
   int cnt[8];
   int lo[8];

@@ -290,7 +290,7 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int total0 = sch->tile_start[G];
-  const int total = total0 + (args.m1 > 0 ? ((args.m1 + BMT - 1) / BMT) * args.n_tiles1 : 0);
+  const int total = total0 + (sch->m1 > 0 ? ((sch->m1 + BMT - 1) / BMT) * args.n_tiles1 : 0);
   TileQueue tq{tq_base};
 
   if ((warp == 0 || warp == C::kAProdWarp) && lane == 0) {

@@ -51,7 +51,8 @@ struct GemmArgs {
   int k_iters0;            // K0 / 64
   void* out0;
   long long ldo0;          // elements between output rows
-  int m1;                  // rows of problem 1 (0 = none)
+  int m1;                  // rows of problem 1 (0 = none; the upper bound when m1_dev is set)
+  const int32_t* m1_dev;   // nullable: rows of problem 1 read when the launch runs, clamped to [0, m1]
   int n_tiles1;
   int k_iters1;
   void* out1;
@@ -222,6 +223,83 @@ cudaError_t launch_dispatch_fp8_seg(const void* x, int n, int H, int k, int E, c
 // rows.  R % 256 == 0 and row_bytes % 128 == 0.
 cudaError_t launch_retile(const void* a, const void* b, int E, int R, long long row_bytes, bool gate_up, void* dst,
                           cudaStream_t s);
+
+// ------------------------------------------------------------ mailbox
+// The single-GPU form of ASAP's asynchronous dispatch and combine (Sections
+// 3.2.1 and 3.2.2): each attention DP group posts a routed micro-batch into
+// its slot and sets the slot's ready flag (an epoch); a service round claims
+// every slot whose flag is set when the round starts, "migrates" the claimed
+// payloads into one expert-major buffer, runs one grouped GEMM pass over all
+// of them, writes each micro-batch's output and sets the slot's completion
+// flag.  Waits inside the kernels are on flags written before the waiting
+// kernel was enqueued (the host orders them with events); each is bounded.
+constexpr int kMboxMaxSlots = 64;
+constexpr int kMboxLog = 4096;  // rounds whose claimed-slot count is recorded
+
+struct MboxSlot {            // one per slot, device memory
+  unsigned long long posted;  // epoch of the slot's last published post (release by the publish kernel)
+  unsigned long long served;  // epoch of its last served post (release by a round's finish kernel)
+  const void* x;              // the post's hidden states [n, H]
+  void* out;                  // its layer output [n, H]
+  int n;
+  int pad_;
+};
+
+struct MboxRound {           // the set the current service round claimed (its claim kernel writes it)
+  int count;                 // claimed slots
+  int n_total;               // their tokens: rows of the shared expert's input
+  int chunks_total;          // their histogram rows (rowmap entries)
+  int rounds;                // service rounds run so far, this one included
+  int slot[kMboxMaxSlots];   // claimed slots, increasing
+  int n[kMboxMaxSlots];
+  int tok0[kMboxMaxSlots];   // first token in the round's combined token order
+  unsigned long long epoch[kMboxMaxSlots];
+  const void* x[kMboxMaxSlots];
+  void* out[kMboxMaxSlots];
+};
+
+// Where each slot's per-post data sits (fixed when the mailbox is made):
+// slot s owns tokens [s * slot_tokens, (s + 1) * slot_tokens) of the idx, w
+// and perm_dst arrays (k entries per token) and histogram rows
+// [s * slot_chunks, (s + 1) * slot_chunks).
+struct MboxGeom {
+  int n_slots, slot_tokens, slot_chunks;
+  int k, E, H;
+};
+
+// Producer: publish a post (after its routing on the same stream).  Records
+// ST_MBOX_OVERRUN when the slot's previous post has not been served.
+cudaError_t launch_mbox_publish(MboxSlot* slots, int slot, const void* x, int n, void* out,
+                                unsigned long long epoch, uint32_t* status, cudaStream_t s);
+// Service round, step 1: wait (at most wait_ns) until slot own_slot has
+// published epoch own_epoch (own_slot < 0: no wait; a wait that runs out
+// records ST_MBOX_WAIT), then claim every slot with posted > served into *r,
+// write the histogram row map, zero the scan's ticket.
+cudaError_t launch_mbox_claim(MboxSlot* slots, MboxGeom g, int own_slot, unsigned long long own_epoch,
+                              unsigned long long wait_ns, MboxRound* r, int32_t* rowmap, int32_t* ticket,
+                              uint32_t* status, cudaStream_t s);
+// The scan over the histogram rows rowmap[0 .. *n_chunks) (chunk_base written
+// at the same rows), otherwise as launch_scan.
+cudaError_t launch_scan_mapped(const int32_t* hist, const int32_t* rowmap, const int32_t* n_chunks, int max_chunks,
+                               int E, int32_t* counts, int32_t* offsets, int32_t* chunk_base, int32_t* ticket,
+                               int32_t* tile_counters, cudaStream_t s);
+// Dispatch of every claimed post into the combined expert segments (rows in
+// (claimed slot, token, slot of k) order); perm_src holds combined token
+// indices, perm_dst the slot's own region; x_sh / xq_sh, xs_sh receive the
+// combined rows of the shared expert.
+cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
+                                 const int32_t* offsets, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
+                                 void* x_sh, uint32_t* status, cudaStream_t s);
+cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
+                                     const int32_t* offsets, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                     int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+// Combine of every claimed post into its own output.
+cudaError_t launch_combine_mbox(const MboxRound* r, MboxGeom g, const void* y_perm, const void* y_shared,
+                                const float* w, const int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+// Service round, last step: release each claimed slot's completion epoch (and
+// its copy in host-mapped memory, nullable) and log the claimed count.
+cudaError_t launch_mbox_finish(MboxSlot* slots, const MboxRound* r, int32_t* log, unsigned long long* served_host,
+                               cudaStream_t s);
 
 inline int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
 

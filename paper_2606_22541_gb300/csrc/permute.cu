@@ -66,18 +66,19 @@ __device__ __forceinline__ uint2 quantize8(uint4 v, float& scale) {
   return make_uint2(w[0], w[1]);
 }
 
+// Chunk c (part ``part`` of its row copies) of one micro-batch; the body of
+// the dispatch kernels (one CTA per chunk and part).
 template <bool FP8>
-__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
-    dispatch_kernel(const uint4* __restrict__ x, int n, int V, int k, int E,
-                    const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
-                    void* __restrict__ x_perm_v, float* __restrict__ xs, uint2* __restrict__ xq_sh,
-                    float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
-                    int32_t* __restrict__ perm_dst, uint32_t* status, const DispatchSeg seg) {
+__device__ __forceinline__ void dispatch_chunk(int c, int part, const uint4* __restrict__ x, int n, int V, int k,
+                                               int E, const int32_t* __restrict__ idx,
+                                               const int32_t* __restrict__ chunk_base, void* __restrict__ x_perm_v,
+                                               float* __restrict__ xs, uint2* __restrict__ xq_sh,
+                                               float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
+                                               int32_t* __restrict__ perm_dst, uint32_t* status,
+                                               const DispatchSeg& seg) {
   __shared__ int wcnt[kRankWarps][kMaxExperts];
   __shared__ int spos[kChunkTokens * kMaxTopK];
   constexpr int kParts = dispatch_parts<FP8>();
-  const int c = blockIdx.x / kParts;
-  const int part = blockIdx.x % kParts;
   const int t0 = c * kChunkTokens;
   const int nt = min(kChunkTokens, n - t0);
   const int ne = nt * k;
@@ -188,6 +189,62 @@ __global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
   }
 }
 
+template <bool FP8>
+__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
+    dispatch_kernel(const uint4* __restrict__ x, int n, int V, int k, int E,
+                    const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base, int n_chunks,
+                    void* __restrict__ x_perm_v, float* __restrict__ xs, uint2* __restrict__ xq_sh,
+                    float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
+                    int32_t* __restrict__ perm_dst, uint32_t* status, const DispatchSeg seg) {
+  constexpr int kParts = dispatch_parts<FP8>();
+  dispatch_chunk<FP8>(blockIdx.x / kParts, blockIdx.x % kParts, x, n, V, k, E, idx, chunk_base, x_perm_v, xs, xq_sh,
+                      xs_sh, perm_src, perm_dst, status, seg);
+}
+
+// Dispatch of a mailbox round: CTA (i, c, part) handles chunk c of the i-th
+// claimed post; CTAs past the claimed posts or their chunks return at once.
+// The post's tokens come first in the combined order at r->tok0[i], its
+// histogram rows and chunk bases are its slot's rows, its idx / perm_dst
+// entries its slot's region.
+template <bool FP8>
+__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
+    dispatch_mbox_kernel(const MboxRound* __restrict__ r, const MboxGeom g, const int32_t* __restrict__ idx,
+                         const int32_t* __restrict__ chunk_base, const int32_t* __restrict__ offsets,
+                         void* __restrict__ x_perm_v, float* __restrict__ xs, void* __restrict__ x_sh,
+                         float* __restrict__ xs_sh, int32_t* __restrict__ perm_src, int32_t* __restrict__ perm_dst,
+                         uint32_t* status) {
+  constexpr int kParts = dispatch_parts<FP8>();
+  const int per_slot = g.slot_chunks * kParts;
+  const int i = blockIdx.x / per_slot;
+  const int rem = blockIdx.x - i * per_slot;
+  const int c = rem / kParts, part = rem % kParts;
+  if (i >= r->count) return;
+  const int n = r->n[i];
+  if (c * kChunkTokens >= n) return;
+  const int slot = r->slot[i];
+  const long long tok0 = r->tok0[i];
+  const int V = g.H / 8;
+  DispatchSeg seg{};
+  seg.expert_offsets = offsets;
+  seg.chunk0 = slot * g.slot_chunks;
+  seg.n_chunks_total = g.n_slots * g.slot_chunks;
+  seg.tok0 = static_cast<int>(tok0);
+  seg.rows_total = static_cast<long long>(r->n_total) * g.k;
+  uint2* xq_sh = nullptr;
+  float* xs_sh_i = nullptr;
+  if constexpr (FP8) {
+    if (x_sh) {
+      xq_sh = static_cast<uint2*>(x_sh) + tok0 * V;
+      xs_sh_i = xs_sh + tok0 * (V / 16);
+    }
+  } else {
+    seg.x_sh = x_sh ? static_cast<void*>(static_cast<uint4*>(x_sh) + tok0 * V) : nullptr;
+  }
+  const long long sidx = static_cast<long long>(slot) * g.slot_tokens * g.k;
+  dispatch_chunk<FP8>(c, part, static_cast<const uint4*>(r->x[i]), n, V, g.k, g.E, idx + sidx, chunk_base, x_perm_v,
+                      xs, xq_sh, xs_sh_i, perm_src, perm_dst + sidx, status, seg);
+}
+
 // Rows of bf16 to e4m3 with a scale per 128 channels; one warp per row.
 __global__ void __launch_bounds__(256) quantize_rows_kernel(const uint4* __restrict__ x, int rows, int V,
                                                             uint2* __restrict__ q, float* __restrict__ s) {
@@ -207,13 +264,12 @@ constexpr int kCombineWarps = 8;
 
 // One warp per token: out[t] = sum_j w[t,j] y_perm[perm_dst[t,j]] (+ y_sh[t]),
 // fp32 fused multiply-adds in slot order, then the shared row, then bf16.
-__global__ void __launch_bounds__(kCombineWarps * 32)
-    combine_kernel(const uint4* __restrict__ y_perm, const uint4* __restrict__ y_sh,
-                   const float* __restrict__ w, const int32_t* __restrict__ perm_dst, int n, int V,
-                   int k, uint4* __restrict__ out, uint32_t* status, long long nk) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t = blockIdx.x * kCombineWarps + warp;
-  if (t >= n) return;
+// The body for one token: w_t, pd_t its k weights and positions, y_sh_t its
+// shared-expert row (nullable), out_t its output row.
+__device__ __forceinline__ void combine_token(const uint4* __restrict__ y_perm, const uint4* __restrict__ y_sh_t,
+                                              const float* __restrict__ w_t, const int32_t* __restrict__ pd_t, int V,
+                                              int k, uint4* __restrict__ out_t, uint32_t* status, long long nk,
+                                              int lane) {
   int p[kMaxTopK];
   float wj[kMaxTopK];
 #pragma unroll
@@ -221,8 +277,8 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     p[j] = -1;
     wj[j] = 0.f;
     if (j < k) {
-      p[j] = perm_dst[static_cast<long long>(t) * k + j];
-      wj[j] = w[static_cast<long long>(t) * k + j];
+      p[j] = pd_t[j];
+      wj[j] = w_t[j];
       if (p[j] < 0 || p[j] >= nk) {
         if (lane == 0) record_status(status, ST_BAD_POSITION);
         p[j] = -1;
@@ -252,8 +308,8 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
         acc[7] = fmaf(a, bf16_hi(yv[j].w), acc[7]);
       }
     }
-    if (y_sh) {
-      const uint4 s = __ldg(y_sh + static_cast<long long>(t) * V + v);
+    if (y_sh_t) {
+      const uint4 s = __ldg(y_sh_t + v);
       acc[0] += bf16_lo(s.x);
       acc[1] += bf16_hi(s.x);
       acc[2] += bf16_lo(s.y);
@@ -263,10 +319,41 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
       acc[6] += bf16_lo(s.w);
       acc[7] += bf16_hi(s.w);
     }
-    out[static_cast<long long>(t) * V + v] =
-        make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
-                   pack_bf16x2(acc[6], acc[7]));
+    out_t[v] = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                          pack_bf16x2(acc[6], acc[7]));
   }
+}
+
+__global__ void __launch_bounds__(kCombineWarps * 32)
+    combine_kernel(const uint4* __restrict__ y_perm, const uint4* __restrict__ y_sh,
+                   const float* __restrict__ w, const int32_t* __restrict__ perm_dst, int n, int V,
+                   int k, uint4* __restrict__ out, uint32_t* status, long long nk) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kCombineWarps + warp;
+  if (t >= n) return;
+  const long long tk = static_cast<long long>(t) * k, tv = static_cast<long long>(t) * V;
+  combine_token(y_perm, y_sh ? y_sh + tv : nullptr, w + tk, perm_dst + tk, V, k, out + tv, status, nk, lane);
+}
+
+// Combine of a mailbox round: CTA (i, b) combines tokens b * kCombineWarps ..
+// of the i-th claimed post into that post's output; its weights and
+// positions are in its slot's region, its shared-expert rows at its place in
+// the combined order.
+__global__ void __launch_bounds__(kCombineWarps * 32)
+    combine_mbox_kernel(const MboxRound* __restrict__ r, const MboxGeom g, const uint4* __restrict__ y_perm,
+                        const uint4* __restrict__ y_sh, const float* __restrict__ w,
+                        const int32_t* __restrict__ perm_dst, uint32_t* status) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int per_slot = (g.slot_tokens + kCombineWarps - 1) / kCombineWarps;
+  const int i = blockIdx.x / per_slot;
+  if (i >= r->count) return;
+  const int t = (blockIdx.x - i * per_slot) * kCombineWarps + warp;
+  if (t >= r->n[i]) return;
+  const int V = g.H / 8;
+  const long long tk = (static_cast<long long>(r->slot[i]) * g.slot_tokens + t) * g.k;
+  const long long nk = static_cast<long long>(r->n_total) * g.k;
+  combine_token(y_perm, y_sh ? y_sh + (static_cast<long long>(r->tok0[i]) + t) * V : nullptr, w + tk, perm_dst + tk, V,
+                g.k, static_cast<uint4*>(r->out[i]) + static_cast<long long>(t) * V, status, nk, lane);
 }
 
 // packed[e][b*256 + r] = gate[e][b*128 + r] for r < 128, up[e][b*128 + r - 128]
@@ -363,6 +450,33 @@ cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float
   combine_kernel<<<ceil_div(n, kCombineWarps), kCombineWarps * 32, 0, s>>>(
       static_cast<const uint4*>(y_perm), static_cast<const uint4*>(y_shared), w, perm_dst, n, H / 8, k,
       static_cast<uint4*>(out), status, rows_total > 0 ? rows_total : static_cast<long long>(n) * k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
+                                 const int32_t* offsets, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
+                                 void* x_sh, uint32_t* status, cudaStream_t s) {
+  const int grid = g.n_slots * g.slot_chunks * dispatch_parts<false>();
+  dispatch_mbox_kernel<false><<<grid, dispatch_warps<false>() * 32, 0, s>>>(r, g, idx, chunk_base, offsets, x_perm,
+                                                                            nullptr, x_sh, nullptr, perm_src,
+                                                                            perm_dst, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
+                                     const int32_t* offsets, void* xq, float* xs, void* xq_sh, float* xs_sh,
+                                     int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+  const int grid = g.n_slots * g.slot_chunks * dispatch_parts<true>();
+  dispatch_mbox_kernel<true><<<grid, dispatch_warps<true>() * 32, 0, s>>>(r, g, idx, chunk_base, offsets, xq, xs,
+                                                                          xq_sh, xs_sh, perm_src, perm_dst, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine_mbox(const MboxRound* r, MboxGeom g, const void* y_perm, const void* y_shared,
+                                const float* w, const int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
+  const int grid = g.n_slots * ceil_div(g.slot_tokens, kCombineWarps);
+  combine_mbox_kernel<<<grid, kCombineWarps * 32, 0, s>>>(r, g, static_cast<const uint4*>(y_perm),
+                                                          static_cast<const uint4*>(y_shared), w, perm_dst, status);
   return cudaGetLastError();
 }
 

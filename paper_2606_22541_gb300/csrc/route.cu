@@ -615,15 +615,23 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* swarp, int& tota
   return r;
 }
 
+// MAPPED (a mailbox round): the rows scanned are rowmap[0 .. *n_chunks_dev)
+// of hist, in that order (n_chunks is then rowmap's length), and chunk_base
+// is written at the same rows.
+template <bool MAPPED>
 __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __restrict__ hist, int n_chunks, int E,
                                                             int32_t* __restrict__ counts,
                                                             int32_t* __restrict__ offsets,
                                                             int32_t* __restrict__ chunk_base,
                                                             int32_t* __restrict__ tile_counters,
-                                                            int32_t* __restrict__ ticket) {
+                                                            int32_t* __restrict__ ticket,
+                                                            const int32_t* __restrict__ rowmap,
+                                                            const int32_t* __restrict__ n_chunks_dev) {
   __shared__ int part[kScanWarps][32];
   __shared__ int swarp[33];
   __shared__ bool last;
+  if constexpr (MAPPED) n_chunks = max(0, min(*n_chunks_dev, n_chunks));  // n_chunks: rowmap's length
+  auto row = [&](int c) -> long long { return MAPPED ? rowmap[c] : c; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int e = blockIdx.x * 32 + lane;
   const bool ve = e < E;
@@ -632,7 +640,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
   int sum = 0;
   if (ve) {
 #pragma unroll 8
-    for (int c = c0; c < c1; ++c) sum += hist[static_cast<long long>(c) * E + e];
+    for (int c = c0; c < c1; ++c) sum += hist[row(c) * E + e];
   }
   part[warp][lane] = sum;
   __syncthreads();
@@ -646,7 +654,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(const int32_t* __res
   if (ve) {
 #pragma unroll 8
     for (int c = c0; c < c1; ++c) {
-      const long long o = static_cast<long long>(c) * E + e;
+      const long long o = row(c) * E + e;
       const int v = hist[o];
       chunk_base[o] = run;
       run += v;
@@ -765,8 +773,16 @@ cudaError_t launch_reduce_splits(const float* parts, int splits, long long plane
 
 cudaError_t launch_scan(const int32_t* hist, int n_chunks, int E, int32_t* counts, int32_t* offsets,
                         int32_t* chunk_base, int32_t* ticket, cudaStream_t s, int32_t* tile_counters) {
-  scan_kernel<<<ceil_div(E, 32), kScanThreads, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base, tile_counters,
-                                                      ticket);
+  scan_kernel<false><<<ceil_div(E, 32), kScanThreads, 0, s>>>(hist, n_chunks, E, counts, offsets, chunk_base,
+                                                             tile_counters, ticket, nullptr, nullptr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scan_mapped(const int32_t* hist, const int32_t* rowmap, const int32_t* n_chunks, int max_chunks,
+                               int E, int32_t* counts, int32_t* offsets, int32_t* chunk_base, int32_t* ticket,
+                               int32_t* tile_counters, cudaStream_t s) {
+  scan_kernel<true><<<ceil_div(E, 32), kScanThreads, 0, s>>>(hist, max_chunks, E, counts, offsets, chunk_base,
+                                                            tile_counters, ticket, rowmap, n_chunks);
   return cudaGetLastError();
 }
 

@@ -1,0 +1,239 @@
+"""The mailbox (device-side ready set): DP-group streams post routed
+micro-batches into slots; service rounds on the MoE stream claim, on the
+device, every post published when they start and serve all of them with one
+grouped GEMM pass.  Whichever posts share a round, each output must equal
+asap_moe_layer on the same micro-batch bit for bit.  Arrival orders and
+delays are driven from the host (posts in random slot order on several
+streams, each behind a random GPU sleep); the one failure case is a round
+started for a post that is never made, whose bounded wait must run out,
+record its status bit and still serve what is ready."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_22541_gb300 import api, inputs
+from paper_2606_22541_gb300._native import AsapError
+from paper_2606_22541_gb300.configs import DSV3, DSV3_FP8, MIXTRAL
+
+from _helpers import bf16_to_f64, compare_rows
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+ST_MBOX_WAIT = 128
+
+DS = inputs.small_variant(DSV3, name="mbox_ds", hidden=1024, inter=256, shared_inter=256,
+                          microbatches=[700, 301, 512, 1000, 96, 333])
+MX = inputs.small_variant(MIXTRAL, name="mbox_mx", hidden=1024, inter=512, microbatches=[1000, 333, 64, 517])
+F8 = inputs.small_variant(DSV3_FP8, name="mbox_f8", hidden=512, inter=256, shared_inter=256,
+                          microbatches=[300, 77, 2, 129])
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+class Case:
+    _cache = {}
+
+    @classmethod
+    def get(cls, cfg):
+        if cfg.name not in cls._cache:
+            cls._cache[cfg.name] = cls(cfg)
+        return cls._cache[cfg.name]
+
+    def __init__(self, cfg):
+        self.cfg = cfg
+        self.w = inputs.make_weights(cfg, DEV)
+        self.h = api.asap_moe_create(cfg, self.w, max(cfg.microbatches))
+        self.xs = inputs.make_microbatches(cfg, DEV)
+        self.ref = []
+        for x in self.xs:
+            o = torch.empty_like(x)
+            api.asap_moe_layer(self.h, x, o, api.workspace(self.h, x.shape[0]))
+            self.ref.append(o)
+        torch.cuda.synchronize()
+
+
+def same_bits(a, b):
+    return torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
+def assert_clean(h, allowed=0):
+    code, word = api.asap_moe_status(h)
+    assert word & ~allowed == 0, f"status {word:#x}"
+    return word
+
+
+@pytest.mark.parametrize("cfg", [DS, MX, F8], ids=lambda c: c.name)
+def test_all_posted_first_are_served_by_one_round(cfg):
+    """Every post published before the first round starts: that round claims
+    all of them; the later rounds find nothing left."""
+    c = Case.get(cfg)
+    n = len(c.xs)
+    m = api.asap_moe_mailbox_create(c.h, n, max(cfg.microbatches))
+    streams = [torch.cuda.Stream() for _ in range(n)]
+    outs = [torch.full_like(x, 7.0) for x in c.xs]
+    eps = [api.asap_moe_mailbox_post(m, i, x, o, stream=s) for i, (x, o, s) in enumerate(zip(c.xs, outs, streams))]
+    torch.cuda.synchronize()
+    server = torch.cuda.Stream()
+    for i in range(n):
+        api.asap_moe_mailbox_serve(m, i, eps[i], stream=server)
+    torch.cuda.synchronize()
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == n and claimed == [n] + [0] * (n - 1)
+    for a, b in zip(c.ref, outs):
+        assert same_bits(a, b)
+    assert [api.asap_moe_mailbox_served(m, i) for i in range(n)] == eps
+    assert_clean(c.h)
+    m.close()
+
+
+@pytest.mark.parametrize("cfg", [DS, MX, F8], ids=lambda c: c.name)
+def test_random_arrivals_and_delays(cfg):
+    """Posts in random slot order on three producer streams, each behind a
+    random GPU sleep, every post served right after it was made: the device
+    decides how the posts group into rounds; the outputs may not depend on
+    it.  Three passes reuse the slots (epochs 1, 2, 3)."""
+    c = Case.get(cfg)
+    n = len(c.xs)
+    rng = np.random.default_rng(7)
+    m = api.asap_moe_mailbox_create(c.h, n, max(cfg.microbatches))
+    producers = [torch.cuda.Stream() for _ in range(3)]
+    server = torch.cuda.Stream()
+    consumer = torch.cuda.Stream()
+    total_posts = 0
+    for rep in range(3):
+        outs = [torch.full_like(x, float(rep + 3)) for x in c.xs]
+        order = rng.permutation(n)
+        for i in order:
+            s = producers[int(rng.integers(0, 3))]
+            with torch.cuda.stream(s):
+                torch.cuda._sleep(int(rng.integers(0, 400_000)))
+            if rep > 0:
+                api.asap_moe_mailbox_wait(m, int(i), stream=s)   # the slot's previous post is done
+            ep = api.asap_moe_mailbox_post(m, int(i), c.xs[i], outs[i], stream=s)
+            assert ep == rep + 1
+            api.asap_moe_mailbox_serve(m, int(i), ep, stream=server)
+            total_posts += 1
+        copies = []
+        for i in range(n):
+            api.asap_moe_mailbox_wait(m, i, stream=consumer)
+            with torch.cuda.stream(consumer):
+                copies.append(outs[i].clone())
+        torch.cuda.synchronize()
+        for a, b, cp in zip(c.ref, outs, copies):
+            assert same_bits(a, b) and same_bits(a, cp)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == total_posts and sum(claimed) == total_posts
+    print(f"[{cfg.name}] posts per round: {claimed}")
+    assert_clean(c.h)
+    m.close()
+
+
+def test_mailbox_output_against_oracle():
+    """The chain to the oracle directly: one round serving three posts of the
+    DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
+    whose routing the float32 logits decide."""
+    c = Case.get(DS)
+    cfg = c.cfg
+    m = api.asap_moe_mailbox_create(c.h, 3, max(cfg.microbatches))
+    outs = [torch.empty_like(x) for x in c.xs[:3]]
+    eps = [api.asap_moe_mailbox_post(m, i, c.xs[i], outs[i]) for i in range(3)]
+    api.asap_moe_mailbox_serve(m, 2, eps[2])
+    torch.cuda.synchronize()
+    assert api.asap_moe_mailbox_rounds(m) == (1, [3])
+    wf = {k: bf16_to_f64(c.w[k]) for k in ("router_w", "w_gate", "w_up", "w_down", "sh_gate", "sh_up", "sh_down")}
+    ocfg = cfg.oracle_cfg()
+    for x, o in zip(c.xs[:3], outs):
+        xf = bf16_to_f64(x)
+        r = oracle.moe_layer(xf, wf["router_w"], wf["w_gate"], wf["w_up"], wf["w_down"], ocfg,
+                             shared=(wf["sh_gate"], wf["sh_up"], wf["sh_down"]))
+        eps_l = oracle.logit_error_bound(xf, wf["router_w"])
+        keep = np.array([oracle.token_decided(r["logits"][t], eps_l[t], ocfg) for t in range(x.shape[0])])
+        compare_rows(bf16_to_f64(o)[keep], r["y"][keep])
+    assert_clean(c.h)
+    m.close()
+
+
+def test_round_for_a_post_never_made_times_out_and_serves_the_rest():
+    """A serve call for a post that nothing publishes (epoch 1 of an unused
+    slot): the round's wait runs out after wait_ns, records status bit 128,
+    and the round still serves the post that is ready."""
+    c = Case.get(DS)
+    m = api.asap_moe_mailbox_create(c.h, 2, max(DS.microbatches), wait_ns=20_000_000)
+    out = torch.empty_like(c.xs[0])
+    ep = api.asap_moe_mailbox_post(m, 0, c.xs[0], out)
+    torch.cuda.synchronize()
+    api.asap_moe_mailbox_serve(m, 1, 1)          # slot 1 is never posted
+    torch.cuda.synchronize()
+    assert same_bits(c.ref[0], out)
+    assert api.asap_moe_mailbox_served(m, 0) == ep and api.asap_moe_mailbox_served(m, 1) == 0
+    word = assert_clean(c.h, allowed=ST_MBOX_WAIT)
+    assert word == ST_MBOX_WAIT
+    # the mailbox is still usable: slot 0 again, then its own round
+    api.asap_moe_mailbox_serve(m, 0, ep)
+    out2 = torch.empty_like(c.xs[1])
+    ep2 = api.asap_moe_mailbox_post(m, 0, c.xs[1], out2)
+    api.asap_moe_mailbox_serve(m, 0, ep2)
+    torch.cuda.synchronize()
+    assert same_bits(c.ref[1], out2)
+    assert api.asap_moe_mailbox_rounds(m) == (3, [1, 0, 1])
+    assert_clean(c.h)
+    m.close()
+
+
+def test_host_side_rules():
+    c = Case.get(DS)
+    m = api.asap_moe_mailbox_create(c.h, 2, 1000)
+    out = torch.empty_like(c.xs[0])
+    ep = api.asap_moe_mailbox_post(m, 0, c.xs[0], out)
+    with pytest.raises(AsapError, match="no serve call"):
+        api.asap_moe_mailbox_post(m, 0, c.xs[0], out)          # backpressure: not served yet
+    with pytest.raises(AsapError, match="no serve call"):
+        api.asap_moe_mailbox_wait(m, 0)
+    with pytest.raises(AsapError, match="slot outside"):
+        api.asap_moe_mailbox_post(m, 2, c.xs[0], out)
+    big = inputs.make_tokens(DS, 1001, 9, DEV)
+    with pytest.raises(AsapError, match="slot_tokens"):
+        api.asap_moe_mailbox_post(m, 1, big, torch.empty_like(big))
+    api.asap_moe_mailbox_serve(m, 0, ep)
+    api.asap_moe_mailbox_wait(m, 0)
+    torch.cuda.synchronize()
+    assert same_bits(c.ref[0], out)
+    empty = torch.empty((0, DS.hidden), dtype=torch.bfloat16, device=DEV)
+    ep0 = api.asap_moe_mailbox_post(m, 1, empty, empty)        # an empty post is served too
+    api.asap_moe_mailbox_serve(m, 1, ep0)
+    torch.cuda.synchronize()
+    assert api.asap_moe_mailbox_served(m, 1) == ep0
+    with pytest.raises(AsapError, match="n_slots"):
+        api.asap_moe_mailbox_create(c.h, 65, 100)
+    assert_clean(c.h)
+    m.close()
+
+
+def test_mailbox_on_a_layer_of_a_multi_layer_handle():
+    cfg = inputs.small_variant(DSV3, name="mbox_layers", hidden=512, inter=256, shared_inter=256,
+                               microbatches=[300, 77])
+    ws = inputs.make_layer_weights(cfg, 2, DEV)
+    h = api.asap_moe_create_layers(cfg, ws, 300)
+    one = api.asap_moe_create(inputs.layer_config(cfg, 1), ws[1], 300)
+    lid = torch.tensor([1], dtype=torch.int32, device=DEV)
+    m = api.asap_moe_mailbox_create(h, 2, 300, layer_id=lid)
+    xs = inputs.make_microbatches(cfg, DEV)
+    outs = [torch.empty_like(x) for x in xs]
+    eps = [api.asap_moe_mailbox_post(m, i, x, o) for i, (x, o) in enumerate(zip(xs, outs))]
+    api.asap_moe_mailbox_serve(m, 0, eps[0])
+    api.asap_moe_mailbox_serve(m, 1, eps[1])
+    for x, o in zip(xs, outs):
+        ref = torch.empty_like(x)
+        api.asap_moe_layer(one, x, ref, api.workspace(one, x.shape[0]))
+        torch.cuda.synchronize()
+        assert same_bits(ref, o)
+    assert_clean(h)
+    m.close()
+    h.close()
+    one.close()
