@@ -47,6 +47,7 @@ def parse_args():
     ap.add_argument("--workload", default="dsv3_bf16")
     ap.add_argument("--kernel-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-mailbox", action="store_true", help="skip the mailbox (device-side ready set) leg")
     ap.add_argument("--cpu-sample-tokens", type=int, default=12)
     ap.add_argument("--microbatches", default=None,
                     help="comma-separated micro-batch sizes overriding the workload's")
@@ -357,6 +358,15 @@ def run_ours(args, dist):
     # ---------------- all micro-batches in one pass (one grouped GEMM per weight matrix)
     result["aggregated"] = aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist)
 
+    # ---------------- the device decides the sets: mailbox posts and service rounds
+    if not args.no_mailbox:
+        result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist)
+
+    # ---------------- per-micro-batch latency of the per-stream step
+    result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
+    if cfg.zipf_s is not None:
+        result["expert_popularity"] = popularity(h, cfg, xs, dev)
+
     # ---------------- end to end through host buffers
     result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
 
@@ -585,6 +595,167 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
                 "grouped_gemm_frac_of_sustained_measured": tf / peaks["bf16_tflops_sustained"],
                 "weight_gb_per_step": wbytes / 1e9})
     return res
+
+
+def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist):
+    """The step's micro-batches posted into a mailbox, each from its own
+    stream, and served by rounds on one MoE stream: the host serves every post
+    right after making it (no host batching), and each round claims on the
+    device every post published by the time it starts, serving all of them
+    with one grouped GEMM pass.  Slots are double-buffered across steps.
+    Outputs are bit-identical to asap_moe_layer's (tested).  Reports the
+    step rate, how the device grouped the posts, and the grouped GEMMs'
+    tensor fraction (algorithmic FLOPs of the step over the event-timed GEMMs
+    of its rounds)."""
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    n_mb = len(xs)
+    m = api.asap_moe_mailbox_create(h, 2 * n_mb, max(x.shape[0] for x in xs))
+    producers = [torch.cuda.Stream() for _ in xs]
+    server = torch.cuda.Stream()
+    main = torch.cuda.current_stream()
+    outs = [[torch.empty_like(x) for x in xs] for _ in range(2)]
+
+    def step(si, gemm_events=None):
+        b = si % 2
+        ev = torch.cuda.Event()
+        ev.record(main)
+        eps = []
+        for i, (x, p) in enumerate(zip(xs, producers)):
+            p.wait_event(ev)
+            eps.append(api.asap_moe_mailbox_post(m, b * n_mb + i, x, outs[b][i], stream=p))
+        for i in range(n_mb):
+            if gemm_events is not None:
+                api.asap_moe_mailbox_time_gemms(m, *gemm_events[i])
+            api.asap_moe_mailbox_serve(m, b * n_mb + i, eps[i], stream=server)
+        for i in range(n_mb):
+            api.asap_moe_mailbox_wait(m, b * n_mb + i, stream=main)
+
+    for si in range(args.warmup):
+        step(si)
+    torch.cuda.synchronize()
+    r0, _ = api.asap_moe_mailbox_rounds(m)
+    dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(main)
+    for si in range(args.steps):
+        step(args.warmup + si)
+    b.record(main)
+    torch.cuda.synchronize()
+    ms = dist.max(a.elapsed_time(b)) / args.steps
+    r1, claimed = api.asap_moe_mailbox_rounds(m)
+    sizes = claimed[r0:r1]
+    # the GEMMs of every round, timed with events on the MoE stream
+    gemm_ms = []
+    nonempty = []
+    base = args.warmup + args.steps
+    for si in range(args.kernel_steps):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_mb)]
+        rb, _ = api.asap_moe_mailbox_rounds(m)
+        step(base + si, evs)
+        torch.cuda.synchronize()
+        ra, cl = api.asap_moe_mailbox_rounds(m)
+        gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in evs))
+        nonempty.append(sum(1 for c in cl[rb:ra] if c > 0))
+    api.asap_moe_mailbox_rounds(m)
+    code, word = api.asap_moe_status(h)
+    m.close()
+    if code != 0:
+        raise RuntimeError(f"device status word {word:#x} after the mailbox leg")
+    flops = kern["gemm_flops"] * n_mb    # per micro-batch mean x micro-batches
+    g = sum(gemm_ms) / len(gemm_ms)
+    tf = flops / (g / 1e3) / 1e12
+    tpk_burst = 2.0 * peaks["bf16_tflops"] if tensor_peak else peaks["bf16_tflops"]
+    tpk_sus = tensor_peak or peaks["bf16_tflops_sustained"]
+    hist = {}
+    for c in sizes:
+        hist[str(c)] = hist.get(str(c), 0) + 1
+    n_tok = sum(x.shape[0] for x in xs)
+    return {"value": dist.world * n_tok / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms,
+            "rounds_per_step": (r1 - r0) / args.steps,
+            "nonempty_rounds_per_step": sum(1 for c in sizes if c > 0) / args.steps,
+            "posts_per_nonempty_round": (sum(sizes) / max(1, sum(1 for c in sizes if c > 0))),
+            "round_sizes_histogram": hist,
+            "grouped_gemm_ms_per_step": g, "grouped_gemm_tflops": tf,
+            "grouped_gemm_frac_of_burst_measured": tf / tpk_burst,
+            "grouped_gemm_frac_of_sustained_measured": tf / tpk_sus,
+            "gemm_timing_nonempty_rounds_per_step": sum(nonempty) / len(nonempty),
+            "note": "asap_moe_mailbox_post from one stream per micro-batch, asap_moe_mailbox_serve for every post "
+                    "right after it on one MoE stream; the rounds claim on the device whatever has been published"}
+
+
+def latency_pass(args, h, xs, outs, wss, streams, main):
+    """Per-micro-batch latency of the per-stream step: CUDA events from the
+    step's first submission (every stream waits on it) to each micro-batch's
+    completion on its own stream; the aggregate rate is the step's tokens
+    over the span to the last completion."""
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    lat = [[] for _ in xs]
+    spans = []
+    for it in range(args.kernel_steps + 1):
+        ev0 = torch.cuda.Event(enable_timing=True)
+        ends = [torch.cuda.Event(enable_timing=True) for _ in xs]
+        ev0.record(main)
+        for x, o, ws, s, e in zip(xs, outs, wss, streams, ends):
+            s.wait_event(ev0)
+            api.asap_moe_layer(h, x, o, ws, stream=s)
+            e.record(s)
+        for s in streams:
+            main.wait_stream(s)
+        torch.cuda.synchronize()
+        if it == 0:
+            continue
+        t = [ev0.elapsed_time(e) for e in ends]
+        for i, v in enumerate(t):
+            lat[i].append(v)
+        spans.append(max(t))
+    n_tok = sum(x.shape[0] for x in xs)
+    span = sum(spans) / len(spans)
+    return {"per_microbatch_ms": [sum(v) / len(v) for v in lat],
+            "microbatch_tokens": [x.shape[0] for x in xs],
+            "first_submit_to_last_complete_ms": span,
+            "aggregate_tokens_per_s": n_tok / (span / 1e3),
+            "note": "CUDA events: step start on the submitting stream -> each micro-batch's completion on its own "
+                    "stream, mean over the kernel steps"}
+
+
+def popularity(h, cfg, xs, dev):
+    """Realised expert popularity of a Zipf-biased workload: each expert's
+    share of the routed (token, slot) pairs over all micro-batches, ranked,
+    beside the Zipf target p_r ~ r^-s; and the exponent fitted to the
+    realised shares of ranks 2..64 by least squares in log-log."""
+    import numpy as np
+    import torch
+    from paper_2606_22541_gb300 import api
+
+    E, k = cfg.n_experts, cfg.top_k
+    tot = np.zeros(E, np.int64)
+    active = []
+    for x in xs:
+        n = x.shape[0]
+        idx = torch.empty((n, k), dtype=torch.int32, device=dev)
+        w = torch.empty((n, k), dtype=torch.float32, device=dev)
+        counts = torch.empty(E, dtype=torch.int32, device=dev)
+        offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+        api.asap_moe_route(h, x, idx, w, counts, offsets, api.workspace(h, n, dev))
+        c = counts.cpu().numpy().astype(np.int64)
+        tot += c
+        active.append(int((c > 0).sum()))
+    share = np.sort(tot)[::-1] / tot.sum()
+    r = np.arange(1, E + 1, dtype=np.float64)
+    target = r ** -cfg.zipf_s
+    target /= target.sum()
+    sel = slice(1, 64)
+    fit = -np.polyfit(np.log(r[sel]), np.log(np.maximum(share[sel], 1e-12)), 1)[0]
+    return {"zipf_s": cfg.zipf_s, "realised_top8_share": [float(v) for v in share[:8]],
+            "zipf_target_top8_share": [float(v) for v in target[:8]],
+            "fitted_exponent_ranks_2_64": float(fit), "experts_with_tokens_total": int((tot > 0).sum()),
+            "active_experts_per_microbatch": active,
+            "note": "share of the routed (token, slot) pairs; with top-8 one expert holds at most 1/8"}
 
 
 def e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist):

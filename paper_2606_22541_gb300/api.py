@@ -277,7 +277,11 @@ def asap_moe_mailbox_served(m, slot):
 
 
 def asap_moe_mailbox_time_gemms(m, ev_before, ev_after):
-    """torch.cuda.Event pair recorded around the next serve call's GEMMs."""
+    """torch.cuda.Event pair (enable_timing=True) recorded around the next
+    serve call's GEMMs."""
+    for ev in (ev_before, ev_after):
+        if ev.cuda_event == 0:   # torch creates the CUDA event at its first record
+            ev.record()
     check("asap_moe_mailbox_time_gemms",
           lib().asap_moe_mailbox_time_gemms(m.ptr, ctypes.c_void_p(ev_before.cuda_event),
                                             ctypes.c_void_p(ev_after.cuda_event)))
