@@ -11,9 +11,11 @@ Recipe (every workload):
   Wg, Wu ~ N(0, 1/sqrt(H)), Wd ~ N(0, 1/sqrt(I)) (std = 1/sqrt(fan_in)), bf16
   router Wr ~ N(0, 0.02) for the tiny layer, N(0, 1/sqrt(H)) otherwise
   shared expert like a routed one with I_s
-  Zipf popularity (skewed workloads): channel 0 of every token is set to 1 and
-  router column 0 to ln p_{pi(e)} - mean, p_r ~ r^-s, pi a seeded expert
-  permutation, so logit e carries a bias ln p_{pi(e)}.
+  Zipf popularity (skewed workloads): channel 0 of every token is set to 1
+  (the rest stays N(0, 1)) and router column 0 to beta (ln p_{pi(e)} - mean),
+  p_r ~ r^-s, pi a seeded expert permutation, so logit e carries a bias
+  beta ln p_{pi(e)}; beta = cfg.zipf_beta, calibrated on the realised expert
+  shares (zipf_calibrate.py).
   FP8: weights drawn as above in fp32, then per 128 x 128 block
   s = amax/448, q = e4m3(w / s) (torch's round-to-nearest-even cast).
 Seeds: torch generator on the target device, seed = cfg.seed * 1000 + tensor id.
@@ -135,7 +137,8 @@ def router_weights_bf16(cfg, device):
     r_std = 0.02 if cfg.name == "tiny" else 1.0 / np.sqrt(H)
     wr = randn_bf16((E, H), r_std, cfg.seed * 1000 + 1, device)
     if cfg.zipf_s is not None:
-        b = torch.tensor(zipf_logit_bias(E, cfg.zipf_s, cfg.seed), dtype=torch.float32, device=device)
+        b = torch.tensor(cfg.zipf_beta * zipf_logit_bias(E, cfg.zipf_s, cfg.seed), dtype=torch.float32,
+                         device=device)
         wr[:, 0] = b.to(torch.bfloat16)
     return wr
 

@@ -237,3 +237,42 @@ def test_mailbox_on_a_layer_of_a_multi_layer_handle():
     m.close()
     h.close()
     one.close()
+
+
+def test_mailbox_full_size_dsv3():
+    """The bench's workload: 4 x 4096 DeepSeek-V3 tokens posted from four
+    streams, every post served right after it on one MoE stream, twice (the
+    second time the slots are reposted): every output bit-identical to
+    asap_moe_layer on the same micro-batch."""
+    cfg = DSV3
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
+    del w
+    torch.cuda.empty_cache()
+    xs = inputs.make_microbatches(cfg, DEV)
+    ref = []
+    ws = api.workspace(h, max(cfg.microbatches))
+    for x in xs:
+        o = torch.empty_like(x)
+        api.asap_moe_layer(h, x, o, ws)
+        ref.append(o)
+    torch.cuda.synchronize()
+    del ws
+    m = api.asap_moe_mailbox_create(h, len(xs), max(cfg.microbatches))
+    producers = [torch.cuda.Stream() for _ in xs]
+    server = torch.cuda.Stream()
+    for rep in range(2):
+        outs = [torch.full_like(x, 5.0) for x in xs]
+        eps = [api.asap_moe_mailbox_post(m, i, x, o, stream=p)
+               for i, (x, o, p) in enumerate(zip(xs, outs, producers))]
+        for i, ep in enumerate(eps):
+            api.asap_moe_mailbox_serve(m, i, ep, stream=server)
+        torch.cuda.synchronize()
+        for a, b in zip(ref, outs):
+            assert same_bits(a, b)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == 2 * len(xs) and sum(claimed) == 2 * len(xs)
+    print(f"[dsv3 full size] posts per round: {claimed}")
+    assert_clean(h)
+    m.close()
+    h.close()

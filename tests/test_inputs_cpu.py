@@ -95,8 +95,9 @@ def test_zipf_workload_plants_the_bias_in_channel_0():
     x = inputs.make_tokens(cfg, 32, 0, CPU)
     assert torch.all(x[:, 0] == 1.0)
     wr = inputs.router_weights_bf16(cfg, CPU)
-    b = torch.tensor(inputs.zipf_logit_bias(16, cfg.zipf_s, cfg.seed)).to(torch.bfloat16)
+    b = torch.tensor(cfg.zipf_beta * inputs.zipf_logit_bias(16, cfg.zipf_s, cfg.seed)).to(torch.bfloat16)
     assert torch.equal(wr[:, 0], b)
+    assert 0.0 < cfg.zipf_beta < 1.0
 
 
 def test_layer_seeds():
