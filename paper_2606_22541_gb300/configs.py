@@ -33,10 +33,10 @@ class LayerConfig:
     # strength of the Zipf logit bias: logit e carries zipf_beta * ln p_pi(e).
     # Calibrated so that the realised shares of the routed (token, slot) pairs
     # follow r^-zipf_s: the exponent fitted to ranks 2..64 of the stress
-    # workload's routing on a GB300 is 1.069 at 0.60, 1.119 at 0.63 and 1.754
-    # at 1.0 and 1.104 at 0.62 (python -m paper_2606_22541_gb300.zipf_calibrate);
-    # the top ranks stay below Zipf's because top-8 routing caps
-    # one expert at 1/8 of the pairs.
+    # workload's routing on a GB300 is 1.069 at 0.60, 1.104 at 0.62, 1.119 at
+    # 0.63 and 1.754 at 1.0 (python -m paper_2606_22541_gb300.zipf_calibrate);
+    # the top ranks stay below Zipf's because top-8 routing caps one expert at
+    # 1/8 of the pairs.
     zipf_beta: float = 0.62
     seed: int = 1000
 
