@@ -276,3 +276,50 @@ def test_mailbox_full_size_dsv3():
     assert_clean(h)
     m.close()
     h.close()
+
+
+def test_posts_and_rounds_from_host_threads():
+    """One host thread per DP group posting on its own stream and a server
+    thread serving each post as it learns of it (through a queue): the
+    mailbox's host state is shared between threads behind its lock; every
+    output still equals asap_moe_layer's."""
+    import queue
+    import threading
+    c = Case.get(DS)
+    n = len(c.xs)
+    m = api.asap_moe_mailbox_create(c.h, n, max(DS.microbatches))
+    outs = [[torch.full_like(x, 9.0) for x in c.xs] for _ in range(2)]
+    q = queue.Queue()
+    errors = []
+
+    def producer(i):
+        try:
+            s = torch.cuda.Stream()
+            for rep in range(2):
+                if rep:
+                    done[i].wait(timeout=30)
+                    api.asap_moe_mailbox_wait(m, i, stream=s)
+                q.put((i, api.asap_moe_mailbox_post(m, i, c.xs[i], outs[rep][i], stream=s)))
+        except Exception as e:   # reported by the main thread
+            errors.append(e)
+
+    done = [threading.Event() for _ in range(n)]
+    server = torch.cuda.Stream()
+    threads = [threading.Thread(target=producer, args=(i,)) for i in range(n)]
+    for t in threads:
+        t.start()
+    for _ in range(2 * n):
+        i, ep = q.get(timeout=60)
+        api.asap_moe_mailbox_serve(m, i, ep, stream=server)
+        done[i].set()
+    for t in threads:
+        t.join(timeout=60)
+    torch.cuda.synchronize()
+    assert not errors, errors
+    for rep in range(2):
+        for a, b in zip(c.ref, outs[rep]):
+            assert same_bits(a, b)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == 2 * n and sum(claimed) == 2 * n
+    assert_clean(c.h)
+    m.close()
