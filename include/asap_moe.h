@@ -394,16 +394,22 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
  *    backpressure of Section 3.2.1).
  *  - x and out of a post must stay valid until the post is served.
  *
- * One mailbox serves one layer (layer_id, or layer 0) of its handle and owns
- * its memory: a server workspace for n_slots * slot_tokens tokens
- * (asap_moe_workspace_size of that many tokens) and a few KB of state.
+ * Layers: each post belongs to one MoE layer of the handle (a device int32
+ * layer id read when the post is published; see asap_moe_layer_dyn).  A round
+ * claims only posts of the layer of the post it was started for, and its
+ * grouped GEMMs read that layer's weights, so one mailbox serves every layer
+ * of a multi-layer handle, in whatever order the layers' posts arrive
+ * (Section 3.4.2); posts of other layers wait for a round of their own.
+ *
+ * A mailbox owns its memory: a server workspace for n_slots * slot_tokens
+ * tokens (asap_moe_workspace_size of that many tokens) and a few KB of state.
  * Calls are thread-safe with respect to each other (one lock per mailbox).
  * ------------------------------------------------------------------------ */
 typedef struct asap_moe_mailbox_s* asap_moe_mailbox_t;
 
 /* Create a mailbox of n_slots slots (1..64) of up to slot_tokens tokens
- * (<= max_tokens) each on h's device.  layer_id: NULL (layer 0) or a 4-byte
- * aligned device int32 read by the kernels when they run.  wait_ns > 0:
+ * (<= max_tokens) each on h's device.  layer_id: the layer of posts made
+ * without one, NULL (layer 0) or a 4-byte aligned device int32.  wait_ns > 0:
  * the limit of a round's wait for a post that has not been published.
  * Allocates; synchronous. */
 int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot_tokens,
@@ -412,12 +418,14 @@ int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot_tokens,
 /* Free the mailbox (synchronises the device first).  NULL is accepted. */
 int asap_moe_mailbox_destroy(asap_moe_mailbox_t m);
 
-/* Post n tokens of x (0 <= n <= slot_tokens) into slot on stream: waits on
- * the stream for the slot's previous round, routes, publishes.  *epoch
- * (nullable) receives the post's epoch (1, 2, ... per slot), the value to
- * serve it with.  Enqueues only. */
+/* Post n tokens of x (0 <= n <= slot_tokens) of the layer at layer_id
+ * (NULL: the mailbox's default layer; a device int32 read when the post's
+ * kernels run, rules of asap_moe_layer_dyn) into slot on stream: waits on the
+ * stream for the slot's previous round, routes with that layer's router,
+ * publishes.  *epoch (nullable) receives the post's epoch (1, 2, ... per
+ * slot), the value to serve it with.  Enqueues only. */
 int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int32_t n,
-                          void* out, void* stream, uint64_t* epoch);
+                          void* out, const int32_t* layer_id, void* stream, uint64_t* epoch);
 
 /* One service round on stream for post epoch of slot, as described above.
  * Enqueues only. */

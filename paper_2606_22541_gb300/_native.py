@@ -62,7 +62,7 @@ SIGNATURES = {
     "asap_moe_set_tiling": [_P, _I],
     "asap_moe_mailbox_create": [_P, _I, _I, _P, ctypes.c_int64, ctypes.POINTER(_P)],
     "asap_moe_mailbox_destroy": [_P],
-    "asap_moe_mailbox_post": [_P, _I, _P, _I, _P, _P, ctypes.POINTER(ctypes.c_uint64)],
+    "asap_moe_mailbox_post": [_P, _I, _P, _I, _P, _P, _P, ctypes.POINTER(ctypes.c_uint64)],
     "asap_moe_mailbox_serve": [_P, _I, ctypes.c_uint64, _P],
     "asap_moe_mailbox_wait": [_P, _I, _P],
     "asap_moe_mailbox_served": [_P, _I, ctypes.POINTER(ctypes.c_uint64)],

@@ -252,13 +252,16 @@ def asap_moe_mailbox_create(h, n_slots, slot_tokens, layer_id=None, wait_ns=2_00
     return m
 
 
-def asap_moe_mailbox_post(m, slot, x, out, stream=None):
-    """Post x (n tokens) into slot; returns the post's epoch."""
+def asap_moe_mailbox_post(m, slot, x, out, stream=None, layer_id=None):
+    """Post x (n tokens) into slot; returns the post's epoch.  layer_id: None
+    (the mailbox's default layer) or a one-element int32 CUDA tensor.  x, out
+    and layer_id must stay alive until the post is served; the mailbox keeps a
+    reference to the slot's last post."""
     ep = ctypes.c_uint64()
     check("asap_moe_mailbox_post",
-          lib().asap_moe_mailbox_post(m.ptr, int(slot), _ptr(x), x.shape[0], _ptr(out), _stream(stream),
-                                      ctypes.byref(ep)))
-    m._keep[int(slot)] = (x, out)
+          lib().asap_moe_mailbox_post(m.ptr, int(slot), _ptr(x), x.shape[0], _ptr(out), _ptr(layer_id),
+                                      _stream(stream), ctypes.byref(ep)))
+    m._keep[int(slot)] = (x, out, layer_id)
     return ep.value
 
 

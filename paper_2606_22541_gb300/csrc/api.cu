@@ -1237,7 +1237,7 @@ ASAP_API int asap_moe_status(asap_moe_t h, uint32_t* word) {
 struct asap_moe_mailbox_s {
   asap_moe_t h = nullptr;
   asap::MboxGeom g{};
-  const int32_t* layer = nullptr;  // device layer id of the posts
+  const int32_t* layer = nullptr;  // device layer id of posts made without one
   unsigned long long wait_ns = 0;
   Layout L{};                      // server workspace: layout for n_slots * slot_tokens tokens
   void* ws = nullptr;
@@ -1345,8 +1345,11 @@ ASAP_API int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot
 ASAP_API int asap_moe_mailbox_destroy(asap_moe_mailbox_t m) { return mbox_free(m); }
 
 ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int32_t n, void* out,
-                                   void* stream, uint64_t* epoch) {
+                                   const int32_t* layer_id, void* stream, uint64_t* epoch) {
   if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  if (layer_id && !valid_layer_ptr(layer_id))
+    return fail(ASAP_ERR_INVALID, "layer_id must be NULL or a 4-byte aligned device pointer");
+  const int32_t* layer = layer_id ? layer_id : m->layer;
   asap_moe_t h = m->h;
   const asap_moe_config& c = h->cfg;
   if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
@@ -1374,19 +1377,19 @@ ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const voi
     // are the slot's, scanned later together with the other claimed posts
     if (fused_route(h)) {
       if ((r = run_route_fused(h, x, n, idx, w, hist, chunk0, chunks_total, nullptr, nullptr, nullptr, nullptr,
-                               nullptr, m->layer, st)) != ASAP_OK)
+                               nullptr, layer, st)) != ASAP_OK)
         return r;
     } else {
       const int splits = router_splits(h, n);
       float* lg = at<float>(m->ws, m->L.logits) +
                   static_cast<long long>(slot) * asap::kMaxRouterSplits * g.slot_tokens * c.n_experts;
-      if ((r = run_router_logits(h, x, n, lg, splits, m->layer, st)) != ASAP_OK) return r;
-      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, m->layer, nullptr), idx, w, hist, chunk0,
+      if ((r = run_router_logits(h, x, n, lg, splits, layer, st)) != ASAP_OK) return r;
+      CU_TRY(asap::launch_gate_seg(lg, splits, n, gate_params(h, layer, nullptr), idx, w, hist, chunk0,
                                    chunks_total, st),
              "gate launch");
     }
   }
-  CU_TRY(asap::launch_mbox_publish(m->slots, slot, x, n, out, ep, h->status, st), "publish launch");
+  CU_TRY(asap::launch_mbox_publish(m->slots, slot, x, n, out, layer, ep, h->status, st), "publish launch");
   CU_TRY(cudaEventRecord(m->post_ev[slot], st), "post event");
   m->posted[slot] = ep;
   if (epoch) *epoch = ep;
@@ -1409,6 +1412,7 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
   int32_t* offsets = at<int32_t>(ws, L.offsets);
   int32_t* counters = at<int32_t>(ws, L.tile_counters);
   const int32_t* n_total = &m->round->n_total;
+  const int32_t* layer = &m->round->layer;  // the layer of the claimed posts, written by the claim
   int r;
   // the post this round is for was published before the round starts
   CU_TRY(cudaStreamWaitEvent(st, m->post_ev[slot], 0), "wait for the post");
@@ -1432,12 +1436,12 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
            "dispatch launch");
     if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, N, at<void>(ws, L.hq),
-                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), m->layer, counters,
+                             at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), layer, counters,
                              st, n_total)) != ASAP_OK)
       return r;
     y_perm = at<void>(ws, L.y_perm);
     if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
-                          at<float>(ws, L.hs_sh), N, y_perm, y_sh, m->layer, counters + 1, st, n_total)) != ASAP_OK)
+                          at<float>(ws, L.hs_sh), N, y_perm, y_sh, layer, counters + 1, st, n_total)) != ASAP_OK)
       return r;
   } else {
     // the shared expert reads the gathered rows from y_sh's region, which its
@@ -1447,10 +1451,10 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
                                       at<int32_t>(ws, L.perm_src), perm_dst, y_sh, h->status, st),
            "dispatch launch");
     if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
-    if ((r = run_gate_up(h, y_perm, offsets, y_sh, N, at<void>(ws, L.h), at<void>(ws, L.h_sh), m->layer, counters, st,
+    if ((r = run_gate_up(h, y_perm, offsets, y_sh, N, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer, counters, st,
                          n_total)) != ASAP_OK)
       return r;
-    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), N, y_perm, y_sh, m->layer, counters + 1,
+    if ((r = run_down(h, at<void>(ws, L.h), offsets, at<void>(ws, L.h_sh), N, y_perm, y_sh, layer, counters + 1,
                       st, n_total)) != ASAP_OK)
       return r;
   }

@@ -242,7 +242,7 @@ struct MboxSlot {            // one per slot, device memory
   const void* x;              // the post's hidden states [n, H]
   void* out;                  // its layer output [n, H]
   int n;
-  int pad_;
+  int layer;                  // the MoE layer the post belongs to (its id when it was published)
 };
 
 struct MboxRound {           // the set the current service round claimed (its claim kernel writes it)
@@ -250,6 +250,7 @@ struct MboxRound {           // the set the current service round claimed (its c
   int n_total;               // their tokens: rows of the shared expert's input
   int chunks_total;          // their histogram rows (rowmap entries)
   int rounds;                // service rounds run so far, this one included
+  int layer;                 // the layer every claimed post belongs to (the GEMMs read its weights)
   int slot[kMboxMaxSlots];   // claimed slots, increasing
   int n[kMboxMaxSlots];
   int tok0[kMboxMaxSlots];   // first token in the round's combined token order
@@ -267,14 +268,17 @@ struct MboxGeom {
   int k, E, H;
 };
 
-// Producer: publish a post (after its routing on the same stream).  Records
-// ST_MBOX_OVERRUN when the slot's previous post has not been served.
-cudaError_t launch_mbox_publish(MboxSlot* slots, int slot, const void* x, int n, void* out,
+// Producer: publish a post (after its routing on the same stream) of the
+// layer whose id is *layer.  Records ST_MBOX_OVERRUN when the slot's previous
+// post has not been served.
+cudaError_t launch_mbox_publish(MboxSlot* slots, int slot, const void* x, int n, void* out, const int32_t* layer,
                                 unsigned long long epoch, uint32_t* status, cudaStream_t s);
 // Service round, step 1: wait (at most wait_ns) until slot own_slot has
 // published epoch own_epoch (own_slot < 0: no wait; a wait that runs out
-// records ST_MBOX_WAIT), then claim every slot with posted > served into *r,
-// write the histogram row map, zero the scan's ticket.
+// records ST_MBOX_WAIT), then claim every slot with posted > served whose post
+// belongs to the same layer as that post (after a wait that ran out: as the
+// lowest pending slot's post) into *r, write the histogram row map, zero the
+// scan's ticket.
 cudaError_t launch_mbox_claim(MboxSlot* slots, MboxGeom g, int own_slot, unsigned long long own_epoch,
                               unsigned long long wait_ns, MboxRound* r, int32_t* rowmap, int32_t* ticket,
                               uint32_t* status, cudaStream_t s);

@@ -7,9 +7,12 @@
 //    the publish kernel sets the slot's ready flag, an epoch, with a release
 //    store (the "bitmap" of region 3 of Table 2).
 //  - A service round's claim kernel polls every slot's flag once and claims
-//    every post that is ready and not yet served (async-dispatch-recv): the
-//    MoE side serves whatever has arrived, in slot order, without waiting for
-//    the others.
+//    every post that is ready and not yet served and belongs to the same MoE
+//    layer as the post the round was started for (async-dispatch-recv): the
+//    MoE side serves whatever has arrived for that layer, in slot order,
+//    without waiting for the others; the grouped GEMMs read the layer's
+//    weights at the id the claim wrote (the layer-oblivious kernels of
+//    Section 3.4.2), so layers are served in whatever order their posts come.
 //  - After the round's grouped GEMMs and combine, the finish kernel sets each
 //    claimed slot's completion flag (async-combine-send; also written to
 //    host-mapped memory, which the attention side can poll).
@@ -41,7 +44,7 @@ __device__ __forceinline__ void st_release_sys_u64(unsigned long long* p, unsign
 
 // One thread: the slot's descriptor, then its ready epoch (release).
 __global__ void mbox_publish_kernel(MboxSlot* slots, int slot, const void* x, int n, void* out,
-                                    unsigned long long epoch, uint32_t* status) {
+                                    const int32_t* layer, unsigned long long epoch, uint32_t* status) {
   if (threadIdx.x != 0) return;
   MboxSlot* m = slots + slot;
   // the previous post of this slot must have been served (the host makes the
@@ -50,6 +53,7 @@ __global__ void mbox_publish_kernel(MboxSlot* slots, int slot, const void* x, in
   m->x = x;
   m->out = out;
   m->n = n;
+  m->layer = *reinterpret_cast<const volatile int32_t*>(layer);
   __threadfence();
   st_release_gpu_u64(&m->posted, epoch);
 }
@@ -61,24 +65,42 @@ __global__ void __launch_bounds__(kMboxMaxSlots) mbox_claim_kernel(MboxSlot* slo
                                                                    int32_t* rowmap, int32_t* ticket,
                                                                    uint32_t* status) {
   __shared__ int s_cnt[2], s_tok[2], s_chk[2];
+  __shared__ int s_layer, s_first;
   const int s = threadIdx.x, lane = s & 31, warp = s >> 5;
-  if (s == 0 && own_slot >= 0) {
-    const uint64_t t0 = globaltimer_ns();
-    while (ld_acquire_u64(&slots[own_slot].posted) < own_epoch) {
-      if (globaltimer_ns() - t0 > wait_ns) {
-        record_status(status, ST_MBOX_WAIT);
-        break;
+  if (s == 0) {
+    bool own = false;
+    if (own_slot >= 0) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!(own = ld_acquire_u64(&slots[own_slot].posted) >= own_epoch)) {
+        if (globaltimer_ns() - t0 > wait_ns) {
+          record_status(status, ST_MBOX_WAIT);
+          break;
+        }
+        __nanosleep(2000);
       }
-      __nanosleep(2000);
     }
+    // the round serves the layer of the post it was started for
+    s_layer = own ? slots[own_slot].layer : 0;
+    s_first = own ? -1 : kMboxMaxSlots;
   }
   __syncthreads();
   bool pend = false;
   unsigned long long posted = 0;
-  int n = 0;
   if (s < g.n_slots) {
     posted = ld_acquire_u64(&slots[s].posted);
     pend = posted > slots[s].served;  // served: written only by this stream's finish kernels
+  }
+  if (s_first >= 0) {
+    // no post to follow (its wait ran out): the layer of the lowest pending slot
+    if (pend) atomicMin(&s_first, s);
+    __syncthreads();
+    if (s == 0 && s_first < g.n_slots) s_layer = slots[s_first].layer;
+    __syncthreads();
+  }
+  const int layer = s_layer;
+  int n = 0;
+  if (pend) {
+    pend = slots[s].layer == layer;  // posts of other layers wait for a round of their own
     if (pend) n = min(max(slots[s].n, 0), g.slot_tokens);
   }
   const int ch = pend ? (n + kChunkTokens - 1) / kChunkTokens : 0;
@@ -119,6 +141,7 @@ __global__ void __launch_bounds__(kMboxMaxSlots) mbox_claim_kernel(MboxSlot* slo
     r->count = ic;
     r->n_total = it;
     r->chunks_total = ih;
+    r->layer = layer;
     r->rounds += 1;
     *ticket = 0;  // the scan that follows counts its CTAs on it
   }
@@ -144,9 +167,9 @@ __global__ void __launch_bounds__(kMboxMaxSlots) mbox_finish_kernel(MboxSlot* sl
 
 }  // namespace
 
-cudaError_t launch_mbox_publish(MboxSlot* slots, int slot, const void* x, int n, void* out,
+cudaError_t launch_mbox_publish(MboxSlot* slots, int slot, const void* x, int n, void* out, const int32_t* layer,
                                 unsigned long long epoch, uint32_t* status, cudaStream_t s) {
-  mbox_publish_kernel<<<1, 32, 0, s>>>(slots, slot, x, n, out, epoch, status);
+  mbox_publish_kernel<<<1, 32, 0, s>>>(slots, slot, x, n, out, layer, epoch, status);
   return cudaGetLastError();
 }
 

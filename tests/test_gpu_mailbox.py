@@ -215,6 +215,39 @@ def test_host_side_rules():
     m.close()
 
 
+def test_one_mailbox_serves_interleaved_layers():
+    """Posts of two layers of one handle interleaved in the slots: each round
+    claims only the ready posts of its own post's layer and runs that
+    layer's weights; every output equals a single-layer handle's."""
+    cfg = inputs.small_variant(DSV3, name="mbox_2layers", hidden=512, inter=256, shared_inter=256,
+                               microbatches=[300, 77, 129, 200])
+    ws = inputs.make_layer_weights(cfg, 2, DEV)
+    h = api.asap_moe_create_layers(cfg, ws, 300)
+    single = [api.asap_moe_create(inputs.layer_config(cfg, l), ws[l], 300) for l in range(2)]
+    ids = [torch.tensor([l], dtype=torch.int32, device=DEV) for l in range(2)]
+    layers = [0, 1, 0, 1]
+    m = api.asap_moe_mailbox_create(h, 4, 300)
+    xs = inputs.make_microbatches(cfg, DEV)
+    outs = [torch.empty_like(x) for x in xs]
+    eps = [api.asap_moe_mailbox_post(m, i, x, o, layer_id=ids[l])
+           for i, (x, o, l) in enumerate(zip(xs, outs, layers))]
+    torch.cuda.synchronize()
+    for i in (1, 0, 3, 2):                  # a layer-1 post first
+        api.asap_moe_mailbox_serve(m, i, eps[i])
+    torch.cuda.synchronize()
+    assert api.asap_moe_mailbox_rounds(m) == (4, [2, 2, 0, 0])
+    for x, o, l in zip(xs, outs, layers):
+        ref = torch.empty_like(x)
+        api.asap_moe_layer(single[l], x, ref, api.workspace(single[l], x.shape[0]))
+        torch.cuda.synchronize()
+        assert same_bits(ref, o)
+    assert_clean(h)
+    m.close()
+    h.close()
+    for one in single:
+        one.close()
+
+
 def test_mailbox_on_a_layer_of_a_multi_layer_handle():
     cfg = inputs.small_variant(DSV3, name="mbox_layers", hidden=512, inter=256, shared_inter=256,
                                microbatches=[300, 77])
@@ -323,3 +356,39 @@ def test_posts_and_rounds_from_host_threads():
     assert rounds == 2 * n and sum(claimed) == 2 * n
     assert_clean(c.h)
     m.close()
+
+
+def test_mailbox_full_size_fp8():
+    """The FP8 workload (8 x 4096 tokens, Zipf popularity) posted from eight
+    streams, every post served right after it: each output bit-identical to
+    asap_moe_layer's on the same micro-batch."""
+    cfg = DSV3_FP8
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
+    del w
+    torch.cuda.empty_cache()
+    xs = inputs.make_microbatches(cfg, DEV)
+    ws = api.workspace(h, max(cfg.microbatches))
+    ref = []
+    for x in xs:
+        o = torch.empty_like(x)
+        api.asap_moe_layer(h, x, o, ws)
+        ref.append(o)
+    torch.cuda.synchronize()
+    del ws
+    m = api.asap_moe_mailbox_create(h, len(xs), max(cfg.microbatches))
+    producers = [torch.cuda.Stream() for _ in xs]
+    server = torch.cuda.Stream()
+    outs = [torch.full_like(x, 5.0) for x in xs]
+    eps = [api.asap_moe_mailbox_post(m, i, x, o, stream=p) for i, (x, o, p) in enumerate(zip(xs, outs, producers))]
+    for i, ep in enumerate(eps):
+        api.asap_moe_mailbox_serve(m, i, ep, stream=server)
+    torch.cuda.synchronize()
+    for a, b in zip(ref, outs):
+        assert same_bits(a, b)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == len(xs) and sum(claimed) == len(xs)
+    print(f"[fp8 full size] posts per round: {claimed}")
+    assert_clean(h)
+    m.close()
+    h.close()
