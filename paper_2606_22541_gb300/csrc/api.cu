@@ -1430,7 +1430,8 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
   if (h->fp8) {
     void* xq_sh = sh ? at<void>(ws, L.xq_sh) : nullptr;
     float* xs_sh = sh ? at<float>(ws, L.xs_sh) : nullptr;
-    CU_TRY(asap::launch_dispatch_fp8_mbox(m->round, g, idx, at<int32_t>(ws, L.chunk_base), offsets, at<void>(ws, L.xq),
+    CU_TRY(asap::launch_dispatch_fp8_mbox(m->round, g, m->rowmap, idx, at<int32_t>(ws, L.chunk_base), offsets,
+                                          at<void>(ws, L.xq),
                                           at<float>(ws, L.xs), xq_sh, xs_sh, at<int32_t>(ws, L.perm_src), perm_dst,
                                           h->status, st),
            "dispatch launch");
@@ -1447,7 +1448,7 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
     // the shared expert reads the gathered rows from y_sh's region, which its
     // own output overwrites only after the gate/up GEMM
     y_perm = at<void>(ws, L.x_perm);
-    CU_TRY(asap::launch_dispatch_mbox(m->round, g, idx, at<int32_t>(ws, L.chunk_base), offsets, y_perm,
+    CU_TRY(asap::launch_dispatch_mbox(m->round, g, m->rowmap, idx, at<int32_t>(ws, L.chunk_base), offsets, y_perm,
                                       at<int32_t>(ws, L.perm_src), perm_dst, y_sh, h->status, st),
            "dispatch launch");
     if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");

@@ -251,6 +251,7 @@ struct MboxRound {           // the set the current service round claimed (its c
   int chunks_total;          // their histogram rows (rowmap entries)
   int rounds;                // service rounds run so far, this one included
   int layer;                 // the layer every claimed post belongs to (the GEMMs read its weights)
+  int index_of[kMboxMaxSlots];  // claimed slot -> its index i below (unclaimed slots: stale)
   int slot[kMboxMaxSlots];   // claimed slots, increasing
   int n[kMboxMaxSlots];
   int tok0[kMboxMaxSlots];   // first token in the round's combined token order
@@ -291,12 +292,14 @@ cudaError_t launch_scan_mapped(const int32_t* hist, const int32_t* rowmap, const
 // (claimed slot, token, slot of k) order); perm_src holds combined token
 // indices, perm_dst the slot's own region; x_sh / xq_sh, xs_sh receive the
 // combined rows of the shared expert.
-cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
-                                 const int32_t* offsets, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
-                                 void* x_sh, uint32_t* status, cudaStream_t s);
-cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
-                                     const int32_t* offsets, void* xq, float* xs, void* xq_sh, float* xs_sh,
-                                     int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s);
+// rowmap: the round's histogram rows (the claim kernel's map).
+cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* rowmap, const int32_t* idx,
+                                 const int32_t* chunk_base, const int32_t* offsets, void* x_perm, int32_t* perm_src,
+                                 int32_t* perm_dst, void* x_sh, uint32_t* status, cudaStream_t s);
+cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* rowmap, const int32_t* idx,
+                                     const int32_t* chunk_base, const int32_t* offsets, void* xq, float* xs,
+                                     void* xq_sh, float* xs_sh, int32_t* perm_src, int32_t* perm_dst,
+                                     uint32_t* status, cudaStream_t s);
 // Combine of every claimed post into its own output.
 cudaError_t launch_combine_mbox(const MboxRound* r, MboxGeom g, const void* y_perm, const void* y_shared,
                                 const float* w, const int32_t* perm_dst, uint32_t* status, cudaStream_t s);

@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kMboxMaxSlots) mbox_claim_kernel(MboxSlot* slo
   }
   if (pend) {
     const int i = ic - 1;
+    r->index_of[s] = i;
     r->slot[i] = s;
     r->n[i] = n;
     r->tok0[i] = it - n;

@@ -201,27 +201,22 @@ __global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
                       xs_sh, perm_src, perm_dst, status, seg);
 }
 
-// Dispatch of a mailbox round: CTA (i, c, part) handles chunk c of the i-th
-// claimed post; CTAs past the claimed posts or their chunks return at once.
-// The post's tokens come first in the combined order at r->tok0[i], its
-// histogram rows and chunk bases are its slot's rows, its idx / perm_dst
-// entries its slot's region.
+// One work item of a mailbox round's dispatch: part ``part`` of the round's
+// chunk vc (see dispatch_mbox_kernel).
 template <bool FP8>
-__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
-    dispatch_mbox_kernel(const MboxRound* __restrict__ r, const MboxGeom g, const int32_t* __restrict__ idx,
-                         const int32_t* __restrict__ chunk_base, const int32_t* __restrict__ offsets,
-                         void* __restrict__ x_perm_v, float* __restrict__ xs, void* __restrict__ x_sh,
-                         float* __restrict__ xs_sh, int32_t* __restrict__ perm_src, int32_t* __restrict__ perm_dst,
-                         uint32_t* status) {
-  constexpr int kParts = dispatch_parts<FP8>();
-  const int per_slot = g.slot_chunks * kParts;
-  const int i = blockIdx.x / per_slot;
-  const int rem = blockIdx.x - i * per_slot;
-  const int c = rem / kParts, part = rem % kParts;
-  if (i >= r->count) return;
+__device__ __forceinline__ void dispatch_mbox_item(int vc, int part, const MboxRound* __restrict__ r,
+                                                   const MboxGeom& g, const int32_t* __restrict__ rowmap,
+                                                   const int32_t* __restrict__ idx,
+                                                   const int32_t* __restrict__ chunk_base,
+                                                   const int32_t* __restrict__ offsets, void* __restrict__ x_perm_v,
+                                                   float* __restrict__ xs, void* __restrict__ x_sh,
+                                                   float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
+                                                   int32_t* __restrict__ perm_dst, uint32_t* status) {
+  const int row = rowmap[vc];
+  const int slot = row / g.slot_chunks;
+  const int c = row - slot * g.slot_chunks;
+  const int i = r->index_of[slot];
   const int n = r->n[i];
-  if (c * kChunkTokens >= n) return;
-  const int slot = r->slot[i];
   const long long tok0 = r->tok0[i];
   const int V = g.H / 8;
   DispatchSeg seg{};
@@ -243,6 +238,28 @@ __global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
   const long long sidx = static_cast<long long>(slot) * g.slot_tokens * g.k;
   dispatch_chunk<FP8>(c, part, static_cast<const uint4*>(r->x[i]), n, V, g.k, g.E, idx + sidx, chunk_base, x_perm_v,
                       xs, xq_sh, xs_sh_i, perm_src, perm_dst + sidx, status, seg);
+}
+
+// Dispatch of a mailbox round: work item q is part q % kParts of the
+// round's chunk q / kParts in the scan's order (the row map lists the claimed
+// posts' histogram rows, post after post); CTA b takes items b, b + gridDim.x,
+// ...  The chunk's post comes at r->tok0[i] in the combined token order, its
+// histogram row and chunk bases are its slot's, its idx / perm_dst entries
+// its slot's region.
+template <bool FP8>
+__global__ void __launch_bounds__(dispatch_warps<FP8>() * 32)
+    dispatch_mbox_kernel(const MboxRound* __restrict__ r, const MboxGeom g, const int32_t* __restrict__ rowmap,
+                         const int32_t* __restrict__ idx, const int32_t* __restrict__ chunk_base,
+                         const int32_t* __restrict__ offsets, void* __restrict__ x_perm_v, float* __restrict__ xs,
+                         void* __restrict__ x_sh, float* __restrict__ xs_sh, int32_t* __restrict__ perm_src,
+                         int32_t* __restrict__ perm_dst, uint32_t* status) {
+  constexpr int kParts = dispatch_parts<FP8>();
+  const int items = r->chunks_total * kParts;
+  for (int q = blockIdx.x; q < items; q += gridDim.x) {
+    dispatch_mbox_item<FP8>(q / kParts, q % kParts, r, g, rowmap, idx, chunk_base, offsets, x_perm_v, xs, x_sh,
+                            xs_sh, perm_src, perm_dst, status);
+    __syncthreads();  // the chunk's shared rank tables are rewritten by the next item
+  }
 }
 
 // Rows of bf16 to e4m3 with a scale per 128 channels; one warp per row.
@@ -335,25 +352,34 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
   combine_token(y_perm, y_sh ? y_sh + tv : nullptr, w + tk, perm_dst + tk, V, k, out + tv, status, nk, lane);
 }
 
-// Combine of a mailbox round: CTA (i, b) combines tokens b * kCombineWarps ..
-// of the i-th claimed post into that post's output; its weights and
-// positions are in its slot's region, its shared-expert rows at its place in
-// the combined order.
+// Combine of a mailbox round: warp w of CTA b combines the tokens
+// (b + j gridDim.x) * kCombineWarps + w of the round's combined token order
+// (the claimed posts one after the other).  A token's post i (the last with
+// r->tok0[i] <= it) writes into its own output; its weights and positions are
+// in its slot's region, its shared-expert row at its place in the combined
+// order.
 __global__ void __launch_bounds__(kCombineWarps * 32)
     combine_mbox_kernel(const MboxRound* __restrict__ r, const MboxGeom g, const uint4* __restrict__ y_perm,
                         const uint4* __restrict__ y_sh, const float* __restrict__ w,
                         const int32_t* __restrict__ perm_dst, uint32_t* status) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int per_slot = (g.slot_tokens + kCombineWarps - 1) / kCombineWarps;
-  const int i = blockIdx.x / per_slot;
-  if (i >= r->count) return;
-  const int t = (blockIdx.x - i * per_slot) * kCombineWarps + warp;
-  if (t >= r->n[i]) return;
+  const int n_total = r->n_total, count = r->count;
   const int V = g.H / 8;
-  const long long tk = (static_cast<long long>(r->slot[i]) * g.slot_tokens + t) * g.k;
-  const long long nk = static_cast<long long>(r->n_total) * g.k;
-  combine_token(y_perm, y_sh ? y_sh + (static_cast<long long>(r->tok0[i]) + t) * V : nullptr, w + tk, perm_dst + tk, V,
-                g.k, static_cast<uint4*>(r->out[i]) + static_cast<long long>(t) * V, status, nk, lane);
+  const long long nk = static_cast<long long>(n_total) * g.k;
+  for (int tg = blockIdx.x * kCombineWarps + warp; tg < n_total; tg += gridDim.x * kCombineWarps) {
+    int lo = 0, hi = count;  // the last claimed post starting at or before tg
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (r->tok0[mid] <= tg) lo = mid; else hi = mid;
+    }
+    const int i = lo;
+    const int t = tg - r->tok0[i];
+    if (t >= r->n[i]) continue;
+    const long long tk = (static_cast<long long>(r->slot[i]) * g.slot_tokens + t) * g.k;
+    combine_token(y_perm, y_sh ? y_sh + (static_cast<long long>(r->tok0[i]) + t) * V : nullptr, w + tk,
+                  perm_dst + tk, V, g.k, static_cast<uint4*>(r->out[i]) + static_cast<long long>(t) * V, status, nk,
+                  lane);
+  }
 }
 
 // packed[e][b*256 + r] = gate[e][b*128 + r] for r < 128, up[e][b*128 + r - 128]
@@ -453,28 +479,30 @@ cudaError_t launch_combine(const void* y_perm, const void* y_shared, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
-                                 const int32_t* offsets, void* x_perm, int32_t* perm_src, int32_t* perm_dst,
-                                 void* x_sh, uint32_t* status, cudaStream_t s) {
-  const int grid = g.n_slots * g.slot_chunks * dispatch_parts<false>();
-  dispatch_mbox_kernel<false><<<grid, dispatch_warps<false>() * 32, 0, s>>>(r, g, idx, chunk_base, offsets, x_perm,
-                                                                            nullptr, x_sh, nullptr, perm_src,
+cudaError_t launch_dispatch_mbox(const MboxRound* r, MboxGeom g, const int32_t* rowmap, const int32_t* idx,
+                                 const int32_t* chunk_base, const int32_t* offsets, void* x_perm, int32_t* perm_src,
+                                 int32_t* perm_dst, void* x_sh, uint32_t* status, cudaStream_t s) {
+  const int grid = g.slot_chunks * dispatch_parts<false>();  // one post's work items; more loop
+  dispatch_mbox_kernel<false><<<grid, dispatch_warps<false>() * 32, 0, s>>>(r, g, rowmap, idx, chunk_base, offsets,
+                                                                            x_perm, nullptr, x_sh, nullptr, perm_src,
                                                                             perm_dst, status);
   return cudaGetLastError();
 }
 
-cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* idx, const int32_t* chunk_base,
-                                     const int32_t* offsets, void* xq, float* xs, void* xq_sh, float* xs_sh,
-                                     int32_t* perm_src, int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
-  const int grid = g.n_slots * g.slot_chunks * dispatch_parts<true>();
-  dispatch_mbox_kernel<true><<<grid, dispatch_warps<true>() * 32, 0, s>>>(r, g, idx, chunk_base, offsets, xq, xs,
-                                                                          xq_sh, xs_sh, perm_src, perm_dst, status);
+cudaError_t launch_dispatch_fp8_mbox(const MboxRound* r, MboxGeom g, const int32_t* rowmap, const int32_t* idx,
+                                     const int32_t* chunk_base, const int32_t* offsets, void* xq, float* xs,
+                                     void* xq_sh, float* xs_sh, int32_t* perm_src, int32_t* perm_dst,
+                                     uint32_t* status, cudaStream_t s) {
+  const int grid = g.slot_chunks * dispatch_parts<true>();  // one post's work items; more loop
+  dispatch_mbox_kernel<true><<<grid, dispatch_warps<true>() * 32, 0, s>>>(r, g, rowmap, idx, chunk_base, offsets, xq,
+                                                                          xs, xq_sh, xs_sh, perm_src, perm_dst,
+                                                                          status);
   return cudaGetLastError();
 }
 
 cudaError_t launch_combine_mbox(const MboxRound* r, MboxGeom g, const void* y_perm, const void* y_shared,
                                 const float* w, const int32_t* perm_dst, uint32_t* status, cudaStream_t s) {
-  const int grid = g.n_slots * ceil_div(g.slot_tokens, kCombineWarps);
+  const int grid = ceil_div(g.slot_tokens, kCombineWarps);  // one post's tokens; more loop
   combine_mbox_kernel<<<grid, kCombineWarps * 32, 0, s>>>(r, g, static_cast<const uint4*>(y_perm),
                                                           static_cast<const uint4*>(y_shared), w, perm_dst, status);
   return cudaGetLastError();
