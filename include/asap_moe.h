@@ -360,11 +360,10 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
 /* ------------------------------------------------------------------------
  * Mailbox: the device decides which micro-batches one grouped GEMM pass
  * serves.  The single-GPU form of the asynchronous primitives of Sections
- * 3.2.1 and 3.2.2 (Table 2: a payload region, a metadata region and a ready
- * bitmap per DP group; the receiver polls the bitmaps, migrates the payload
- * into its private memory, clears the flags, and returns results with a
- * completion bitmap), with the MoE side serving DP groups out of order
- * (Section 3.3).
+ * 3.2.1 and 3.2.2 (Table 2: per DP group, regions for the token data and the
+ * per-expert counts plus ready bits that the MoE side checks before copying a
+ * group's data into its own memory; results return with completion bits),
+ * with the MoE side serving DP groups out of order (Section 3.3).
  *
  *  - A DP group's stream POSTS a micro-batch into its slot: the post routes
  *    it (exactly as asap_moe_route) into the slot's region and then sets the
