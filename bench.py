@@ -364,6 +364,11 @@ def run_ours(args, dist):
     if not args.no_mailbox:
         result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
                                          latest_first=args.mailbox_latest_first)
+        pl = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
+                          latest_first=args.mailbox_latest_first, pipelined=True)
+        result["mailbox"]["pipelined"] = {key: pl[key] for key in (
+            "value", "ms_per_step", "nonempty_rounds_per_step", "posts_per_nonempty_round", "round_sizes_histogram",
+            "grouped_gemm_frac_of_burst_measured", "grouped_gemm_frac_of_sustained_measured", "steps")}
 
     # ---------------- per-micro-batch latency of the per-stream step
     result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
@@ -600,7 +605,7 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
     return res
 
 
-def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_first=False):
+def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_first=False, pipelined=False):
     """The step's micro-batches posted into a mailbox, each from its own
     stream, and served by rounds on one MoE stream: the host serves every post
     right after making it (no host batching), and each round claims on the
@@ -611,7 +616,11 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     tensor fraction (algorithmic FLOPs of the step over the event-timed GEMMs
     of its rounds).  latest_first: the step's rounds are started from its
     last post backwards (a server that, knowing of several posts, starts the
-    round from the newest; the device still claims whatever is published)."""
+    round from the newest; the device still claims whatever is published).
+    pipelined: no barrier between steps: a step's posts wait only for the
+    rounds that served their slots' previous posts (the post's own
+    backpressure), so they are made while the previous step's rounds run, as
+    in a serving loop where DP groups keep sending."""
     import torch
     from paper_2606_22541_gb300 import api
 
@@ -628,7 +637,8 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
         ev.record(main)
         eps = []
         for i, (x, p) in enumerate(zip(xs, producers)):
-            p.wait_event(ev)
+            if not pipelined:
+                p.wait_event(ev)
             eps.append(api.asap_moe_mailbox_post(m, b * n_mb + i, x, outs[b][i], stream=p))
         for r, i in enumerate(reversed(range(n_mb)) if latest_first else range(n_mb)):
             if gemm_events is not None:
@@ -688,6 +698,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "grouped_gemm_frac_of_sustained_measured": tf / tpk_sus,
             "gemm_timing_nonempty_rounds_per_step": sum(nonempty) / len(nonempty),
             "serve_order": "latest post first" if latest_first else "post order",
+            "steps": "back to back, no barrier between steps" if pipelined else "one barrier per step",
             "note": "asap_moe_mailbox_post from one stream per micro-batch, asap_moe_mailbox_serve for every post "
                     "right after it on one MoE stream; the rounds claim on the device whatever has been published"}
 

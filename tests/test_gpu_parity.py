@@ -328,6 +328,42 @@ def test_expert_ffn_matches_oracle(cfg):
     assert_clean(c)
 
 
+def test_expert_ffn_segment_tails_at_mma_boundaries():
+    """Segments whose last 128-row half holds 1, 63, 64, 65, 127 or 128 rows,
+    with one, two and three 128-row halves (a half of at most 64 rows takes
+    M = 64 MMAs): single and paired m-tiles give the same bits, equal to the
+    oracle's values."""
+    cfg = DS_SMALL
+    c = Case.get(cfg)
+    n, k, E, H = max(cfg.microbatches), cfg.top_k, cfg.n_experts, cfg.hidden
+    sizes = [1, 63, 64, 65, 127, 128, 129, 191, 192, 193, 257, 320, 321, 0, 2]
+    counts = np.zeros(E, np.int64)
+    counts[:len(sizes)] = sizes
+    counts[E - 1] = n * k - counts.sum()          # the rest in the last expert
+    assert counts[E - 1] >= 0
+    offsets_np = oracle.expert_offsets(counts)
+    x = c.tokens(0, n)
+    x_perm = inputs.randn_bf16((n * k, H), 1.0, 92, DEV)
+    offsets = torch.tensor(offsets_np, dtype=torch.int32, device=DEV)
+    outs = []
+    try:
+        for mode in (api.TILING_SINGLE, api.TILING_PAIRED):
+            api.asap_moe_set_tiling(c.h, mode)
+            y_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=DEV)
+            y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+            api.asap_moe_expert_ffn(c.h, x_perm, offsets, x, y_perm, y_sh, c.ws(n))
+            outs.append(y_perm)
+        torch.cuda.synchronize()
+    finally:
+        api.asap_moe_set_tiling(c.h, api.TILING_AUTO)
+    assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
+    lim = int(offsets_np[len(sizes)])               # the boundary segments
+    ref = oracle.expert_ffn(bf16_to_f64(x_perm[:lim]), offsets_np[:len(sizes) + 1], c.wf["w_gate"], c.wf["w_up"],
+                            c.wf["w_down"])
+    compare_rows(bf16_to_f64(outs[1][:lim]), ref)
+    assert_clean(c)
+
+
 @pytest.mark.parametrize("hot", ["first", "middle", "last"])
 def test_expert_ffn_all_rows_in_one_expert(hot):
     """Every routed row in one expert, every other segment empty, with single
