@@ -50,6 +50,10 @@ def parse_args():
     ap.add_argument("--no-mailbox", action="store_true", help="skip the mailbox (device-side ready set) leg")
     ap.add_argument("--mailbox-latest-first", action="store_true",
                     help="start each step's mailbox rounds from its last post instead of its first")
+    ap.add_argument("--mailbox-back-to-back", action="store_true",
+                    help="mailbox leg without a barrier between steps")
+    ap.add_argument("--mailbox-priority", type=int, default=0,
+                    help="1: the posting streams get the highest CUDA stream priority")
     ap.add_argument("--cpu-sample-tokens", type=int, default=12)
     ap.add_argument("--microbatches", default=None,
                     help="comma-separated micro-batch sizes overriding the workload's")
@@ -363,12 +367,8 @@ def run_ours(args, dist):
     # ---------------- the device decides the sets: mailbox posts and service rounds
     if not args.no_mailbox:
         result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
-                                         latest_first=args.mailbox_latest_first)
-        pl = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
-                          latest_first=args.mailbox_latest_first, pipelined=True)
-        result["mailbox"]["pipelined"] = {key: pl[key] for key in (
-            "value", "ms_per_step", "nonempty_rounds_per_step", "posts_per_nonempty_round", "round_sizes_histogram",
-            "grouped_gemm_frac_of_burst_measured", "grouped_gemm_frac_of_sustained_measured", "steps")}
+                                         latest_first=args.mailbox_latest_first,
+                                         pipelined=args.mailbox_back_to_back)
 
     # ---------------- per-micro-batch latency of the per-stream step
     result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
@@ -626,7 +626,9 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
 
     n_mb = len(xs)
     m = api.asap_moe_mailbox_create(h, 2 * n_mb, max(x.shape[0] for x in xs))
-    producers = [torch.cuda.Stream() for _ in xs]
+    # --mailbox-priority: the DP groups' streams above the MoE stream
+    hi = torch.cuda.Stream.priority_range()[1] if args.mailbox_priority else 0
+    producers = [torch.cuda.Stream(priority=hi) for _ in xs]
     server = torch.cuda.Stream()
     main = torch.cuda.current_stream()
     outs = [[torch.empty_like(x) for x in xs] for _ in range(2)]
@@ -699,6 +701,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "gemm_timing_nonempty_rounds_per_step": sum(nonempty) / len(nonempty),
             "serve_order": "latest post first" if latest_first else "post order",
             "steps": "back to back, no barrier between steps" if pipelined else "one barrier per step",
+            "posting_stream_priority": "highest" if args.mailbox_priority else "default",
             "note": "asap_moe_mailbox_post from one stream per micro-batch, asap_moe_mailbox_serve for every post "
                     "right after it on one MoE stream; the rounds claim on the device whatever has been published"}
 
