@@ -48,6 +48,8 @@ def parse_args():
     ap.add_argument("--kernel-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-mailbox", action="store_true", help="skip the mailbox (device-side ready set) leg")
+    ap.add_argument("--no-extra-workloads", action="store_true",
+                    help="skip the brief per-stream and aggregated timing of the other workloads")
     ap.add_argument("--mailbox-latest-first", action="store_true",
                     help="start each step's mailbox rounds from its last post instead of its first")
     ap.add_argument("--mailbox-back-to-back", action="store_true",
@@ -378,13 +380,84 @@ def run_ours(args, dist):
     # ---------------- end to end through host buffers
     result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
 
+    # ---------------- the other workloads, briefly (N = 1 only)
+    if dist.world == 1 and not args.no_extra_workloads:
+        h.close()
+        del xs, outs, wss
+        torch.cuda.empty_cache()
+        result["other_workloads"] = {name: other_workload(args, name, dev)
+                                     for name in ("mixtral", "dsv3_stress", "dsv3_fp8") if name != cfg.name}
+        h = None
+
     # ---------------- float64 oracle on the host cores
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(cfg, dev, args.cpu_sample_tokens)
     else:
         result["cpu_baseline"] = None
-    h.close()
+    if h is not None:
+        h.close()
     return result
+
+
+def other_workload(args, name, dev):
+    """Another configuration's per-stream step (every micro-batch through
+    asap_moe_layer on its own stream; each step's streams wait for the
+    previous step on the device, as in the headline) and its host-aggregated
+    step (asap_moe_layer_batched), timed with CUDA events: W warm-up and
+    K = max(3, steps // 2) timed steps each."""
+    import torch
+    from paper_2606_22541_gb300 import api, inputs
+    from paper_2606_22541_gb300.configs import CONFIGS
+
+    cfg = CONFIGS[name]
+    mbs = cfg.microbatches
+    w = inputs.make_weights(cfg, dev)
+    h = api.asap_moe_create(cfg, w, sum(mbs))
+    del w
+    torch.cuda.empty_cache()
+    xs = inputs.make_microbatches(cfg, dev)
+    outs = [torch.empty_like(x) for x in xs]
+    wss = [api.workspace(h, x.shape[0], dev) for x in xs]
+    streams = [torch.cuda.Stream(device=dev) for _ in xs]
+    main = torch.cuda.current_stream()
+    steps = max(3, args.steps // 2)
+
+    def per_stream():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        for x, o, ws, s in zip(xs, outs, wss, streams):
+            s.wait_event(ev)
+            api.asap_moe_layer(h, x, o, ws, stream=s)
+        for s in streams:
+            main.wait_stream(s)
+
+    ws_all = api.workspace(h, sum(mbs), dev)
+
+    def aggregated():
+        api.asap_moe_layer_batched(h, xs, outs, ws_all)
+
+    res = {}
+    for key, fn in (("per_stream", per_stream), ("aggregated", aggregated)):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(main)
+        for _ in range(steps):
+            fn()
+        b.record(main)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        res[key] = {"value": sum(mbs) / (ms / 1e3), "unit": "tokens/s", "ms_per_step": ms}
+    code, word = api.asap_moe_status(h)
+    h.close()
+    if code != 0:
+        raise RuntimeError(f"{name}: device status word {word:#x}")
+    res.update({"microbatches": mbs, "dtype": cfg.dtype, "steps": steps,
+                "note": "per-stream: one stream per micro-batch through asap_moe_layer; aggregated: "
+                        "asap_moe_layer_batched over the step's micro-batches"})
+    return res
 
 
 def kernel_pass(args, h, cfg, xs, dev):
