@@ -69,7 +69,7 @@ extern "C" {
 typedef enum {
   ASAP_OK = 0,
   ASAP_ERR_INVALID = -1,      /* bad argument or configuration */
-  ASAP_ERR_UNSUPPORTED = -2,  /* valid request this build does not implement */
+  ASAP_ERR_UNSUPPORTED = -2,  /* valid request the library does not implement */
   ASAP_ERR_WORKSPACE = -3,    /* workspace missing or too small */
   ASAP_ERR_CUDA = -4,         /* a CUDA runtime call or launch failed */
   ASAP_ERR_DEVICE_STATUS = -5 /* a kernel recorded an error (asap_moe_status) */
