@@ -20,10 +20,13 @@ constexpr unsigned kFull = 0xffffffffu;
 // The bf16 dispatch splits a chunk's row copies over two CTAs (every one
 // ranks the chunk's entries, the first writes the permutation), so 4096
 // tokens run 256 CTAs, more than the 152 SMs (measured on GB300: 112 -> 107
-// us); the FP8 dispatch, which also quantises, is faster with one CTA per
-// chunk (85 us vs 100 us).
+// us; four CTAs per chunk: 111 us); the FP8 dispatch, which also quantises,
+// is faster with one CTA per chunk (85 us vs 100 us).
+#ifndef ASAP_DISPATCH_PARTS
+#define ASAP_DISPATCH_PARTS 2
+#endif
 template <bool FP8>
-__host__ __device__ constexpr int dispatch_parts() { return FP8 ? 1 : 2; }
+__host__ __device__ constexpr int dispatch_parts() { return FP8 ? 1 : ASAP_DISPATCH_PARTS; }
 constexpr int kRankWarps = kChunkTokens * kMaxTopK / 32;  // warps that rank the chunk's entries
 template <bool FP8>
 __host__ __device__ constexpr int dispatch_warps() {
