@@ -6,7 +6,8 @@ output on a sample of at least SAMPLE_PER_MB decided tokens per micro-batch
 last token, the first and last tokens routed to its most and to its least
 loaded expert (the ends of those segments and the last m-tiles of the
 grouped GEMMs), and seeded random tokens; concurrent submission must equal
-serial submission bit for bit."""
+serial submission bit for bit.  A last case runs the largest micro-batch
+the stress workload's length recipe allows."""
 import numpy as np
 import pytest
 import torch
@@ -30,7 +31,13 @@ def _built():
     __graft_entry__.build()
 
 
-@pytest.mark.parametrize("cfg", [MIXTRAL, DSV3, STRESS], ids=lambda c: c.name)
+# the largest micro-batch the stress workload's length recipe allows (its
+# clip at 16384 tokens) through one call: the route without a K split, 512
+# dispatch chunks, about 512 rows per expert in the grouped GEMMs
+STRESS_MAX = inputs.small_variant(STRESS, name="dsv3_stress_max_microbatch", microbatches=[16384])
+
+
+@pytest.mark.parametrize("cfg", [MIXTRAL, DSV3, STRESS, STRESS_MAX], ids=lambda c: c.name)
 def test_full_size_streams_against_oracle(cfg):
     w = inputs.make_weights(cfg, DEV)
     h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
