@@ -392,6 +392,10 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
  *    was made for the previous post returns ASAP_ERR_INVALID (the sender's
  *    backpressure of Section 3.2.1).
  *  - x and out of a post must stay valid until the post is served.
+ *  - Rounds run one after another: each serve call makes its stream wait for
+ *    the mailbox's previous round (they share one server workspace), so
+ *    serve calls may come from any stream; one MoE stream is the usual case,
+ *    where that wait costs nothing.
  *
  * Layers: each post belongs to one MoE layer of the handle (a device int32
  * layer id read when the post is published; see asap_moe_layer_dyn).  A round

@@ -1250,6 +1250,8 @@ struct asap_moe_mailbox_s {
   std::vector<cudaEvent_t> post_ev, served_ev;
   std::vector<unsigned long long> posted, serve_called;  // host view: last post, last serve call per slot
   cudaEvent_t gemm_ev0 = nullptr, gemm_ev1 = nullptr;   // recorded around the next round's GEMMs
+  cudaEvent_t round_ev = nullptr;  // end of the last round (rounds share the server workspace)
+  bool any_round = false;
   std::mutex mu;
 };
 
@@ -1269,6 +1271,7 @@ int mbox_free(asap_moe_mailbox_t m) {
   if (m->served_host) cudaFreeHost(m->served_host);
   for (cudaEvent_t e : m->post_ev) cudaEventDestroy(e);
   for (cudaEvent_t e : m->served_ev) cudaEventDestroy(e);
+  if (m->round_ev) cudaEventDestroy(m->round_ev);
   cudaSetDevice(prev);
   delete m;
   return ASAP_OK;
@@ -1335,6 +1338,8 @@ ASAP_API int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot
     if ((e = cudaEventCreateWithFlags(&m->post_ev[i], cudaEventDisableTiming)) != cudaSuccess ||
         (e = cudaEventCreateWithFlags(&m->served_ev[i], cudaEventDisableTiming)) != cudaSuccess)
       return restore(bail(cuda_fail(e, "mailbox events")));
+  if ((e = cudaEventCreateWithFlags(&m->round_ev, cudaEventDisableTiming)) != cudaSuccess)
+    return restore(bail(cuda_fail(e, "mailbox events")));
   m->posted.assign(n_slots, 0);
   m->serve_called.assign(n_slots, 0);
   if ((e = cudaDeviceSynchronize()) != cudaSuccess) return restore(bail(cuda_fail(e, "mailbox create sync")));
@@ -1414,8 +1419,11 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
   const int32_t* n_total = &m->round->n_total;
   const int32_t* layer = &m->round->layer;  // the layer of the claimed posts, written by the claim
   int r;
-  // the post this round is for was published before the round starts
+  // the post this round is for was published before the round starts; the
+  // previous round (on whatever stream it was served) is done with the
+  // server workspace
   CU_TRY(cudaStreamWaitEvent(st, m->post_ev[slot], 0), "wait for the post");
+  if (m->any_round) CU_TRY(cudaStreamWaitEvent(st, m->round_ev, 0), "wait for the previous round");
   CU_TRY(asap::launch_mbox_claim(m->slots, g, slot, epoch, m->wait_ns, m->round, m->rowmap, at<int32_t>(ws, L.ticket),
                                  h->status, st),
          "claim launch");
@@ -1465,6 +1473,8 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
          "combine launch");
   CU_TRY(asap::launch_mbox_finish(m->slots, m->round, m->log, m->served_host_dev, st), "finish launch");
   CU_TRY(cudaEventRecord(m->served_ev[slot], st), "served event");
+  CU_TRY(cudaEventRecord(m->round_ev, st), "round event");
+  m->any_round = true;
   if (epoch > m->serve_called[slot]) m->serve_called[slot] = epoch;
   return ASAP_OK;
 }

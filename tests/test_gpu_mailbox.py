@@ -134,6 +134,39 @@ def test_random_arrivals_and_delays(cfg):
     m.close()
 
 
+def test_serve_calls_from_several_streams():
+    """Serve calls spread over three server streams (a round per post, its
+    stream chosen at random): each round waits for the mailbox's previous
+    round, so rounds never overlap on the shared server workspace, and the
+    outputs stay bit-identical over passes that reuse the slots."""
+    c = Case.get(DS)
+    n = len(c.xs)
+    rng = np.random.default_rng(11)
+    m = api.asap_moe_mailbox_create(c.h, n, max(DS.microbatches))
+    producers = [torch.cuda.Stream() for _ in range(2)]
+    servers = [torch.cuda.Stream() for _ in range(3)]
+    for rep in range(3):
+        outs = [torch.full_like(x, float(rep + 1)) for x in c.xs]
+        for i in rng.permutation(n):
+            s = producers[int(rng.integers(0, 2))]
+            with torch.cuda.stream(s):
+                torch.cuda._sleep(int(rng.integers(0, 200_000)))
+            if rep > 0:
+                api.asap_moe_mailbox_wait(m, int(i), stream=s)
+            ep = api.asap_moe_mailbox_post(m, int(i), c.xs[i], outs[i], stream=s)
+            srv = servers[int(rng.integers(0, 3))]
+            with torch.cuda.stream(srv):
+                torch.cuda._sleep(int(rng.integers(0, 200_000)))
+            api.asap_moe_mailbox_serve(m, int(i), ep, stream=srv)
+        torch.cuda.synchronize()
+        for a, b in zip(c.ref, outs):
+            assert same_bits(a, b)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == 3 * n and sum(claimed) == 3 * n
+    assert_clean(c.h)
+    m.close()
+
+
 def test_mailbox_output_against_oracle():
     """The chain to the oracle directly: one round serving three posts of the
     DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
