@@ -47,5 +47,6 @@ def test_batched_equals_separate_calls(cfg, lengths):
     _check(cfg, lengths)
 
 
-def test_batched_full_size_dsv3():
-    _check(DSV3, DSV3.microbatches)
+@pytest.mark.parametrize("cfg", [DSV3, STRESS, MIXTRAL], ids=lambda c: c.name)
+def test_batched_full_size(cfg):
+    _check(cfg, cfg.microbatches)

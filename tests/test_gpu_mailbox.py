@@ -14,7 +14,7 @@ import torch
 import oracle
 from paper_2606_22541_gb300 import api, inputs
 from paper_2606_22541_gb300._native import AsapError
-from paper_2606_22541_gb300.configs import DSV3, DSV3_FP8, MIXTRAL
+from paper_2606_22541_gb300.configs import DSV3, DSV3_FP8, MIXTRAL, STRESS
 
 from _helpers import bf16_to_f64, compare_rows
 
@@ -305,12 +305,14 @@ def test_mailbox_on_a_layer_of_a_multi_layer_handle():
     one.close()
 
 
-def test_mailbox_full_size_dsv3():
-    """The bench's workload: 4 x 4096 DeepSeek-V3 tokens posted from four
-    streams, every post served right after it on one MoE stream, twice (the
-    second time the slots are reposted): every output bit-identical to
+@pytest.mark.parametrize("cfg", [DSV3, STRESS, MIXTRAL], ids=lambda c: c.name)
+def test_mailbox_full_size(cfg):
+    """The bench's workloads at full size (DeepSeek-V3 4 x 4096; the stress
+    workload's 8 ragged micro-batches of 362 to 8045 tokens with Zipf
+    experts; Mixtral's 4 micro-batches), each posted from its own stream,
+    every post served right after it on one MoE stream, twice (the second
+    time the slots are reposted): every output bit-identical to
     asap_moe_layer on the same micro-batch."""
-    cfg = DSV3
     w = inputs.make_weights(cfg, DEV)
     h = api.asap_moe_create(cfg, w, max(cfg.microbatches))
     del w
@@ -338,7 +340,7 @@ def test_mailbox_full_size_dsv3():
             assert same_bits(a, b)
     rounds, claimed = api.asap_moe_mailbox_rounds(m)
     assert rounds == 2 * len(xs) and sum(claimed) == 2 * len(xs)
-    print(f"[dsv3 full size] posts per round: {claimed}")
+    print(f"[{cfg.name} full size] posts per round: {claimed}")
     assert_clean(h)
     m.close()
     h.close()
