@@ -193,11 +193,11 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
                       cudaStream_t st) {
   const asap_moe_config& c = h->cfg;
   if (h->tc_router) {
-    CUtensorMap maps[2];
+    CUtensorMap maps[4];
     std::string err;
     if (!asap::encode_tmap_bf16(&maps[0], x, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
-    maps[1] = maps[0];
+    maps[1] = maps[2] = maps[3] = maps[0];  // the fp32 logits are stored without TMA
     asap::GemmArgs a{};
     a.lref = lref(h, layer);
     a.bmap0 = a.bmap1 = asap::MAP_ROUTER;
@@ -335,6 +335,10 @@ int ub_mtiles(const asap_moe_config& c, long long nk, int bm = asap::kGemmBM) {
   return asap::ceil_div(nk, bm) + static_cast<int>(std::min<long long>(c.n_experts, nk));
 }
 
+// Rows of the output boxes the bf16 GEMM epilogues store with TMA (one epilogue
+// warp's 32 rows).
+constexpr uint32_t kStoreRows = 32;
+
 // GEMM1: h = silu(X Wg^T) * (X Wu^T) on the routed segments, plus the shared
 // expert on x (problem 1 of the same launch).
 // counter: a zeroed int the launch claims its tiles from (nullptr: static order).
@@ -349,14 +353,19 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
   const bool pair = use_pair(h, nk, c.inter / 128, sh ? n : 0, c.shared_inter / 128);
   const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
-  CUtensorMap maps[2];
+  CUtensorMap maps[4];
   if (!asap::encode_tmap_bf16(&maps[0], x_perm, nk, c.hidden, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "x_perm: " + err);
+  if (!asap::encode_tmap_bf16(&maps[2], hbuf, nk, c.inter, kStoreRows, &err))
+    return fail(ASAP_ERR_INVALID, "h: " + err);
   if (sh) {
     if (!asap::encode_tmap_bf16(&maps[1], x, n, c.hidden, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "x: " + err);
+    if (!asap::encode_tmap_bf16(&maps[3], hsh, n, c.shared_inter, kStoreRows, &err))
+      return fail(ASAP_ERR_INVALID, "h_shared: " + err);
   } else {
     maps[1] = maps[0];
+    maps[3] = maps[2];
   }
   asap::GemmArgs a{};
   a.lref = lref(h, layer);
@@ -399,14 +408,19 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   const bool pair = use_pair(h, nk, c.hidden / asap::kGemmBN, sh ? n : 0, c.hidden / asap::kGemmBN);
   const int bm = pair ? 2 * asap::kGemmBM : asap::kGemmBM;
   std::string err;
-  CUtensorMap maps[2];
+  CUtensorMap maps[4];
   if (!asap::encode_tmap_bf16(&maps[0], hbuf, nk, c.inter, asap::kGemmBM, &err))
     return fail(ASAP_ERR_INVALID, "h: " + err);
+  if (!asap::encode_tmap_bf16(&maps[2], y_perm, nk, c.hidden, kStoreRows, &err))
+    return fail(ASAP_ERR_INVALID, "y_perm: " + err);
   if (sh) {
     if (!asap::encode_tmap_bf16(&maps[1], hsh, n, c.shared_inter, asap::kGemmBM, &err))
       return fail(ASAP_ERR_INVALID, "h_shared: " + err);
+    if (!asap::encode_tmap_bf16(&maps[3], y_sh, n, c.hidden, kStoreRows, &err))
+      return fail(ASAP_ERR_INVALID, "y_shared: " + err);
   } else {
     maps[1] = maps[0];
+    maps[3] = maps[2];
   }
   asap::GemmArgs a{};
   a.lref = lref(h, layer);

@@ -98,18 +98,32 @@ __host__ __device__ constexpr size_t smem_bytes() {
 }
 
 
-// One round of a warp's coalesced stores: lane l holds 8 chunks of 16 bytes
-// (pk, 32 words) of its row l.  Every lane writes them to the warp's 4 KB
-// staging buffer (chunk j of row r at slot j ^ (r % 8), so neither side of
-// the exchange has bank conflicts), then lanes 8u .. 8u+7 store the 8 chunks
-// of rows u, u + 4, ...: each store instruction writes four rows x 128
-// contiguous bytes instead of 32 rows x 16 bytes.  Rows from ``valid_rows``
-// on are not stored.  out: the warp's first row at the round's first column.
+// One round of a warp's stores: lane l holds 8 chunks of 16 bytes (pk, 32
+// words) of its row l.  Every lane writes them to the warp's 4 KB staging
+// buffer, chunk j of row r at slot j ^ (r % 8): the layout of a [32 rows, 64
+// columns] bf16 box under the 128-byte swizzle (the buffer is 1024-byte
+// aligned).  A warp whose 32 rows all belong to the tile (valid_rows == 32)
+// stores the buffer with one TMA store of that box (tm, column x, row y);
+// otherwise lanes 8u .. 8u+7 store the 8 chunks of rows u, u + 4, ... below
+// valid_rows, each store instruction four rows x 128 contiguous bytes (out:
+// the warp's first row at the round's first column).  The buffer is rewritten
+// only after the previous round's TMA store has read it.
 __device__ __forceinline__ void store_round(const uint32_t* pk, uint4* stage, int lane, uint16_t* out, long long ldo,
-                                            int valid_rows) {
+                                            int valid_rows, const CUtensorMap* tm, int x, int y) {
+  if (lane == 0) bulk_wait_group_read0();
+  __syncwarp();
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     stage[lane * 8 + (j ^ (lane & 7))] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+  if (valid_rows == 32) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tm, smem_u32(stage), x, y);
+      bulk_commit_group();
+    }
+    return;
+  }
   __syncwarp();
   const int ru = lane >> 3, cu = lane & 7;
   uint16_t* dst = out + ru * ldo + cu * 8;
@@ -166,7 +180,8 @@ __device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t
 // loop).  The fp32 epilogue (router logits) stores as it reads.
 template <int EPI, bool EARLY>
 __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr, int row,
-                                              uint32_t tempty, uint4* stage, int lane, int lanes = 32) {
+                                              uint32_t tempty, uint4* stage, int lane, int lanes,
+                                              const CUtensorMap* tm) {
   // output row of the tile's row 0; split-K slices of problem 0 write separate planes
   const long long orow_t = static_cast<long long>(T.a_row) + (T.p1 ? 0 : T.split * a.split_rows0);
   if constexpr (EPI == EPI_F32) {
@@ -195,6 +210,8 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
     uint16_t* out = static_cast<uint16_t*>(T.p1 ? a.out1 : a.out0);
     const long long ldo = T.p1 ? a.ldo1 : a.ldo0;
     uint16_t* out_w = out + (orow_t + wrow0) * ldo + static_cast<long long>(T.n_tile) * kOutCols;
+    // the warp's box origin for the TMA stores: column of the round, row
+    const int bx = T.n_tile * kOutCols, by = static_cast<int>(orow_t + wrow0);
     if constexpr (EARLY) {
       uint32_t pk[kRounds * 32];
 #pragma unroll
@@ -202,13 +219,14 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
       tc_fence_before();
       mbar_arrive(tempty);
 #pragma unroll
-      for (int rd = 0; rd < kRounds; ++rd) store_round(pk + 32 * rd, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+      for (int rd = 0; rd < kRounds; ++rd)
+        store_round(pk + 32 * rd, stage, lane, out_w + 64 * rd, ldo, valid_rows, tm, bx + 64 * rd, by);
     } else {
 #pragma unroll 1
       for (int rd = 0; rd < kRounds; ++rd) {
         uint32_t pk[32];
         tmem_to_bf16_64<EPI>(taddr, 64 * rd, pk);
-        store_round(pk, stage, lane, out_w + 64 * rd, ldo, valid_rows);
+        store_round(pk, stage, lane, out_w + 64 * rd, ldo, valid_rows, tm, bx + 64 * rd, by);
       }
       tc_fence_before();
       mbar_arrive(tempty);
@@ -218,8 +236,9 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
 
 template <int EPI, bool PAIR>
 __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
-    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
-                        const __grid_constant__ CUtensorMap tmA1, const GemmArgs args) {
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
+                        const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
+                        const GemmArgs args) {
   using C = Gemm<EPI, PAIR>;
   constexpr int SA = C::SA, SB = C::SB, A_BYTES = C::A_BYTES, BMT = C::BMT;
   static_assert(8 * (2 * SA + 2 * SB + 5) + kTileQBytes + 8 <= kBarBytes, "barrier area");
@@ -233,7 +252,11 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
   uint8_t* gbase = smem_raw;
   const uint32_t sA = base;
   const uint32_t sB = base + SA * A_BYTES;
-  uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES;
+  // bf16 store staging, kStageWarpBytes per epilogue warp, right after the
+  // rings so that every warp's buffer is 1024-byte aligned (the 128-byte
+  // swizzle of its TMA stores); then the barriers and the schedule table
+  uint4* stage_all = reinterpret_cast<uint4*>(gbase + SA * A_BYTES + SB * B_BYTES);
+  uint8_t* bar_area = gbase + SA * A_BYTES + SB * B_BYTES + stage_bytes<EPI, PAIR>();
   const uint32_t bar0 = smem_u32(bar_area);
   // mbarriers (8 bytes each): fullA[SA], emptyA[SA], fullB[SB], emptyB[SB],
   // tfull[2], tempty[2], drain, tile queue full[kTileQ], empty[kTileQ]
@@ -247,9 +270,7 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
   const uint32_t tq_base = bar0 + 8u * (2 * SA + 2 * SB + 5);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * (2 * SA + 2 * SB + 5) + kTileQBytes);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  // bf16 store staging, kStageWarpBytes per epilogue warp (16-byte aligned)
-  uint4* stage_all = reinterpret_cast<uint4*>(bar_area + kBarBytes);
-  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes + stage_bytes<EPI, PAIR>());
+  Sched* sch = reinterpret_cast<Sched*>(bar_area + kBarBytes);
   // consumers of each queued tile id: A producer, MMA issuer, the epilogue warps
   constexpr int kTileQConsumers = 2 + C::EPI_WARPS;
 
@@ -486,12 +507,15 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
         // arrives on tempty itself
         epilogue_tile<EPI, PAIR && EPI == EPI_BF16>(T, args, taddr, erow, tempty_bar(acc),
                                                     stage_all + (warp - 2) * (kStageWarpBytes / 16), lane,
-                                                    m64 ? 16 : 32);
+                                                    m64 ? 16 : 32, T.p1 ? &tmO1 : &tmO0);
       } else {
         tc_fence_before();
         mbar_arrive(tempty_bar(acc));
       }
     }
+    // the warp's TMA stores are complete before its staging buffer goes away
+    if (lane == 0) bulk_wait_group0();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -511,7 +535,7 @@ cudaError_t set_attr() {
 template <int EPI, bool PAIR>
 void launch(const CUtensorMap* maps, const GemmArgs& args, int grid, cudaStream_t stream) {
   grouped_gemm_kernel<EPI, PAIR><<<dim3(grid), dim3(Gemm<EPI, PAIR>::kThreads), smem_bytes<EPI, PAIR>(), stream>>>(
-      maps[0], maps[1], args);
+      maps[0], maps[1], maps[2], maps[3], args);
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

@@ -76,8 +76,10 @@ constexpr int kGemmBK = 64;
 
 cudaError_t gemm_set_attributes();
 // maps: A0, A1 (A1 may repeat A0 when m1 == 0), encoded for boxes of 128 rows,
-// or 256 rows with pair; the B maps come from the layer table.  pair: tiles of
-// two 128-row m-tiles sharing the weight boxes (EPI_SWIGLU and EPI_BF16).
+// or 256 rows with pair; then O0, O1, the bf16 outputs out0 / out1 encoded for
+// boxes of 32 rows (O1 may repeat O0 when m1 == 0; EPI_F32 ignores both).  The
+// B maps come from the layer table.  pair: tiles of two 128-row m-tiles
+// sharing the weight boxes (EPI_SWIGLU and EPI_BF16).
 cudaError_t gemm_launch(int epi, bool pair, const CUtensorMap* maps, const GemmArgs& args, int grid,
                         cudaStream_t stream);
 // Encode a 2-D row-major bf16 tensor [rows, cols] for 128-byte-swizzled
