@@ -287,6 +287,8 @@ def run_ours(args, dist):
     main = torch.cuda.current_stream()
     tokens_per_step = sum(mbs)
 
+    nvtx = torch.cuda.nvtx.range  # named ranges for a trace of the run (no cost without a tracing tool)
+
     def step():
         ev = torch.cuda.Event()
         ev.record(main)
@@ -296,8 +298,9 @@ def run_ours(args, dist):
         for s in streams:
             main.wait_stream(s)
 
-    for _ in range(args.warmup):
-        step()
+    with nvtx("warm-up steps"):
+        for _ in range(args.warmup):
+            step()
     torch.cuda.synchronize()
     dist.barrier()
     torch.cuda.synchronize()
@@ -306,8 +309,10 @@ def run_ours(args, dist):
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(main)
-    for _ in range(args.steps):
-        step()
+    with nvtx("timed steps"):
+        for _ in range(args.steps):
+            with nvtx("step"):
+                step()
     t_end.record(main)
     torch.cuda.synchronize()
     dist.barrier()
@@ -345,7 +350,8 @@ def run_ours(args, dist):
     }
 
     # ---------------- per-kernel timings, each on the stream it runs on
-    kern = kernel_pass(args, h, cfg, xs, dev)
+    with nvtx("per-kernel pass"):
+        kern = kernel_pass(args, h, cfg, xs, dev)
     peaks, peaks_src = load_peaks()
     result["kernels"] = kern["table"]
     tensor_peak = None
@@ -364,21 +370,25 @@ def run_ours(args, dist):
         "note": "algorithmic FLOPs of both grouped GEMMs (routed + shared) over their event-timed durations"}
 
     # ---------------- all micro-batches in one pass (one grouped GEMM per weight matrix)
-    result["aggregated"] = aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist)
+    with nvtx("host-aggregated pass"):
+        result["aggregated"] = aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist)
 
     # ---------------- the device decides the sets: mailbox posts and service rounds
     if not args.no_mailbox:
-        result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
-                                         latest_first=args.mailbox_latest_first,
-                                         pipelined=args.mailbox_back_to_back)
+        with nvtx("mailbox pass"):
+            result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
+                                             latest_first=args.mailbox_latest_first,
+                                             pipelined=args.mailbox_back_to_back)
 
     # ---------------- per-micro-batch latency of the per-stream step
-    result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
+    with nvtx("latency pass"):
+        result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
     if cfg.zipf_s is not None:
         result["expert_popularity"] = popularity(h, cfg, xs, dev)
 
     # ---------------- end to end through host buffers
-    result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
+    with nvtx("end-to-end pass"):
+        result["e2e"] = e2e_pass(args, h, cfg, xs, outs, wss, streams, main, dist)
 
     # ---------------- the other workloads, briefly (N = 1 only)
     if dist.world == 1 and not args.no_extra_workloads:
