@@ -380,6 +380,17 @@ def run_ours(args, dist):
                                              latest_first=args.mailbox_latest_first,
                                              pipelined=args.mailbox_back_to_back)
 
+    # the same fraction where several micro-batches share the GEMMs: sets the
+    # device chose (mailbox rounds) and sets the host chose (aggregated call)
+    gtf = result["grouped_gemm_tensor_frac"]
+    gtf["note"] += ("; per-stream launches (one micro-batch each) here, the mailbox rounds' and the "
+                    "host-aggregated launches' in mailbox_* and aggregated_*")
+    for leg in ("mailbox", "aggregated"):
+        r = result.get(leg) or {}
+        for k in ("of_burst_measured", "of_sustained_measured"):
+            if "grouped_gemm_frac_" + k in r:
+                gtf[f"{leg}_{k}"] = r["grouped_gemm_frac_" + k]
+
     # ---------------- per-micro-batch latency of the per-stream step
     with nvtx("latency pass"):
         result["latency"] = latency_pass(args, h, xs, outs, wss, streams, main)
