@@ -183,9 +183,11 @@ bool fused_route(asap_moe_t h) {
 // zeroes tile_counters (nullable); without, hist columns [chunk0, chunk0 +
 // ceil(n/32)) of n_chunks_total are left for one scan over several
 // micro-batches.
+// narrow: no cluster; each CTA computes its tile's K slices one after the
+// other (same logits bits), so concurrent routes share the GPU in one wave.
 int run_route_fused(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* hist, int chunk0,
                     int n_chunks_total, int32_t* ticket, int32_t* counts, int32_t* offsets, int32_t* chunk_base,
-                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st);
+                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st, bool narrow = false);
 
 // Router logits as ``splits`` planes of partial sums [splits][n][E] (planes
 // are added in order by the consumer); splits == 1 writes the logits.
@@ -226,7 +228,7 @@ int run_router_logits(asap_moe_t h, const void* x, int n, float* logits, int spl
 
 int run_route_fused(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, int32_t* hist, int chunk0,
                     int n_chunks_total, int32_t* ticket, int32_t* counts, int32_t* offsets, int32_t* chunk_base,
-                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st) {
+                    int32_t* tile_counters, const int32_t* layer, cudaStream_t st, bool narrow) {
   const asap_moe_config& c = h->cfg;
   CUtensorMap tmx;
   std::string err;
@@ -236,7 +238,9 @@ int run_route_fused(asap_moe_t h, const void* x, int n, int32_t* idx, float* w, 
   a.status = h->status;
   a.n = n;
   a.k_iters = c.hidden / asap::kGemmBK;
-  a.splits = router_splits(h, n);
+  const int splits = router_splits(h, n);
+  a.splits = narrow ? 1 : splits;
+  a.seq_slices = narrow ? splits : 1;
   a.top_k = c.top_k;
   a.n_groups = c.n_groups;
   a.topk_groups = c.topk_groups;
@@ -1396,7 +1400,7 @@ ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const voi
     // are the slot's, scanned later together with the other claimed posts
     if (fused_route(h)) {
       if ((r = run_route_fused(h, x, n, idx, w, hist, chunk0, chunks_total, nullptr, nullptr, nullptr, nullptr,
-                               nullptr, layer, st)) != ASAP_OK)
+                               nullptr, layer, st, /*narrow=*/true)) != ASAP_OK)
         return r;
     } else {
       const int splits = router_splits(h, n);

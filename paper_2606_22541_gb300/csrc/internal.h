@@ -166,6 +166,10 @@ struct RouteFusedArgs {
   LayerRef lref;  // router weights: table[layer].map[MAP_ROUTER]; selection bias
   uint32_t* status;
   int n, k_iters, splits;
+  // seq_slices > 1 (with splits == 1): one CTA per tile computes the partial
+  // logits of that many K slices one after the other and adds them in slice
+  // order, the bits of a cluster of seq_slices CTAs without the cluster
+  int seq_slices;
   int top_k, n_groups, topk_groups;
   float route_scale;
   int32_t* idx;

@@ -8,6 +8,12 @@
 //    logits of the tile over K slice r (the same slices as the standalone
 //    router GEMM): TMA rings of x [128 x 64] and router-weight [256 x 64]
 //    boxes, tcgen05.mma kind::f16 M=128 N=256 into one TMEM accumulator.
+//  - Or (seq_slices > 1, no cluster) one CTA computes the slices one after
+//    the other: slice 0 into TMEM columns 0.., each later slice into columns
+//    256.., which the epilogue warps add into the first buffer (TMEM load,
+//    fp32 add, TMEM store) while the next slice streams -- the same sum in
+//    the same order, so the same logits, on a quarter of the SMs.  Several
+//    micro-batches routed at once then run side by side in one wave.
 //  - Each 32-token quarter q of the tile is gated by CTA q % splits.  The
 //    epilogue warps read their quarter from TMEM and store it into the owning
 //    CTA's shared memory through distributed shared memory, one slot per K
@@ -61,9 +67,9 @@ constexpr int kScratchEnd = kWarpSumOff + 40 * 4;
 static_assert(kScratchEnd <= kRingBytes, "the gate's scratch overlays the operand rings");
 static_assert(kThreads == kRouteExperts, "the scan gives one thread per expert");
 constexpr int kBarOff = kRingBytes;
-// mbarriers fullA[kRA], emptyA[kRA], fullB[kRB], emptyB[kRB], tfull, drain;
-// then the TMEM address, abort flag, last-CTA flag and the bias pointer
-constexpr int kNumBars = 2 * kRA + 2 * kRB + 2;
+// mbarriers fullA[kRA], emptyA[kRA], fullB[kRB], emptyB[kRB], tfull, drain,
+// bfree; then the TMEM address, abort flag, last-CTA flag and the bias pointer
+constexpr int kNumBars = 2 * kRA + 2 * kRB + 3;
 constexpr int kBarBytes = 8 * kNumBars + 32;
 constexpr size_t kSmem = kRingBytes + kBarBytes;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kGemmBM, kGemmBN);
@@ -125,6 +131,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto emptyB = [&](int s) { return bar0 + 8u * (2 * kRA + kRB + s); };
   const uint32_t tfull = bar0 + 8u * (2 * kRA + 2 * kRB);
   const uint32_t drain = tfull + 8u;
+  const uint32_t bfree = drain + 8u;  // sequential slices: the second TMEM buffer was added in
+  // K slices computed one after the other by this CTA (1 with a cluster)
+  const int nseq = splits == 1 ? max(a.seq_slices, 1) : 1;
+  const uint32_t tmem_cols = nseq > 1 ? 2 * kGemmBN : kGemmBN;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_area + 8 * kNumBars);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
@@ -149,6 +159,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       mbar_init(tfull, 1);
       mbar_init(drain, 1);
+      mbar_init(bfree, 128);  // the four epilogue warps
       *abort_flag = 0;
       *last_flag = 0;
       *acc_bad = aligned ? 0 : 1;
@@ -158,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!aligned) record_status(a.status, ST_SMEM_ALIGN);
     }
   } else if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), kGemmBN);
+    tmem_alloc(smem_u32(tmem_slot), tmem_cols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -206,17 +217,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     int sa = 0, sb = 0;
     uint32_t pa = 0, pb = 0;
     bool good = true, issued = false;
+    // slice q of nseq covers k-blocks [k_iters q / nseq, k_iters (q + 1) / nseq)
+    // (the bounds of a cluster's CTAs); slice 0 accumulates into TMEM columns
+    // 0.., the later ones into columns 256.., which the epilogue warps add into
+    // the first buffer before the next slice may start there
+    int q = 0, q_start = kb0;
+    int q_end = nseq > 1 ? static_cast<int>(static_cast<long long>(a.k_iters) / nseq) : kb1;
     for (int kb = kb0; kb < kb1; ++kb) {
+      if (kb == q_start && q >= 2 && !mbar_wait(bfree, (q - 2) & 1, abort_flag)) {
+        good = false;
+        break;
+      }
       if (!mbar_wait(fullA(sa), pa, abort_flag) || !mbar_wait(fullB(sb), pb, abort_flag)) {
         good = false;
         break;
       }
       tc_fence_after();
       const uint32_t a_addr = sA + sa * kABytes, b_addr = sB + sb * kBBytes;
+      const uint32_t d = tmem_base + (q == 0 ? 0u : static_cast<uint32_t>(kGemmBN));
 #pragma unroll
       for (int kk = 0; kk < kGemmBK / 16; ++kk)
-        tc_mma_bf16(tmem_base, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kIdesc,
-                    (kb > kb0 || kk > 0) ? 1u : 0u);
+        tc_mma_bf16(d, smem_desc_sw128(a_addr + kk * 32), smem_desc_sw128(b_addr + kk * 32), kIdesc,
+                    (kb > q_start || kk > 0) ? 1u : 0u);
       issued = true;
       tc_commit(emptyA(sa));
       tc_commit(emptyB(sb));
@@ -227,6 +249,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (++sb == kRB) {
         sb = 0;
         pb ^= 1u;
+      }
+      if (kb + 1 == q_end && q + 1 < nseq) {
+        tc_commit(tfull);  // slice q complete
+        ++q;
+        q_start = kb + 1;
+        q_end = static_cast<int>(static_cast<long long>(a.k_iters) * (q + 1) / nseq);
       }
     }
     if (good) {
@@ -243,6 +271,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= 2 && warp <= 5) {
     if (aligned) {
       ok = __all_sync(kFull, mbar_wait(tfull, 0, abort_flag));
+      // sequential slices: add slice q (columns 256..) into the sum of the
+      // slices before it (columns 0..), in slice order, each warp its 32 lanes
+      const uint32_t lanes = tmem_base + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+      for (int qs = 1; ok && qs < nseq; ++qs) {
+        ok = __all_sync(kFull, mbar_wait(tfull, qs & 1, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < kGemmBN; c += 16) {
+          uint32_t acc[16], part[16];
+          tmem_ld16(lanes + c, acc);
+          tmem_ld16(lanes + kGemmBN + c, part);
+          tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[i] = __float_as_uint(__uint_as_float(acc[i]) + __uint_as_float(part[i]));
+          tmem_st16(lanes + c, acc);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(bfree);
+      }
       if (!ok && lane == 0) {
         *abort_flag = 1;
         *acc_bad = 1;
@@ -527,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kGemmBN);
+    tmem_dealloc(tmem_base, tmem_cols);
   }
 }
 
@@ -542,7 +591,8 @@ cudaError_t launch_route_fused(const CUtensorMap& tmX, const RouteFusedArgs& a, 
   if (a.n <= 0) return cudaSuccess;
   if (!(a.splits == 1 || a.splits == 2 || a.splits == 4) || !(a.n_groups == 1 || a.n_groups == 2 ||
                                                               a.n_groups == 4 || a.n_groups == 8) ||
-      a.top_k < 1 || a.top_k > kMaxTopK || a.k_iters < a.splits)
+      a.top_k < 1 || a.top_k > kMaxTopK || a.k_iters < a.splits ||
+      !(a.seq_slices <= 1 || (a.splits == 1 && (a.seq_slices == 2 || a.seq_slices == 4) && a.k_iters >= a.seq_slices)))
     return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(ceil_div(a.n, kGemmBM) * a.splits);
