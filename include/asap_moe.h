@@ -366,8 +366,10 @@ int asap_moe_layer_batched_dyn(asap_moe_t h, const int32_t* layer_id, int32_t co
  * with the MoE side serving DP groups out of order (Section 3.3).
  *
  *  - A DP group's stream POSTS a micro-batch into its slot: the post routes
- *    it (exactly as asap_moe_route) into the slot's region and then sets the
- *    slot's ready flag, an epoch, with a release store.
+ *    it (the bits of asap_moe_route; for E = 256 with grouped gating one CTA
+ *    per 128-token tile instead of a cluster, so posts made together route
+ *    side by side) into the slot's region and then sets the slot's ready
+ *    flag, an epoch, with a release store.
  *  - The MoE stream SERVES: a service round claims, on the device, every
  *    post whose flag is set and that has not been served when the round
  *    starts; dispatches all claimed posts into one expert-major buffer (the
