@@ -777,6 +777,10 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     for si in range(args.kernel_steps):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_mb)]
         rb, _ = api.asap_moe_mailbox_rounds(m)
+        # as in the timed steps, every post is enqueued before the device
+        # reaches the step (a step right after a host synchronize would
+        # otherwise route its first post before the host has made the others)
+        head_start(main)
         step(base + si, evs)
         torch.cuda.synchronize()
         ra, cl = api.asap_moe_mailbox_rounds(m)
