@@ -52,6 +52,8 @@ def parse_args():
                     help="skip the brief per-stream and aggregated timing of the other workloads")
     ap.add_argument("--mailbox-latest-first", action="store_true",
                     help="start each step's mailbox rounds from its last post instead of its first")
+    ap.add_argument("--mailbox-depth", type=int, default=2,
+                    help="mailbox slots per micro-batch stream: the posts a DP group may have in flight")
     ap.add_argument("--mailbox-back-to-back", action="store_true",
                     help="mailbox leg without a barrier between steps")
     ap.add_argument("--mailbox-priority", type=int, default=0,
@@ -731,16 +733,17 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     from paper_2606_22541_gb300 import api
 
     n_mb = len(xs)
-    m = api.asap_moe_mailbox_create(h, 2 * n_mb, max(x.shape[0] for x in xs))
+    depth = max(1, args.mailbox_depth)
+    m = api.asap_moe_mailbox_create(h, depth * n_mb, max(x.shape[0] for x in xs))
     # --mailbox-priority: the DP groups' streams above the MoE stream
     hi = torch.cuda.Stream.priority_range()[1] if args.mailbox_priority else 0
     producers = [torch.cuda.Stream(priority=hi) for _ in xs]
     server = torch.cuda.Stream()
     main = torch.cuda.current_stream()
-    outs = [[torch.empty_like(x) for x in xs] for _ in range(2)]
+    outs = [[torch.empty_like(x) for x in xs] for _ in range(depth)]
 
     def step(si, gemm_events=None):
-        b = si % 2
+        b = si % depth
         ev = torch.cuda.Event()
         ev.record(main)
         eps = []
@@ -811,6 +814,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "gemm_timing_nonempty_rounds_per_step": sum(nonempty) / len(nonempty),
             "serve_order": "latest post first" if latest_first else "post order",
             "steps": "back to back, no barrier between steps" if pipelined else "one barrier per step",
+            "slots_per_stream": depth,
             "posting_stream_priority": "highest" if args.mailbox_priority else "default",
             "note": "asap_moe_mailbox_post from one stream per micro-batch, asap_moe_mailbox_serve for every post "
                     "right after it on one MoE stream; the rounds claim on the device whatever has been published"}
