@@ -167,6 +167,31 @@ def test_serve_calls_from_several_streams():
     m.close()
 
 
+def test_post_routes_match_layer_routes_at_every_slice_count():
+    """A post routes with one CTA per tile adding its K slices in turn; the
+    layer call routes with a cluster per tile (one CTA per slice).  Sizes
+    chosen so the slice count is 4 (1, 33 and 700 tokens), 2 (5000) and 1
+    (10000) at H = 2048: every post's output equals asap_moe_layer's bit for
+    bit, all five served by one round."""
+    cfg = inputs.small_variant(DSV3, name="mbox_slices", hidden=2048, inter=128, shared_inter=128,
+                               microbatches=[1, 33, 700, 5000, 10000])
+    c = Case.get(cfg)
+    n = len(c.xs)
+    m = api.asap_moe_mailbox_create(c.h, n, max(cfg.microbatches))
+    streams = [torch.cuda.Stream() for _ in range(n)]
+    outs = [torch.full_like(x, 9.0) for x in c.xs]
+    eps = [api.asap_moe_mailbox_post(m, i, x, o, stream=s) for i, (x, o, s) in enumerate(zip(c.xs, outs, streams))]
+    torch.cuda.synchronize()
+    for i in range(n):
+        api.asap_moe_mailbox_serve(m, i, eps[i])
+    torch.cuda.synchronize()
+    assert api.asap_moe_mailbox_rounds(m) == (n, [n] + [0] * (n - 1))
+    for a, b in zip(c.ref, outs):
+        assert same_bits(a, b)
+    assert_clean(c.h)
+    m.close()
+
+
 def test_mailbox_output_against_oracle():
     """The chain to the oracle directly: one round serving three posts of the
     DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
