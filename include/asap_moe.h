@@ -34,6 +34,11 @@
  *    thread-local message describing the last failure of this thread.
  *  - A handle is immutable after create; concurrent calls on different
  *    streams with different workspaces are safe.
+ *  - A handle belongs to the device that was current at create.  Enqueuing
+ *    calls launch on the caller's current device, so they must be made with
+ *    that device current and a stream (or NULL, its default stream) of it;
+ *    create, destroy, status and the mailbox's create, destroy and rounds
+ *    select the handle's device themselves.
  *  - Kernels that detect a bad index or a wait that exceeds its time limit
  *    record it in a device status word of the handle instead of trapping;
  *    asap_moe_status reads and clears it.
