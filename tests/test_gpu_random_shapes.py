@@ -18,7 +18,7 @@ from _helpers import bf16_to_f64, weights_f64, compare_rows, routing_check
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda"
-N_CASES = 16
+N_CASES = 48
 
 
 def random_config(i):
