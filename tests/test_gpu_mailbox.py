@@ -192,6 +192,46 @@ def test_post_routes_match_layer_routes_at_every_slice_count():
     m.close()
 
 
+@pytest.mark.parametrize("cfg", [DS, MX], ids=lambda c: c.name)
+def test_randomised_posts_sizes_slots_and_streams(cfg):
+    """120 posts of random sizes (0, 1, 31-33 around a chunk boundary, up to
+    the slot's capacity) into random slots from three producer streams, each
+    behind a random GPU sleep, each served at once from one of two server
+    streams: every output bit-identical to asap_moe_layer."""
+    c = Case.get(cfg)
+    rng = np.random.default_rng(321)
+    T = max(cfg.microbatches)
+    m = api.asap_moe_mailbox_create(c.h, 5, T)
+    prods = [torch.cuda.Stream() for _ in range(3)]
+    servers = [torch.cuda.Stream() for _ in range(2)]
+    inflight = []
+    for it in range(120):
+        s = int(rng.integers(0, 5))
+        n = int(rng.choice([0, 1, 31, 32, 33, int(rng.integers(1, T + 1))]))
+        x = inputs.make_tokens(cfg, n, 100 + it, DEV) if n else torch.empty((0, cfg.hidden), dtype=torch.bfloat16,
+                                                                            device=DEV)
+        ref = torch.empty_like(x)
+        if n:
+            api.asap_moe_layer(c.h, x, ref, api.workspace(c.h, n))
+        out = torch.full_like(x, 3.0)
+        p = prods[int(rng.integers(0, 3))]
+        with torch.cuda.stream(p):
+            torch.cuda._sleep(int(rng.integers(0, 100_000)))
+        ep = api.asap_moe_mailbox_post(m, s, x, out, stream=p)
+        api.asap_moe_mailbox_serve(m, s, ep, stream=servers[int(rng.integers(0, 2))])
+        inflight.append((out, ref))
+        if it % 40 == 39:
+            torch.cuda.synchronize()
+            assert all(same_bits(o, r) for o, r in inflight)
+            inflight.clear()
+    torch.cuda.synchronize()
+    assert all(same_bits(o, r) for o, r in inflight)
+    rounds, claimed = api.asap_moe_mailbox_rounds(m)
+    assert rounds == 120 and sum(claimed) == 120
+    assert_clean(c.h)
+    m.close()
+
+
 def test_mailbox_output_against_oracle():
     """The chain to the oracle directly: one round serving three posts of the
     DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
