@@ -7,7 +7,7 @@ import torch
 
 import oracle
 from paper_2606_22541_gb300 import api, inputs
-from paper_2606_22541_gb300.configs import DSV3_FP8
+from paper_2606_22541_gb300.configs import DSV3_FP8, LayerConfig
 
 from _helpers import bf16_to_f64, routing_check, sample_tokens
 
@@ -200,6 +200,66 @@ def test_fp8_full_size_streams_against_oracle():
         norm, worst = compare_fp8(g[lo:hi], ref[lo:hi])
         print(f"[fp8 mb{i}] {hi - lo} tokens: normwise {norm:.3e} elementwise {worst:.3e}")
         lo = hi
+    code, word = api.asap_moe_status(h)
+    assert code == 0 and word == 0
+    h.close()
+
+
+def random_fp8_config(i):
+    """A seeded random FP8 layer: 8 to 256 experts, the three gating rules,
+    H and I multiples of the 128-channel scale blocks, with and without a
+    shared expert, ragged token counts."""
+    rng = np.random.default_rng(9000 + i)
+    E = int(rng.choice([8, 16, 32, 64, 256]))
+    gating = str(rng.choice(["softmax", "softmax_renorm", "sigmoid_grouped"]))
+    k = int(rng.integers(1, min(8, E) + 1))
+    H = int(rng.choice([256, 512, 1024]))
+    I = int(rng.choice([128, 256]))
+    sh = int(rng.integers(0, 2))
+    Is = int(rng.choice([128, 256])) if sh else 0
+    ng, tg = 1, 1
+    if gating == "sigmoid_grouped":
+        ng = int(rng.choice([g for g in (1, 2, 4, 8) if E % g == 0 and E // g >= 2]))
+        tg = int(rng.integers(-(-k // (E // ng)), ng + 1))
+    n = int(rng.integers(1, 900))
+    return LayerConfig(f"f8rand{i}", hidden=H, n_experts=E, top_k=k, inter=I, n_shared=sh, shared_inter=Is,
+                       gating=gating, n_groups=ng, topk_groups=tg, route_scale=float(rng.choice([1.0, 2.5])),
+                       dtype="fp8_e4m3_block128", microbatches=[n], seed=9500 + i)
+
+
+@pytest.mark.parametrize("cfg", [random_fp8_config(i) for i in range(12)], ids=lambda c: c.name)
+def test_fp8_random_shapes_against_oracle(cfg):
+    """The FP8 layer on seeded random shapes against the oracle's FP8
+    emulation, on up to 64 decided tokens (40 more seeds were checked once)."""
+    n, k, H = cfg.microbatches[0], cfg.top_k, cfg.hidden
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, n)
+    x = inputs.make_tokens(cfg, n, 0, DEV)
+    out = torch.empty_like(x)
+    api.asap_moe_layer(h, x, out, api.workspace(h, n))
+    torch.cuda.synchronize()
+    ocfg = cfg.oracle_cfg()
+    wr = bf16_to_f64(w["router_w"])
+    shared = shared_expert(w) if cfg.n_shared else None
+    xf = bf16_to_f64(x)
+    L = oracle.router_logits(xf, wr)
+    idx_ref, w_ref = oracle.route(L, ocfg)
+    eps = oracle.logit_error_bound(xf, wr)
+    dec = np.array([oracle.token_decided(L[t], eps[t], ocfg) for t in range(n)])
+    cache = {}
+
+    def get_expert(e):
+        if e not in cache:
+            cache[e] = dequant_expert(w, e)
+        return cache[e]
+
+    pick = np.nonzero(dec)[0][:64]
+    ref = np.zeros((len(pick), H))
+    for j, t in enumerate(pick):
+        wg, wu, wd = zip(*[get_expert(int(e)) for e in idx_ref[t]])
+        ref[j] = oracle.moe_layer_tokens_fp8(xf[t:t + 1], np.arange(k)[None], w_ref[t:t + 1], list(wg), list(wu),
+                                             list(wd), shared)[0]
+    compare_fp8(bf16_to_f64(out)[pick], ref)
     code, word = api.asap_moe_status(h)
     assert code == 0 and word == 0
     h.close()
