@@ -742,9 +742,11 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     main = torch.cuda.current_stream()
     outs = [[torch.empty_like(x) for x in xs] for _ in range(depth)]
 
-    def step(si, gemm_events=None):
+    consumers = [torch.cuda.Stream() for _ in xs]
+
+    def step(si, gemm_events=None, latency=None):
         b = si % depth
-        ev = torch.cuda.Event()
+        ev = torch.cuda.Event(enable_timing=latency is not None)
         ev.record(main)
         eps = []
         for i, (x, p) in enumerate(zip(xs, producers)):
@@ -755,6 +757,16 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             if gemm_events is not None:
                 api.asap_moe_mailbox_time_gemms(m, *gemm_events[r])
             api.asap_moe_mailbox_serve(m, b * n_mb + i, eps[i], stream=server)
+        if latency is not None:
+            # each post's completion as its DP group would see it: a stream of
+            # its own waits for the post's round
+            ends = []
+            for i, c in enumerate(consumers):
+                api.asap_moe_mailbox_wait(m, b * n_mb + i, stream=c)
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(c)
+                ends.append(e)
+            latency.append((ev, ends))
         for i in range(n_mb):
             api.asap_moe_mailbox_wait(m, b * n_mb + i, stream=main)
 
@@ -776,6 +788,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     # the GEMMs of every round, timed with events on the MoE stream
     gemm_ms = []
     nonempty = []
+    lat = []
     base = args.warmup + args.steps
     for si in range(args.kernel_steps):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_mb)]
@@ -784,7 +797,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
         # reaches the step (a step right after a host synchronize would
         # otherwise route its first post before the host has made the others)
         head_start(main)
-        step(base + si, evs)
+        step(base + si, evs, lat)
         torch.cuda.synchronize()
         ra, cl = api.asap_moe_mailbox_rounds(m)
         gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in evs))
@@ -794,6 +807,8 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     m.close()
     if code != 0:
         raise RuntimeError(f"device status word {word:#x} after the mailbox leg")
+    post_ms = [[e0.elapsed_time(e) for e in ends] for e0, ends in lat]
+    post_lat = [sum(v[i] for v in post_ms) / len(post_ms) for i in range(n_mb)]
     flops = kern["gemm_flops"] * n_mb    # per micro-batch mean x micro-batches
     g = sum(gemm_ms) / len(gemm_ms)
     tf = flops / (g / 1e3) / 1e12
@@ -812,6 +827,9 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "grouped_gemm_frac_of_burst_measured": tf / tpk_burst,
             "grouped_gemm_frac_of_sustained_measured": tf / tpk_sus,
             "gemm_timing_nonempty_rounds_per_step": sum(nonempty) / len(nonempty),
+            "post_latency_ms": post_lat,
+            "post_latency_note": "in the GEMM-timing steps: step start (every DP-group stream waits on it) to "
+                                 "each post's completion as seen by a stream of its own",
             "serve_order": "latest post first" if latest_first else "post order",
             "steps": "back to back, no barrier between steps" if pipelined else "one barrier per step",
             "slots_per_stream": depth,
