@@ -52,6 +52,9 @@ def parse_args():
                     help="skip the brief per-stream and aggregated timing of the other workloads")
     ap.add_argument("--mailbox-latest-first", action="store_true",
                     help="start each step's mailbox rounds from its last post instead of its first")
+    ap.add_argument("--mailbox-closed-loop", action="store_true",
+                    help="steps back to back, each DP-group stream posting its next micro-batch only once its "
+                         "previous one has been served (its layer output is back)")
     ap.add_argument("--mailbox-depth", type=int, default=2,
                     help="mailbox slots per micro-batch stream: the posts a DP group may have in flight")
     ap.add_argument("--mailbox-back-to-back", action="store_true",
@@ -380,7 +383,8 @@ def run_ours(args, dist):
         with nvtx("mailbox pass"):
             result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
                                              latest_first=args.mailbox_latest_first,
-                                             pipelined=args.mailbox_back_to_back)
+                                             pipelined=args.mailbox_back_to_back or args.mailbox_closed_loop,
+                                             closed_loop=args.mailbox_closed_loop)
 
     # the same fraction where several micro-batches share the GEMMs: sets the
     # device chose (mailbox rounds) and sets the host chose (aggregated call)
@@ -713,7 +717,8 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
     return res
 
 
-def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_first=False, pipelined=False):
+def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_first=False, pipelined=False,
+                 closed_loop=False):
     """The step's micro-batches posted into a mailbox, each from its own
     stream, and served by rounds on one MoE stream: the host serves every post
     right after making it (no host batching), and each round claims on the
@@ -725,6 +730,9 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
     of its rounds).  latest_first: the step's rounds are started from its
     last post backwards (a server that, knowing of several posts, starts the
     round from the newest; the device still claims whatever is published).
+    closed_loop (with pipelined): a DP group's stream makes its next post only
+    once its previous post has been served, as a prefill pipeline whose next
+    step needs this layer's output would.
     pipelined: no barrier between steps: a step's posts wait only for the
     rounds that served their slots' previous posts (the post's own
     backpressure), so they are made while the previous step's rounds run, as
@@ -752,6 +760,8 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
         for i, (x, p) in enumerate(zip(xs, producers)):
             if not pipelined:
                 p.wait_event(ev)
+            elif closed_loop and si > 0:
+                api.asap_moe_mailbox_wait(m, ((si - 1) % depth) * n_mb + i, stream=p)
             eps.append(api.asap_moe_mailbox_post(m, b * n_mb + i, x, outs[b][i], stream=p))
         for r, i in enumerate(reversed(range(n_mb)) if latest_first else range(n_mb)):
             if gemm_events is not None:
@@ -831,7 +841,8 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "post_latency_note": "in the GEMM-timing steps: step start (every DP-group stream waits on it) to "
                                  "each post's completion as seen by a stream of its own",
             "serve_order": "latest post first" if latest_first else "post order",
-            "steps": "back to back, no barrier between steps" if pipelined else "one barrier per step",
+            "steps": ("closed loop per DP group, no barrier between steps" if closed_loop else
+                      "back to back, no barrier between steps" if pipelined else "one barrier per step"),
             "slots_per_stream": depth,
             "posting_stream_priority": "highest" if args.mailbox_priority else "default",
             "note": "asap_moe_mailbox_post from one stream per micro-batch, asap_moe_mailbox_serve for every post "
