@@ -55,6 +55,9 @@ def parse_args():
     ap.add_argument("--mailbox-closed-loop", action="store_true",
                     help="steps back to back, each DP-group stream posting its next micro-batch only once its "
                          "previous one has been served (its layer output is back)")
+    ap.add_argument("--mailbox-serve-many", action="store_true",
+                    help="one asap_moe_mailbox_serve_many call per step for the step's posts instead of one serve "
+                         "call per post")
     ap.add_argument("--mailbox-depth", type=int, default=2,
                     help="mailbox slots per micro-batch stream: the posts a DP group may have in flight")
     ap.add_argument("--mailbox-back-to-back", action="store_true",
@@ -763,7 +766,13 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             elif closed_loop and si > 0:
                 api.asap_moe_mailbox_wait(m, ((si - 1) % depth) * n_mb + i, stream=p)
             eps.append(api.asap_moe_mailbox_post(m, b * n_mb + i, x, outs[b][i], stream=p))
+        if args.mailbox_serve_many:
+            if gemm_events is not None:
+                api.asap_moe_mailbox_time_gemms(m, *gemm_events[0])
+            api.asap_moe_mailbox_serve_many(m, [b * n_mb + i for i in range(n_mb)], eps, stream=server)
         for r, i in enumerate(reversed(range(n_mb)) if latest_first else range(n_mb)):
+            if args.mailbox_serve_many:
+                break
             if gemm_events is not None:
                 api.asap_moe_mailbox_time_gemms(m, *gemm_events[r])
             api.asap_moe_mailbox_serve(m, b * n_mb + i, eps[i], stream=server)
@@ -810,7 +819,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
         step(base + si, evs, lat)
         torch.cuda.synchronize()
         ra, cl = api.asap_moe_mailbox_rounds(m)
-        gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in evs))
+        gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in (evs[:1] if args.mailbox_serve_many else evs)))
         nonempty.append(sum(1 for c in cl[rb:ra] if c > 0))
     api.asap_moe_mailbox_rounds(m)
     code, word = api.asap_moe_status(h)
@@ -840,7 +849,8 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "post_latency_ms": post_lat,
             "post_latency_note": "in the GEMM-timing steps: step start (every DP-group stream waits on it) to "
                                  "each post's completion as seen by a stream of its own",
-            "serve_order": "latest post first" if latest_first else "post order",
+            "serve_order": ("one serve_many call per step" if args.mailbox_serve_many else
+                            "latest post first" if latest_first else "post order"),
             "steps": ("closed loop per DP group, no barrier between steps" if closed_loop else
                       "back to back, no barrier between steps" if pipelined else "one barrier per step"),
             "slots_per_stream": depth,

@@ -441,6 +441,18 @@ int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int
  * Enqueues only. */
 int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream);
 
+/* One service round on stream for several posts the caller knows were made:
+ * count (1..n_slots) distinct slots with, per slot, the epoch
+ * asap_moe_mailbox_post returned (a post already made; otherwise
+ * ASAP_ERR_INVALID).  The stream waits for all of them, so the round serves
+ * them all (with any other ready post of the first one's layer), and each
+ * listed slot's completion is ordered after this round: a sender that posts
+ * again once its previous post is served (a closed loop) is released by the
+ * round that served it.  No counterpart in the paper, whose MoE side serves
+ * one DP group at a time.  Enqueues only. */
+int asap_moe_mailbox_serve_many(asap_moe_mailbox_t m, int32_t count, const int32_t* slots,
+                                const uint64_t* epochs, void* stream);
+
 /* Make stream wait until the round of the serve call for slot's last post
  * has finished (its out is then complete).  ASAP_ERR_INVALID when no serve
  * call has been made for that post. */

@@ -64,6 +64,7 @@ SIGNATURES = {
     "asap_moe_mailbox_destroy": [_P],
     "asap_moe_mailbox_post": [_P, _I, _P, _I, _P, _P, _P, ctypes.POINTER(ctypes.c_uint64)],
     "asap_moe_mailbox_serve": [_P, _I, ctypes.c_uint64, _P],
+    "asap_moe_mailbox_serve_many": [_P, _I, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_uint64), _P],
     "asap_moe_mailbox_wait": [_P, _I, _P],
     "asap_moe_mailbox_served": [_P, _I, ctypes.POINTER(ctypes.c_uint64)],
     "asap_moe_mailbox_time_gemms": [_P, _P, _P],

@@ -269,6 +269,13 @@ def asap_moe_mailbox_serve(m, slot, epoch, stream=None):
     check("asap_moe_mailbox_serve", lib().asap_moe_mailbox_serve(m.ptr, int(slot), int(epoch), _stream(stream)))
 
 
+def asap_moe_mailbox_serve_many(m, slots, epochs, stream=None):
+    n = len(slots)
+    cs = (ctypes.c_int32 * n)(*[int(v) for v in slots])
+    ce = (ctypes.c_uint64 * n)(*[int(v) for v in epochs])
+    check("asap_moe_mailbox_serve_many", lib().asap_moe_mailbox_serve_many(m.ptr, n, cs, ce, _stream(stream)))
+
+
 def asap_moe_mailbox_wait(m, slot, stream=None):
     check("asap_moe_mailbox_wait", lib().asap_moe_mailbox_wait(m.ptr, int(slot), _stream(stream)))
 

@@ -1419,14 +1419,19 @@ ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const voi
   return ASAP_OK;
 }
 
-ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream) {
-  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+namespace {
+
+// One service round on st for the posts (slots[i], epochs[i]) (count >= 1,
+// distinct slots, validated by the caller, mailbox lock held): the stream
+// waits for each of those posts and for the previous round; the claim waits
+// (bounded) for the first one's flag and claims every published, unserved
+// post of its layer; each listed slot's served event is recorded after the
+// round.
+int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uint64_t* epochs, cudaStream_t st) {
   asap_moe_t h = m->h;
   const asap_moe_config& c = h->cfg;
-  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
-  if (epoch < 1) return fail(ASAP_ERR_INVALID, "epoch must be >= 1 (the value asap_moe_mailbox_post returned)");
-  std::lock_guard<std::mutex> lock(m->mu);
-  cudaStream_t st = S(stream);
+  const int32_t slot = slots[0];
+  const uint64_t epoch = epochs[0];
   const asap::MboxGeom& g = m->g;
   const Layout& L = m->L;
   void* ws = m->ws;
@@ -1440,7 +1445,7 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
   // the post this round is for was published before the round starts; the
   // previous round (on whatever stream it was served) is done with the
   // server workspace
-  CU_TRY(cudaStreamWaitEvent(st, m->post_ev[slot], 0), "wait for the post");
+  for (int i = 0; i < count; ++i) CU_TRY(cudaStreamWaitEvent(st, m->post_ev[slots[i]], 0), "wait for the post");
   if (m->any_round) CU_TRY(cudaStreamWaitEvent(st, m->round_ev, 0), "wait for the previous round");
   CU_TRY(asap::launch_mbox_claim(m->slots, g, slot, epoch, m->wait_ns, m->round, m->rowmap, at<int32_t>(ws, L.ticket),
                                  h->status, st),
@@ -1490,11 +1495,42 @@ ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t
   CU_TRY(asap::launch_combine_mbox(m->round, g, y_perm, y_sh, at<float>(ws, L.w), perm_dst, h->status, st),
          "combine launch");
   CU_TRY(asap::launch_mbox_finish(m->slots, m->round, m->log, m->served_host_dev, st), "finish launch");
-  CU_TRY(cudaEventRecord(m->served_ev[slot], st), "served event");
+  for (int i = 0; i < count; ++i) {
+    CU_TRY(cudaEventRecord(m->served_ev[slots[i]], st), "served event");
+    if (epochs[i] > m->serve_called[slots[i]]) m->serve_called[slots[i]] = epochs[i];
+  }
   CU_TRY(cudaEventRecord(m->round_ev, st), "round event");
   m->any_round = true;
-  if (epoch > m->serve_called[slot]) m->serve_called[slot] = epoch;
   return ASAP_OK;
+}
+
+}  // namespace
+
+ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+  if (epoch < 1) return fail(ASAP_ERR_INVALID, "epoch must be >= 1 (the value asap_moe_mailbox_post returned)");
+  std::lock_guard<std::mutex> lock(m->mu);
+  return serve_round(m, 1, &slot, &epoch, S(stream));
+}
+
+ASAP_API int asap_moe_mailbox_serve_many(asap_moe_mailbox_t m, int32_t count, const int32_t* slots,
+                                         const uint64_t* epochs, void* stream) {
+  if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  if (count < 1 || count > m->g.n_slots || !slots || !epochs)
+    return fail(ASAP_ERR_INVALID, "count must be in [1, n_slots] with host arrays of count slots and epochs");
+  std::lock_guard<std::mutex> lock(m->mu);
+  uint64_t seen = 0;
+  for (int i = 0; i < count; ++i) {
+    const int32_t s = slots[i];
+    if (s < 0 || s >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
+    if (seen & (1ull << s)) return fail(ASAP_ERR_INVALID, "a slot is listed twice");
+    seen |= 1ull << s;
+    if (epochs[i] < 1 || epochs[i] > m->posted[s])
+      return fail(ASAP_ERR_INVALID, "slot " + std::to_string(s) + ": epoch " + std::to_string(epochs[i]) +
+                                        " is not a post made to it");
+  }
+  return serve_round(m, count, slots, epochs, S(stream));
 }
 
 ASAP_API int asap_moe_mailbox_wait(asap_moe_mailbox_t m, int32_t slot, void* stream) {

@@ -232,6 +232,40 @@ def test_randomised_posts_sizes_slots_and_streams(cfg):
     m.close()
 
 
+def test_serve_many_closed_loop():
+    """Each DP group posts its next micro-batch only once its previous one is
+    served (its stream waits for it); one serve_many call per step names the
+    step's posts.  Every round serves all of them, the outputs equal
+    asap_moe_layer's bit for bit, and bad requests are refused."""
+    c = Case.get(DS)
+    n = len(c.xs)
+    m = api.asap_moe_mailbox_create(c.h, n, max(DS.microbatches))
+    prods = [torch.cuda.Stream() for _ in range(n)]
+    server = torch.cuda.Stream()
+    for step in range(3):
+        outs = [torch.full_like(x, float(step + 2)) for x in c.xs]
+        eps = []
+        for i, (x, o, p) in enumerate(zip(c.xs, outs, prods)):
+            if step:
+                api.asap_moe_mailbox_wait(m, i, stream=p)
+            eps.append(api.asap_moe_mailbox_post(m, i, x, o, stream=p))
+        api.asap_moe_mailbox_serve_many(m, list(range(n)), eps, stream=server)
+        for i, p in enumerate(prods):
+            api.asap_moe_mailbox_wait(m, i, stream=p)
+        torch.cuda.synchronize()
+        for a, b in zip(c.ref, outs):
+            assert same_bits(a, b)
+    assert api.asap_moe_mailbox_rounds(m) == (3, [n, n, n])
+    with pytest.raises(AsapError):
+        api.asap_moe_mailbox_serve_many(m, [0, 0], [3, 3])          # a slot listed twice
+    with pytest.raises(AsapError):
+        api.asap_moe_mailbox_serve_many(m, [0], [4])                 # epoch 4 was never posted
+    with pytest.raises(AsapError):
+        api.asap_moe_mailbox_serve_many(m, [], [])                   # nothing to serve
+    assert_clean(c.h)
+    m.close()
+
+
 def test_mailbox_output_against_oracle():
     """The chain to the oracle directly: one round serving three posts of the
     DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
