@@ -387,7 +387,14 @@ def run_ours(args, dist):
             result["mailbox"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
                                              latest_first=args.mailbox_latest_first,
                                              pipelined=args.mailbox_back_to_back or args.mailbox_closed_loop,
-                                             closed_loop=args.mailbox_closed_loop)
+                                             closed_loop=args.mailbox_closed_loop,
+                                             serve_many=args.mailbox_serve_many)
+        # a serving loop: each DP group posts its next micro-batch once its
+        # previous one is served, the server names each step's posts in one call
+        if not (args.mailbox_closed_loop and args.mailbox_serve_many):
+            with nvtx("mailbox serving-loop pass"):
+                result["mailbox_serving_loop"] = mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist,
+                                                              pipelined=True, closed_loop=True, serve_many=True)
 
     # the same fraction where several micro-batches share the GEMMs: sets the
     # device chose (mailbox rounds) and sets the host chose (aggregated call)
@@ -721,7 +728,7 @@ def aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist):
 
 
 def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_first=False, pipelined=False,
-                 closed_loop=False):
+                 closed_loop=False, serve_many=False):
     """The step's micro-batches posted into a mailbox, each from its own
     stream, and served by rounds on one MoE stream: the host serves every post
     right after making it (no host batching), and each round claims on the
@@ -766,12 +773,12 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             elif closed_loop and si > 0:
                 api.asap_moe_mailbox_wait(m, ((si - 1) % depth) * n_mb + i, stream=p)
             eps.append(api.asap_moe_mailbox_post(m, b * n_mb + i, x, outs[b][i], stream=p))
-        if args.mailbox_serve_many:
+        if serve_many:
             if gemm_events is not None:
                 api.asap_moe_mailbox_time_gemms(m, *gemm_events[0])
             api.asap_moe_mailbox_serve_many(m, [b * n_mb + i for i in range(n_mb)], eps, stream=server)
         for r, i in enumerate(reversed(range(n_mb)) if latest_first else range(n_mb)):
-            if args.mailbox_serve_many:
+            if serve_many:
                 break
             if gemm_events is not None:
                 api.asap_moe_mailbox_time_gemms(m, *gemm_events[r])
@@ -819,7 +826,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
         step(base + si, evs, lat)
         torch.cuda.synchronize()
         ra, cl = api.asap_moe_mailbox_rounds(m)
-        gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in (evs[:1] if args.mailbox_serve_many else evs)))
+        gemm_ms.append(sum(e0.elapsed_time(e1) for e0, e1 in (evs[:1] if serve_many else evs)))
         nonempty.append(sum(1 for c in cl[rb:ra] if c > 0))
     api.asap_moe_mailbox_rounds(m)
     code, word = api.asap_moe_status(h)
@@ -849,7 +856,7 @@ def mailbox_pass(args, h, cfg, xs, dev, peaks, tensor_peak, kern, dist, latest_f
             "post_latency_ms": post_lat,
             "post_latency_note": "in the GEMM-timing steps: step start (every DP-group stream waits on it) to "
                                  "each post's completion as seen by a stream of its own",
-            "serve_order": ("one serve_many call per step" if args.mailbox_serve_many else
+            "serve_order": ("one serve_many call per step" if serve_many else
                             "latest post first" if latest_first else "post order"),
             "steps": ("closed loop per DP group, no barrier between steps" if closed_loop else
                       "back to back, no barrier between steps" if pipelined else "one barrier per step"),
