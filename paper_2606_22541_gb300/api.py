@@ -270,6 +270,7 @@ def asap_moe_mailbox_serve(m, slot, epoch, stream=None):
 
 
 def asap_moe_mailbox_serve_many(m, slots, epochs, stream=None):
+    """One service round for the posts (slots[i], epochs[i]) already made."""
     n = len(slots)
     cs = (ctypes.c_int32 * n)(*[int(v) for v in slots])
     ce = (ctypes.c_uint64 * n)(*[int(v) for v in epochs])
