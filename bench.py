@@ -377,6 +377,17 @@ def run_ours(args, dist):
         "peaks": peaks_src,
         "note": "algorithmic FLOPs of both grouped GEMMs (routed + shared) over their event-timed durations"}
 
+    # route, dispatch and combine of a micro-batch together (the HBM-bound
+    # steps around the grouped GEMMs)
+    small = [nm for nm in ("route", "dispatch", "combine") if nm in kern["table"]]
+    sb = sum(kern["alg"][nm]["bytes"] for nm in small)
+    sms = sum(kern["avg"][nm] for nm in small)
+    result["route_dispatch_combine"] = {
+        "alg_bytes": sb, "ms": sms, "gbs": sb / (sms / 1e3) / 1e9,
+        "frac_of_measured_hbm": sb / (sms / 1e3) / 1e9 / peaks["hbm_gbs"],
+        "note": "the three steps' algorithmic bytes over their summed event times in the per-kernel pass "
+                "(the standalone dispatch call includes its histogram and scan)"}
+
     # ---------------- all micro-batches in one pass (one grouped GEMM per weight matrix)
     with nvtx("host-aggregated pass"):
         result["aggregated"] = aggregated_pass(args, h, cfg, xs, dev, peaks, tensor_peak, dist)
