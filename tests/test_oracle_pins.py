@@ -710,3 +710,42 @@ def test_pins_catch_planted_mistakes(monkeypatch):
     monkeypatch.setattr(gating, "_order", lambda keys: np.lexsort((np.arange(len(keys)), np.asarray(keys))))
     idx, _ = gating.route_token_softmax(l, 2, False)
     assert list(idx) != S
+
+
+def test_router_logits_hand_worked_and_one_hot():
+    """router_logits against values worked by hand (the logits are the dot
+    products of each token with each expert's router row) and against
+    one-hot tokens, which must pick out one router column exactly."""
+    x = np.array([[1.0, 2.0, -1.0], [0.5, 0.0, 4.0]])
+    wr = np.array([[2.0, 0.0, 1.0], [-1.0, 3.0, 0.5], [0.0, 0.0, 0.0], [1.0, 1.0, 1.0]])
+    # token 0: 2 + 0 - 1 = 1; -1 + 6 - 0.5 = 4.5; 0; 1 + 2 - 1 = 2
+    # token 1: 1 + 0 + 4 = 5; -0.5 + 0 + 2 = 1.5; 0; 0.5 + 0 + 4 = 4.5
+    want = np.array([[1.0, 4.5, 0.0, 2.0], [5.0, 1.5, 0.0, 4.5]])
+    assert np.array_equal(oracle.router_logits(x, wr), want)
+    rng = np.random.default_rng(3)
+    W = rng.standard_normal((6, 5))
+    eye = np.eye(5)
+    L = oracle.router_logits(eye, W)
+    assert L.shape == (5, 6)
+    assert np.array_equal(L, W.T)                     # token j = e_j gives column j of Wr
+    assert np.array_equal(oracle.router_logits(np.zeros((2, 5)), W), np.zeros((2, 6)))
+
+
+def test_expert_ffn_hand_worked_segments():
+    """expert_ffn on two experts' segments with values worked by hand:
+    expert 0 (gate row [1, 0], up row [0, 1], down column [1, 2]) on token
+    [1, 2] gives g = 1, u = 2, h = silu(1) * 2 and y = [h, 2h]; expert 1 has
+    an empty segment; expert 2 (gate row [0, 0]) gives h = silu(0) * u = 0.
+    silu(1) = 1 / (1 + e^-1) exactly as the closed form."""
+    wg = np.array([[[1.0, 0.0]], [[5.0, 5.0]], [[0.0, 0.0]]])      # [E=3, I=1, H=2]
+    wu = np.array([[[0.0, 1.0]], [[5.0, 5.0]], [[3.0, 4.0]]])
+    wd = np.array([[[1.0], [2.0]], [[9.0], [9.0]], [[1.0], [1.0]]])  # [E, H=2, I=1]
+    x_perm = np.array([[1.0, 2.0], [7.0, -3.0]])
+    offsets = np.array([0, 1, 1, 2])                                 # expert 1's segment is empty
+    y = oracle.expert_ffn(x_perm, offsets, wg, wu, wd)
+    h = 1.0 / (1.0 + np.exp(-1.0)) * 2.0
+    assert np.allclose(y[0], [h, 2.0 * h], rtol=0, atol=1e-15)
+    assert np.array_equal(y[1], [0.0, 0.0])
+    # callables decode one expert at a time and give the same result
+    y2 = oracle.expert_ffn(x_perm, offsets, lambda e: wg[e], lambda e: wu[e], lambda e: wd[e])
+    assert np.array_equal(y, y2)
