@@ -254,13 +254,24 @@ def asap_moe_mailbox_create(h, n_slots, slot_tokens, layer_id=None, wait_ns=2_00
 
 def asap_moe_mailbox_post(m, slot, x, out, stream=None, layer_id=None):
     """Post x (n tokens) into slot; returns the post's epoch.  layer_id: None
-    (the mailbox's default layer) or a one-element int32 CUDA tensor.  x, out
-    and layer_id must stay alive until the post is served; the mailbox keeps a
-    reference to the slot's last post."""
+    (the mailbox's default layer) or a one-element int32 CUDA tensor.  The
+    mailbox keeps x, out and layer_id alive until the slot is posted again or
+    the mailbox is closed."""
+    s = torch.cuda.current_stream() if stream is None else stream
     ep = ctypes.c_uint64()
     check("asap_moe_mailbox_post",
           lib().asap_moe_mailbox_post(m.ptr, int(slot), _ptr(x), x.shape[0], _ptr(out), _ptr(layer_id),
-                                      _stream(stream), ctypes.byref(ep)))
+                                      _stream(s), ctypes.byref(ep)))
+    old = m._keep.get(int(slot))
+    if old is not None:
+        # The post just enqueued on s waits for the round that served the
+        # slot's previous post, so once s reaches this point that round is
+        # done with the previous tensors.  Recording s on them keeps the
+        # caching allocator from handing their memory to another stream
+        # before then, even when this reference was the last one.
+        for t in old:
+            if t is not None:
+                t.record_stream(s)
     m._keep[int(slot)] = (x, out, layer_id)
     return ep.value
 
