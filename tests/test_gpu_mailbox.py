@@ -266,6 +266,39 @@ def test_serve_many_closed_loop():
     m.close()
 
 
+def test_repost_keeps_the_previous_tensors_until_their_round_is_done():
+    """The binding holds a post's tensors until its slot is posted again.  A
+    repost drops the last reference to the previous x while the round that
+    reads it may not have run yet (here it starts ~25 ms late); the memory
+    must not go to another allocation on the main stream before that round
+    is done, so the first post's output still equals asap_moe_layer's."""
+    c = Case.get(DS)
+    m = api.asap_moe_mailbox_create(c.h, 1, max(DS.microbatches))
+    p = torch.cuda.Stream()
+    server = torch.cuda.Stream()
+    main = torch.cuda.current_stream()
+    x0 = c.xs[0]
+    o1 = torch.full_like(x0, 3.0)
+    o2 = torch.full_like(x0, 4.0)
+    tmp = x0.clone()
+    p.wait_stream(main)
+    ep1 = api.asap_moe_mailbox_post(m, 0, tmp, o1, stream=p)
+    del tmp                                   # the mailbox holds the only reference now
+    with torch.cuda.stream(server):
+        torch.cuda._sleep(50_000_000)
+    api.asap_moe_mailbox_serve(m, 0, ep1, stream=server)
+    ep2 = api.asap_moe_mailbox_post(m, 0, x0, o2, stream=p)   # drops the previous x
+    junk = torch.empty_like(x0)
+    junk.fill_(-5.0)
+    api.asap_moe_mailbox_serve(m, 0, ep2, stream=server)
+    api.asap_moe_mailbox_wait(m, 0, stream=main)
+    torch.cuda.synchronize()
+    assert same_bits(c.ref[0], o1)
+    assert same_bits(c.ref[0], o2)
+    assert_clean(c.h)
+    m.close()
+
+
 def test_mailbox_output_against_oracle():
     """The chain to the oracle directly: one round serving three posts of the
     DeepSeek-V3-shaped layer, compared with the float64 layer on the tokens
