@@ -204,7 +204,8 @@ enum {
 int asap_moe_set_tiling(asap_moe_t h, int32_t mode);
 
 /* Free everything create allocated.  Synchronises the device first.  NULL is
- * accepted. */
+ * accepted.  Refused with ASAP_ERR_INVALID (nothing freed) while a mailbox
+ * created on h is alive: destroy the mailboxes first. */
 int asap_moe_destroy(asap_moe_t h);
 
 /* Pure host computation: bytes of workspace one call with n tokens needs.  The

@@ -44,8 +44,10 @@ class Handle:
         return self.ccfg.max_tokens
 
     def close(self):
+        """Frees the handle; raises AsapError (and keeps it) while a mailbox
+        created on it is open."""
         if self.ptr:
-            lib().asap_moe_destroy(self.ptr)
+            check("asap_moe_destroy", lib().asap_moe_destroy(self.ptr))
             self.ptr = None
 
     def __del__(self):

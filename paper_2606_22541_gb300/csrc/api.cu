@@ -6,6 +6,7 @@
 #include "internal.h"
 #include "gemm_config.h"
 
+#include <atomic>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -40,6 +41,7 @@ struct asap_moe_s {
   bool tc_router = false;             // router GEMM on the tensor core (E == 256)
   bool fp8 = false;                   // e4m3 experts with fp32 128 x 128 block scales
   int tiling = ASAP_TILING_AUTO;       // BF16 grouped GEMM tile shape (asap_moe_set_tiling)
+  std::atomic<int> mailboxes{0};      // live mailboxes created on this handle
 };
 
 namespace {
@@ -624,6 +626,9 @@ ASAP_API int asap_moe_workspace_size(const asap_moe_config* cfg, int32_t n_token
 
 ASAP_API int asap_moe_destroy(asap_moe_t h) {
   if (!h) return ASAP_OK;
+  if (const int live = h->mailboxes.load())
+    return fail(ASAP_ERR_INVALID, std::to_string(live) +
+                                      " mailbox(es) created on this handle are still alive; destroy them first");
   int prev = 0;
   cudaGetDevice(&prev);
   cudaSetDevice(h->device);
@@ -1361,11 +1366,18 @@ ASAP_API int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot
   m->posted.assign(n_slots, 0);
   m->serve_called.assign(n_slots, 0);
   if ((e = cudaDeviceSynchronize()) != cudaSuccess) return restore(bail(cuda_fail(e, "mailbox create sync")));
+  h->mailboxes.fetch_add(1);
   *out = m;
   return restore(ASAP_OK);
 }
 
-ASAP_API int asap_moe_mailbox_destroy(asap_moe_mailbox_t m) { return mbox_free(m); }
+ASAP_API int asap_moe_mailbox_destroy(asap_moe_mailbox_t m) {
+  if (!m) return ASAP_OK;
+  asap_moe_t h = m->h;
+  const int r = mbox_free(m);
+  h->mailboxes.fetch_sub(1);
+  return r;
+}
 
 ASAP_API int asap_moe_mailbox_post(asap_moe_mailbox_t m, int32_t slot, const void* x, int32_t n, void* out,
                                    const int32_t* layer_id, void* stream, uint64_t* epoch) {

@@ -380,6 +380,32 @@ def test_host_side_rules():
     m.close()
 
 
+def test_handle_outlives_its_mailboxes():
+    """Destroying a handle while a mailbox created on it is open is refused
+    (the mailbox uses the handle's weights and device); once the mailboxes
+    are closed the handle is freed."""
+    cfg = inputs.small_variant(DS, name="mbox_owner", microbatches=[64])
+    h = api.asap_moe_create(cfg, inputs.make_weights(cfg, DEV), 64)
+    m1 = api.asap_moe_mailbox_create(h, 1, 64)
+    m2 = api.asap_moe_mailbox_create(h, 1, 64)
+    with pytest.raises(AsapError, match="2 mailbox"):
+        h.close()
+    m1.close()
+    with pytest.raises(AsapError, match="1 mailbox"):
+        h.close()
+    x = inputs.make_tokens(cfg, 64, 5, DEV)
+    out = torch.empty_like(x)
+    ref = torch.empty_like(x)
+    ep = api.asap_moe_mailbox_post(m2, 0, x, out)              # the handle still works
+    api.asap_moe_mailbox_serve(m2, 0, ep)
+    api.asap_moe_layer(h, x, ref, api.workspace(h, 64))
+    torch.cuda.synchronize()
+    assert same_bits(ref, out)
+    m2.close()
+    h.close()
+    assert h.ptr is None
+
+
 def test_one_mailbox_serves_interleaved_layers():
     """Posts of two layers of one handle interleaved in the slots: each round
     claims only the ready posts of its own post's layer and runs that
