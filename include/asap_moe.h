@@ -422,7 +422,8 @@ typedef struct asap_moe_mailbox_s* asap_moe_mailbox_t;
  * (<= max_tokens) each on h's device.  layer_id: the layer of posts made
  * without one, NULL (layer 0) or a 4-byte aligned device int32.  wait_ns > 0:
  * the limit of a round's wait for a post that has not been published.
- * Allocates; synchronous. */
+ * Allocates; synchronous.  h must outlive the mailbox: asap_moe_destroy(h)
+ * is refused while the mailbox is alive. */
 int asap_moe_mailbox_create(asap_moe_t h, int32_t n_slots, int32_t slot_tokens,
                             const int32_t* layer_id, int64_t wait_ns, asap_moe_mailbox_t* out);
 
