@@ -47,6 +47,6 @@ def test_batched_equals_separate_calls(cfg, lengths):
     _check(cfg, lengths)
 
 
-@pytest.mark.parametrize("cfg", [DSV3, STRESS, MIXTRAL], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", [DSV3, STRESS, MIXTRAL, DSV3_FP8], ids=lambda c: c.name)
 def test_batched_full_size(cfg):
     _check(cfg, cfg.microbatches)
