@@ -386,7 +386,7 @@ def run_ours(args, dist):
         "alg_bytes": sb, "ms": sms, "gbs": sb / (sms / 1e3) / 1e9,
         "frac_of_measured_hbm": sb / (sms / 1e3) / 1e9 / peaks["hbm_gbs"],
         "note": "the three steps' algorithmic bytes over their summed event times in the per-kernel pass "
-                "(the standalone dispatch call includes its histogram and scan)"}
+                "(events recorded by asap_moe_layer between its own steps)"}
 
     # ---------------- all micro-batches in one pass (one grouped GEMM per weight matrix)
     with nvtx("host-aggregated pass"):
@@ -519,9 +519,10 @@ def head_start(stream):
 
 
 def kernel_pass(args, h, cfg, xs, dev):
-    """The same work as the timed steps, launched call by call on one stream
-    with CUDA events between the calls, so every kernel's duration is taken on
-    the stream it runs on without overlap from the other micro-batches."""
+    """The same work as the timed steps, one asap_moe_layer call after
+    another on one stream, each recording CUDA events between its own steps
+    (asap_moe_time_layer), so every kernel of the layer is timed where it
+    runs, without overlap from the other micro-batches."""
     import numpy as np
     import torch
     from paper_2606_22541_gb300 import api
@@ -529,65 +530,39 @@ def kernel_pass(args, h, cfg, xs, dev):
     n = max(x.shape[0] for x in xs)
     k, E, H, I, Is = cfg.top_k, cfg.n_experts, cfg.hidden, cfg.inter, cfg.shared_inter
     s = torch.cuda.current_stream()
-    logits = torch.empty((n, E), dtype=torch.float32, device=dev)
     idx = torch.empty((n, k), dtype=torch.int32, device=dev)
     w = torch.empty((n, k), dtype=torch.float32, device=dev)
     counts = torch.empty(E, dtype=torch.int32, device=dev)
     offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
-    x_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=dev)
-    perm_src = torch.empty(n * k, dtype=torch.int32, device=dev)
-    perm_dst = torch.empty((n, k), dtype=torch.int32, device=dev)
-    hbuf = torch.empty((n * k, I), dtype=torch.bfloat16, device=dev)
-    hsh = torch.empty((n, Is), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
-    y_perm = torch.empty((n * k, H), dtype=torch.bfloat16, device=dev)
-    y_sh = torch.empty((n, H), dtype=torch.bfloat16, device=dev) if cfg.n_shared else None
     out = torch.empty((n, H), dtype=torch.bfloat16, device=dev)
     ws = api.workspace(h, n, dev)
     fp8 = cfg.dtype != "bf16"
     names = ["route", "dispatch", "gemm_gate_up_swiglu", "gemm_down", "combine"]
     if fp8:
         names = ["route", "dispatch", "expert_ffn_fp8", "combine"]
-        x_perm = torch.empty((n * k, H), dtype=torch.uint8, device=dev)
-        xsc = torch.empty((n * k, H // 128), dtype=torch.float32, device=dev)
     times = {nm: [] for nm in names}
     active = []   # experts with tokens, per micro-batch (for the weight bytes)
+    for x in xs:
+        m = x.shape[0]
+        api.asap_moe_route(h, x, idx[:m], w[:m], counts, offsets, ws, stream=s)
+        torch.cuda.synchronize()
+        active.append(int((counts > 0).sum().item()))
     for it in range(args.kernel_steps + 1):
         rec = []
         head_start(s)
         for x in xs:
             m = x.shape[0]
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
-            ev[0].record(s)
-            api.asap_moe_route(h, x, idx[:m], w[:m], counts, offsets, ws, stream=s)
-            ev[1].record(s)
-            api.asap_moe_dispatch(h, x, idx[:m], x_perm[:m * k], perm_src[:m * k], perm_dst[:m], ws, stream=s,
-                                  x_perm_scales=xsc[:m * k] if fp8 else None)
-            ev[2].record(s)
-            if fp8:
-                api.asap_moe_expert_ffn(h, x_perm[:m * k], offsets, x, y_perm[:m * k],
-                                        y_sh[:m] if y_sh is not None else None, ws, stream=s,
-                                        x_perm_scales=xsc[:m * k])
-                ev[3].record(s)
-            else:
-                api.asap_moe_expert_gate_up(h, x_perm[:m * k], offsets, x, hbuf[:m * k],
-                                            hsh[:m] if hsh is not None else None, stream=s, ws=ws)
-                ev[3].record(s)
-                api.asap_moe_expert_down(h, hbuf[:m * k], offsets, hsh[:m] if hsh is not None else None, m,
-                                         y_perm[:m * k], y_sh[:m] if y_sh is not None else None, stream=s, ws=ws)
-                ev[4].record(s)
-            api.asap_moe_combine(h, y_perm[:m * k], y_sh[:m] if y_sh is not None else None, w[:m], perm_dst[:m],
-                                 out[:m], stream=s)
-            ev[len(names)].record(s)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+            api.asap_moe_time_layer(ev)
+            api.asap_moe_layer(h, x, out[:m], ws, stream=s)
             rec.append(ev)
-            if it == 0:
-                torch.cuda.synchronize()
-                active.append(int((counts > 0).sum().item()))
         torch.cuda.synchronize()
         if it == 0:
             continue   # warm-up round
         for ev in rec:
-            for j, nm in enumerate(names):
-                times[nm].append(ev[j].elapsed_time(ev[j + 1]))
+            d = [ev[j].elapsed_time(ev[j + 1]) for j in range(5)]   # route, dispatch, gate/up, down, combine
+            for nm, v in zip(names, [d[0], d[1], d[2] + d[3], d[4]] if fp8 else d):
+                times[nm].append(v)
     avg = {nm: sum(v) / len(v) for nm, v in times.items()}
     mins = {nm: min(v) for nm, v in times.items()}
     mean_active = sum(active) / len(active)

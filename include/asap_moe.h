@@ -311,6 +311,16 @@ int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws,
 int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int32_t n,
                        void* out, void* ws, size_t ws_bytes, void* stream);
 
+/* Timing hook: the next asap_moe_layer or asap_moe_layer_dyn call made by
+ * this thread records events[0] (a cudaEvent_t; NULL entries are skipped) on
+ * its stream before its first kernel and events[i] after its i-th step:
+ * 1 route, 2 dispatch, 3 gate/up GEMM, 4 down GEMM, 5 combine, so each of
+ * the layer's own kernels can be timed where it runs.  count in [0, 6]
+ * (0 clears the request); the request is consumed by that next call even if
+ * it fails or has n = 0, which then records nothing.  Host state of the
+ * calling thread only; enqueues nothing itself. */
+int asap_moe_time_layer(int32_t count, void* const* events);
+
 /* asap_moe_route without any device allocation (no counterpart in the
  * paper; this entry point exists for callers that cannot allocate).
  *

@@ -208,6 +208,17 @@ def asap_moe_layer_batched_dyn(h, layer_id, xs, outs, ws, stream=None):
           lib().asap_moe_layer_batched_dyn(h.ptr, _ptr(layer_id), cnt, xa, na, oa, p, n, _stream(stream)))
 
 
+def asap_moe_time_layer(events):
+    """Events (torch.cuda.Event, enable_timing=True; up to 6) for this
+    thread's next asap_moe_layer / _dyn call to record: before its first
+    kernel and after route, dispatch, gate/up, down and combine."""
+    for ev in events:
+        if ev.cuda_event == 0:   # torch creates the CUDA event at its first record
+            ev.record()
+    arr = (ctypes.c_void_p * max(1, len(events)))(*[ev.cuda_event for ev in events])
+    check("asap_moe_time_layer", lib().asap_moe_time_layer(len(events), arr))
+
+
 def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
     """asap_moe_route with its scratch in the library's static device array
     (at most 4096 tokens; calls overlapping on the GPU race)."""

@@ -1001,9 +1001,27 @@ ASAP_API int asap_moe_combine(asap_moe_t h, const void* y_perm, const void* y_sh
 
 namespace {
 
+// Events that asap_moe_time_layer asked this thread's next layer call to
+// record: before its first kernel and after each of its five steps.
+constexpr int kLayerEvents = 6;
+thread_local cudaEvent_t g_layer_ev[kLayerEvents] = {};
+
+// The pending events of this thread, taken (the request is cleared) when a
+// layer call starts, so each request serves one call whatever its outcome.
+struct LayerEvents {
+  cudaEvent_t ev[kLayerEvents] = {};
+  LayerEvents() {
+    for (int i = 0; i < kLayerEvents; ++i) {
+      ev[i] = g_layer_ev[i];
+      g_layer_ev[i] = nullptr;
+    }
+  }
+  cudaError_t mark(int i, cudaStream_t st) const { return ev[i] ? cudaEventRecord(ev[i], st) : cudaSuccess; }
+};
+
 // The whole layer for one micro-batch, weights of layer *layer (device).
 int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_t ws_bytes, const int32_t* layer,
-              void* stream) {
+              void* stream, const LayerEvents& tev) {
   int r = check_call(h, n, ws, ws_bytes, true);
   if (r != ASAP_OK || n == 0) return r;
   if (!x || !out || !aligned16(x) || !aligned16(out)) return fail(ASAP_ERR_INVALID, "NULL or unaligned tensor");
@@ -1019,7 +1037,9 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
   int32_t* perm_dst = at<int32_t>(ws, L.perm_dst);
   int32_t* counters = at<int32_t>(ws, L.tile_counters);  // zeroed by the scan kernel
   void* y_sh = c.n_shared ? at<void>(ws, L.y_sh) : nullptr;
+  CU_TRY(tev.mark(0, st), "timing event");
   if ((r = run_route(h, x, n, idx, w, counts, offsets, ws, layer, st)) != ASAP_OK) return r;
+  CU_TRY(tev.mark(1, st), "timing event");
   if (h->fp8) {
     void* xq_sh = c.n_shared ? at<void>(ws, L.xq_sh) : nullptr;
     float* xs_sh = c.n_shared ? at<float>(ws, L.xs_sh) : nullptr;
@@ -1027,28 +1047,37 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
                                      offsets, at<void>(ws, L.xq), at<float>(ws, L.xs), xq_sh, xs_sh, perm_src,
                                      perm_dst, h->status, st),
            "dispatch launch");
+    CU_TRY(tev.mark(2, st), "timing event");
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, n, at<void>(ws, L.hq),
                              at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), layer, counters,
                              st)) != ASAP_OK)
       return r;
+    CU_TRY(tev.mark(3, st), "timing event");
     void* y_perm = at<void>(ws, L.y_perm);
     if ((r = run_down_fp8(h, at<void>(ws, L.hq), at<float>(ws, L.hs), offsets, at<void>(ws, L.hq_sh),
                           at<float>(ws, L.hs_sh), n, y_perm, y_sh, layer, counters + 1, st)) != ASAP_OK)
       return r;
+    CU_TRY(tev.mark(4, st), "timing event");
     CU_TRY(asap::launch_combine(y_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
            "combine launch");
+    CU_TRY(tev.mark(5, st), "timing event");
     return ASAP_OK;
   }
   void* x_perm = at<void>(ws, L.x_perm);
   CU_TRY(asap::launch_dispatch(x, n, c.hidden, c.top_k, c.n_experts, idx, at<int32_t>(ws, L.chunk_base), offsets,
                                x_perm, perm_src, perm_dst, h->status, st),
          "dispatch launch");
+  CU_TRY(tev.mark(2, st), "timing event");
   // y_perm reuses x_perm's rows: the down GEMM never reads x_perm
-  if ((r = run_expert_ffn(h, x_perm, offsets, x, n, x_perm, y_sh, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer,
-                          counters, st)) != ASAP_OK)
-    return r;
+  void* hbuf = at<void>(ws, L.h);
+  void* hsh = at<void>(ws, L.h_sh);
+  if ((r = run_gate_up(h, x_perm, offsets, x, n, hbuf, hsh, layer, counters, st)) != ASAP_OK) return r;
+  CU_TRY(tev.mark(3, st), "timing event");
+  if ((r = run_down(h, hbuf, offsets, hsh, n, x_perm, y_sh, layer, counters + 1, st)) != ASAP_OK) return r;
+  CU_TRY(tev.mark(4, st), "timing event");
   CU_TRY(asap::launch_combine(x_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
          "combine launch");
+  CU_TRY(tev.mark(5, st), "timing event");
   return ASAP_OK;
 }
 
@@ -1189,17 +1218,26 @@ bool valid_layer_ptr(const int32_t* layer) {
 
 }  // namespace
 
+ASAP_API int asap_moe_time_layer(int32_t count, void* const* events) {
+  if (count < 0 || count > kLayerEvents || (count > 0 && !events))
+    return fail(ASAP_ERR_INVALID, "count must be in [0, " + std::to_string(kLayerEvents) + "] with an events array");
+  for (int i = 0; i < kLayerEvents; ++i) g_layer_ev[i] = i < count ? static_cast<cudaEvent_t>(events[i]) : nullptr;
+  return ASAP_OK;
+}
+
 ASAP_API int asap_moe_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_t ws_bytes,
                             void* stream) {
+  const LayerEvents tev;  // taken by this call whatever its outcome
   if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
-  return run_layer(h, x, n, out, ws, ws_bytes, h->layer_ids, stream);
+  return run_layer(h, x, n, out, ws, ws_bytes, h->layer_ids, stream, tev);
 }
 
 ASAP_API int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int32_t n, void* out,
                                 void* ws, size_t ws_bytes, void* stream) {
+  const LayerEvents tev;
   if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
   if (!valid_layer_ptr(layer_id)) return fail(ASAP_ERR_INVALID, "layer_id must be a non-NULL 4-byte aligned device pointer");
-  return run_layer(h, x, n, out, ws, ws_bytes, layer_id, stream);
+  return run_layer(h, x, n, out, ws, ws_bytes, layer_id, stream, tev);
 }
 
 ASAP_API int asap_moe_layer_batched(asap_moe_t h, int32_t count, const void* const* xs, const int32_t* ns,

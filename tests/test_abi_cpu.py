@@ -110,3 +110,15 @@ def test_tiling_modes_match_the_header(L):
     assert vals == {"AUTO": api.TILING_AUTO, "SINGLE": api.TILING_SINGLE, "PAIRED": api.TILING_PAIRED}
     # a NULL handle is rejected on the host
     assert L.asap_moe_set_tiling(None, api.TILING_AUTO) == _native.ASAP_ERR_INVALID
+
+
+def test_time_layer_validates_its_request(L):
+    arr = (ctypes.c_void_p * 7)()
+    assert L.asap_moe_time_layer(-1, arr) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_time_layer(7, arr) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_time_layer(2, None) == _native.ASAP_ERR_INVALID
+    assert L.asap_moe_time_layer(0, None) == _native.ASAP_OK
+    # NULL entries are allowed (skipped when the layer records them); a
+    # failing layer call takes the request and records nothing
+    assert L.asap_moe_time_layer(6, arr) == _native.ASAP_OK
+    assert L.asap_moe_layer(None, None, 1, None, None, 0, None) == _native.ASAP_ERR_INVALID
