@@ -232,14 +232,15 @@ def test_randomised_posts_sizes_slots_and_streams(cfg):
     m.close()
 
 
-def test_serve_many_closed_loop():
+@pytest.mark.parametrize("cfg", [DS, F8], ids=lambda c: c.name)
+def test_serve_many_closed_loop(cfg):
     """Each DP group posts its next micro-batch only once its previous one is
     served (its stream waits for it); one serve_many call per step names the
     step's posts.  Every round serves all of them, the outputs equal
     asap_moe_layer's bit for bit, and bad requests are refused."""
-    c = Case.get(DS)
+    c = Case.get(cfg)
     n = len(c.xs)
-    m = api.asap_moe_mailbox_create(c.h, n, max(DS.microbatches))
+    m = api.asap_moe_mailbox_create(c.h, n, max(cfg.microbatches))
     prods = [torch.cuda.Stream() for _ in range(n)]
     server = torch.cuda.Stream()
     for step in range(3):

@@ -7,7 +7,7 @@ import torch
 
 import oracle
 from paper_2606_22541_gb300 import api, inputs
-from paper_2606_22541_gb300.configs import TINY, MIXTRAL, DSV3, STRESS
+from paper_2606_22541_gb300.configs import TINY, MIXTRAL, DSV3, DSV3_FP8, STRESS
 
 from _helpers import bf16_to_f64, weights_f64, compare_rows, routing_check
 
@@ -462,25 +462,27 @@ def test_layer_equals_composed_calls_bit_for_bit(cfg):
     assert_clean(c)
 
 
-def test_layer_timing_events_mark_its_steps_and_change_no_bit():
+@pytest.mark.parametrize("cfg", [DS_SMALL, inputs.small_variant(DSV3_FP8, name="fp8_timing", hidden=512, inter=256,
+                                                                 shared_inter=256, microbatches=[300])],
+                         ids=lambda c: c.name)
+def test_layer_timing_events_mark_its_steps_and_change_no_bit(cfg):
     """asap_moe_time_layer: the next layer call records the six events in
     order around its five steps, on its own stream, and computes the same
     bits; the request is used once (the call after it records nothing)."""
-    cfg = DS_SMALL
-    c = Case.get(cfg)
+    h = api.asap_moe_create(cfg, inputs.make_weights(cfg, DEV), max(cfg.microbatches))
     n, H = cfg.microbatches[0], cfg.hidden
-    x = c.tokens(0)
-    ws = c.ws(n)
+    x = inputs.make_tokens(cfg, n, 0, DEV)
+    ws = api.workspace(h, n)
     s = torch.cuda.Stream()
     ref = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
-    api.asap_moe_layer(c.h, x, ref, ws)
+    api.asap_moe_layer(h, x, ref, ws)
     torch.cuda.synchronize()
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
     api.asap_moe_time_layer(ev)
     out = torch.empty_like(ref)
     with torch.cuda.stream(s):
         torch.cuda._sleep(1_000_000)              # the recorded events must wait for the layer's stream
-        api.asap_moe_layer(c.h, x, out, ws, stream=s)
+        api.asap_moe_layer(h, x, out, ws, stream=s)
     torch.cuda.synchronize()
     d = [ev[j].elapsed_time(ev[j + 1]) for j in range(5)]
     assert all(v > 0 for v in d), d
@@ -488,11 +490,13 @@ def test_layer_timing_events_mark_its_steps_and_change_no_bit():
     late = torch.cuda.Event(enable_timing=True)
     late.record()
     out2 = torch.empty_like(ref)
-    api.asap_moe_layer(c.h, x, out2, ws)             # no request pending: ev keep their times
+    api.asap_moe_layer(h, x, out2, ws)               # no request pending: ev keep their times
     torch.cuda.synchronize()
     assert ev[5].elapsed_time(late) >= 0
     assert torch.equal(ref.view(torch.int16), out2.view(torch.int16))
-    assert_clean(c)
+    code, word = api.asap_moe_status(h)
+    assert code == 0 and word == 0, f"device status word {word:#x}"
+    h.close()
 
 
 @pytest.mark.parametrize("cfg", [DS_SMALL, ST_SMALL], ids=lambda c: c.name)
