@@ -317,8 +317,10 @@ int asap_moe_layer_dyn(asap_moe_t h, const int32_t* layer_id, const void* x, int
  * 1 route, 2 dispatch, 3 gate/up GEMM, 4 down GEMM, 5 combine, so each of
  * the layer's own kernels can be timed where it runs.  count in [0, 6]
  * (0 clears the request); the request is consumed by that next call even if
- * it fails or has n = 0, which then records nothing.  Host state of the
- * calling thread only; enqueues nothing itself. */
+ * it fails or has n = 0, which then records nothing.  The events must stay
+ * valid until that call returns (recording a destroyed event fails the call
+ * with ASAP_ERR_CUDA).  Host state of the calling thread only; enqueues
+ * nothing itself. */
 int asap_moe_time_layer(int32_t count, void* const* events);
 
 /* asap_moe_route without any device allocation (no counterpart in the
