@@ -5,6 +5,7 @@ Tensors are torch CUDA tensors (the binding passes their device pointers);
 of the layer runs in libasap_moe's kernels; nothing here computes.
 """
 import ctypes
+import threading
 
 import torch
 
@@ -15,6 +16,10 @@ from .configs import GATING, DTYPE
 
 def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+# this thread's pending asap_moe_time_layer events (kept alive for the C side)
+_timing = threading.local()
 
 
 def _stream(stream):
@@ -174,7 +179,10 @@ def asap_moe_combine(h, y_perm, y_shared, w, perm_dst, out, stream=None):
 
 def asap_moe_layer(h, x, out, ws, stream=None):
     p, n = _ws(ws)
-    check("asap_moe_layer", lib().asap_moe_layer(h.ptr, _ptr(x), x.shape[0], _ptr(out), p, n, _stream(stream)))
+    try:
+        check("asap_moe_layer", lib().asap_moe_layer(h.ptr, _ptr(x), x.shape[0], _ptr(out), p, n, _stream(stream)))
+    finally:
+        _timing.events = None   # the call has taken this thread's timing request
 
 
 def asap_moe_layer_batched(h, xs, outs, ws, stream=None):
@@ -193,8 +201,11 @@ def asap_moe_layer_dyn(h, layer_id, x, out, ws, stream=None):
     """asap_moe_layer for the layer whose id the kernels read from layer_id
     (a one-element int32 CUDA tensor) when they run."""
     p, n = _ws(ws)
-    check("asap_moe_layer_dyn", lib().asap_moe_layer_dyn(h.ptr, _ptr(layer_id), _ptr(x), x.shape[0], _ptr(out), p, n,
-                                                         _stream(stream)))
+    try:
+        check("asap_moe_layer_dyn", lib().asap_moe_layer_dyn(h.ptr, _ptr(layer_id), _ptr(x), x.shape[0], _ptr(out), p,
+                                                             n, _stream(stream)))
+    finally:
+        _timing.events = None   # the call has taken this thread's timing request
 
 
 def asap_moe_layer_batched_dyn(h, layer_id, xs, outs, ws, stream=None):
@@ -212,11 +223,13 @@ def asap_moe_time_layer(events):
     """Events (torch.cuda.Event, enable_timing=True; up to 6) for this
     thread's next asap_moe_layer / _dyn call to record: before its first
     kernel and after route, dispatch, gate/up, down and combine."""
+    events = list(events)
     for ev in events:
         if ev.cuda_event == 0:   # torch creates the CUDA event at its first record
             ev.record()
     arr = (ctypes.c_void_p * max(1, len(events)))(*[ev.cuda_event for ev in events])
     check("asap_moe_time_layer", lib().asap_moe_time_layer(len(events), arr))
+    _timing.events = events     # alive until the layer call that records them returns
 
 
 def asap_moe_route_noalloc(h, x, idx, w, counts, offsets, stream=None):
