@@ -478,7 +478,10 @@ int asap_moe_mailbox_served(asap_moe_mailbox_t m, int32_t slot, uint64_t* epoch)
 
 /* Record ev_before / ev_after (cudaEvent_t) on the stream right before the
  * first and right after the last grouped GEMM of the next serve call (for
- * timing the GEMMs of a round).  NULL events clear the request. */
+ * timing the GEMMs of a round).  NULL events clear the request.  The next
+ * asap_moe_mailbox_serve or _serve_many call takes the request whatever its
+ * outcome (a call that fails before its GEMMs records nothing); the events
+ * must stay valid until that call returns. */
 int asap_moe_mailbox_time_gemms(asap_moe_mailbox_t m, void* ev_before, void* ev_after);
 
 /* Synchronise the device; *rounds = service rounds run so far; claimed

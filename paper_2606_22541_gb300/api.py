@@ -303,7 +303,10 @@ def asap_moe_mailbox_post(m, slot, x, out, stream=None, layer_id=None):
 
 
 def asap_moe_mailbox_serve(m, slot, epoch, stream=None):
-    check("asap_moe_mailbox_serve", lib().asap_moe_mailbox_serve(m.ptr, int(slot), int(epoch), _stream(stream)))
+    try:
+        check("asap_moe_mailbox_serve", lib().asap_moe_mailbox_serve(m.ptr, int(slot), int(epoch), _stream(stream)))
+    finally:
+        m._timing = None
 
 
 def asap_moe_mailbox_serve_many(m, slots, epochs, stream=None):
@@ -311,7 +314,10 @@ def asap_moe_mailbox_serve_many(m, slots, epochs, stream=None):
     n = len(slots)
     cs = (ctypes.c_int32 * n)(*[int(v) for v in slots])
     ce = (ctypes.c_uint64 * n)(*[int(v) for v in epochs])
-    check("asap_moe_mailbox_serve_many", lib().asap_moe_mailbox_serve_many(m.ptr, n, cs, ce, _stream(stream)))
+    try:
+        check("asap_moe_mailbox_serve_many", lib().asap_moe_mailbox_serve_many(m.ptr, n, cs, ce, _stream(stream)))
+    finally:
+        m._timing = None
 
 
 def asap_moe_mailbox_wait(m, slot, stream=None):
@@ -333,6 +339,7 @@ def asap_moe_mailbox_time_gemms(m, ev_before, ev_after):
     check("asap_moe_mailbox_time_gemms",
           lib().asap_moe_mailbox_time_gemms(m.ptr, ctypes.c_void_p(ev_before.cuda_event),
                                             ctypes.c_void_p(ev_after.cuda_event)))
+    m._timing = (ev_before, ev_after)   # alive until the serve call that records them returns
 
 
 def asap_moe_mailbox_rounds(m, cap=4096):

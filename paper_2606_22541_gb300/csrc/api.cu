@@ -11,6 +11,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <utility>
 #include <vector>
 
 #define ASAP_API extern "C" __attribute__((visibility("default")))
@@ -1477,7 +1478,8 @@ namespace {
 // (bounded) for the first one's flag and claims every published, unserved
 // post of its layer; each listed slot's served event is recorded after the
 // round.
-int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uint64_t* epochs, cudaStream_t st) {
+int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uint64_t* epochs, cudaStream_t st,
+                cudaEvent_t gemm_ev0, cudaEvent_t gemm_ev1) {
   asap_moe_t h = m->h;
   const asap_moe_config& c = h->cfg;
   const int32_t slot = slots[0];
@@ -1516,7 +1518,7 @@ int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uin
                                           at<float>(ws, L.xs), xq_sh, xs_sh, at<int32_t>(ws, L.perm_src), perm_dst,
                                           h->status, st),
            "dispatch launch");
-    if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
+    if (gemm_ev0) CU_TRY(cudaEventRecord(gemm_ev0, st), "timing event");
     if ((r = run_gate_up_fp8(h, at<void>(ws, L.xq), at<float>(ws, L.xs), offsets, xq_sh, xs_sh, N, at<void>(ws, L.hq),
                              at<float>(ws, L.hs), at<void>(ws, L.hq_sh), at<float>(ws, L.hs_sh), layer, counters,
                              st, n_total)) != ASAP_OK)
@@ -1532,7 +1534,7 @@ int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uin
     CU_TRY(asap::launch_dispatch_mbox(m->round, g, m->rowmap, idx, at<int32_t>(ws, L.chunk_base), offsets, y_perm,
                                       at<int32_t>(ws, L.perm_src), perm_dst, y_sh, h->status, st),
            "dispatch launch");
-    if (m->gemm_ev0) CU_TRY(cudaEventRecord(m->gemm_ev0, st), "timing event");
+    if (gemm_ev0) CU_TRY(cudaEventRecord(gemm_ev0, st), "timing event");
     if ((r = run_gate_up(h, y_perm, offsets, y_sh, N, at<void>(ws, L.h), at<void>(ws, L.h_sh), layer, counters, st,
                          n_total)) != ASAP_OK)
       return r;
@@ -1540,8 +1542,7 @@ int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uin
                       st, n_total)) != ASAP_OK)
       return r;
   }
-  if (m->gemm_ev1) CU_TRY(cudaEventRecord(m->gemm_ev1, st), "timing event");
-  m->gemm_ev0 = m->gemm_ev1 = nullptr;
+  if (gemm_ev1) CU_TRY(cudaEventRecord(gemm_ev1, st), "timing event");
   CU_TRY(asap::launch_combine_mbox(m->round, g, y_perm, y_sh, at<float>(ws, L.w), perm_dst, h->status, st),
          "combine launch");
   CU_TRY(asap::launch_mbox_finish(m->slots, m->round, m->log, m->served_host_dev, st), "finish launch");
@@ -1556,20 +1557,30 @@ int serve_round(asap_moe_mailbox_t m, int count, const int32_t* slots, const uin
 
 }  // namespace
 
+// The mailbox's pending GEMM timing events, taken (the request is cleared)
+// by the serve call that starts now, whatever its outcome.  Mailbox lock held.
+static std::pair<cudaEvent_t, cudaEvent_t> take_gemm_timing(asap_moe_mailbox_t m) {
+  const std::pair<cudaEvent_t, cudaEvent_t> ev{m->gemm_ev0, m->gemm_ev1};
+  m->gemm_ev0 = m->gemm_ev1 = nullptr;
+  return ev;
+}
+
 ASAP_API int asap_moe_mailbox_serve(asap_moe_mailbox_t m, int32_t slot, uint64_t epoch, void* stream) {
   if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  std::lock_guard<std::mutex> lock(m->mu);
+  const auto ev = take_gemm_timing(m);
   if (slot < 0 || slot >= m->g.n_slots) return fail(ASAP_ERR_INVALID, "slot outside [0, n_slots)");
   if (epoch < 1) return fail(ASAP_ERR_INVALID, "epoch must be >= 1 (the value asap_moe_mailbox_post returned)");
-  std::lock_guard<std::mutex> lock(m->mu);
-  return serve_round(m, 1, &slot, &epoch, S(stream));
+  return serve_round(m, 1, &slot, &epoch, S(stream), ev.first, ev.second);
 }
 
 ASAP_API int asap_moe_mailbox_serve_many(asap_moe_mailbox_t m, int32_t count, const int32_t* slots,
                                          const uint64_t* epochs, void* stream) {
   if (!m) return fail(ASAP_ERR_INVALID, "NULL mailbox");
+  std::lock_guard<std::mutex> lock(m->mu);
+  const auto ev = take_gemm_timing(m);
   if (count < 1 || count > m->g.n_slots || !slots || !epochs)
     return fail(ASAP_ERR_INVALID, "count must be in [1, n_slots] with host arrays of count slots and epochs");
-  std::lock_guard<std::mutex> lock(m->mu);
   uint64_t seen = 0;
   for (int i = 0; i < count; ++i) {
     const int32_t s = slots[i];
@@ -1580,7 +1591,7 @@ ASAP_API int asap_moe_mailbox_serve_many(asap_moe_mailbox_t m, int32_t count, co
       return fail(ASAP_ERR_INVALID, "slot " + std::to_string(s) + ": epoch " + std::to_string(epochs[i]) +
                                         " is not a post made to it");
   }
-  return serve_round(m, count, slots, epochs, S(stream));
+  return serve_round(m, count, slots, epochs, S(stream), ev.first, ev.second);
 }
 
 ASAP_API int asap_moe_mailbox_wait(asap_moe_mailbox_t m, int32_t slot, void* stream) {
