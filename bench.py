@@ -55,6 +55,8 @@ def parse_args():
     ap.add_argument("--mailbox-closed-loop", action="store_true",
                     help="steps back to back, each DP-group stream posting its next micro-batch only once its "
                          "previous one has been served (its layer output is back)")
+    ap.add_argument("--fused-combine", action="store_true",
+                    help="asap_moe_layer combines inside the down GEMM (asap_moe_set_combine) instead of a kernel after it")
     ap.add_argument("--mailbox-serve-many", action="store_true",
                     help="one asap_moe_mailbox_serve_many call per step for the step's posts instead of one serve "
                          "call per post")
@@ -287,6 +289,8 @@ def run_ours(args, dist):
     weights = inputs.make_weights(cfg, dev)
     h = api.asap_moe_create(cfg, weights, sum(mbs))   # sum: the batched call serves all at once
     del weights
+    if args.fused_combine and cfg.dtype == "bf16":   # the fused combine is the bf16 down GEMM's
+        api.asap_moe_set_combine(h, api.COMBINE_FUSED)
     torch.cuda.empty_cache()
     xs = inputs.make_microbatches(cfg, dev)
     outs = [torch.empty_like(x) for x in xs]
@@ -330,9 +334,10 @@ def run_ours(args, dist):
     if code != 0:
         raise RuntimeError(f"device status word {word:#x} after the timed region")
     # route (one kernel for E = 256 with grouped sigmoid gating, else router,
-    # gate and scan), dispatch, gate/up GEMM, down GEMM, combine
+    # gate and scan), dispatch, gate/up GEMM, down GEMM, combine (none when
+    # the combine runs inside the down GEMM)
     fused = cfg.n_experts == 256 and cfg.gating == "sigmoid_grouped" and cfg.n_groups in (1, 2, 4, 8)
-    launches_per_mb = (1 if fused else 3) + 4
+    launches_per_mb = (1 if fused else 3) + (3 if args.fused_combine and cfg.dtype == "bf16" else 4)
     result = {
         "metric": METRIC,
         "value": dist.world * tokens_per_step * args.steps / (elapsed_ms / 1e3),
@@ -352,7 +357,8 @@ def run_ours(args, dist):
                                + f", {len(mbs)} micro-batches ({','.join(map(str, mbs))} tokens), one CUDA stream each",
                    "tokens_per_step": tokens_per_step, "microbatches": mbs,
                    "parallelism": f"replicas x{dist.world} (no data-path collective)",
-                   "l2": f"inputs larger than L2: {weight_gb(cfg):.1f} GB of expert weights streamed every step"},
+                   "l2": f"inputs larger than L2: {weight_gb(cfg):.1f} GB of expert weights streamed every step",
+                   **({"combine": "fused into the down GEMM"} if args.fused_combine and cfg.dtype == "bf16" else {})},
         "gpu_launches": launches_per_mb * len(mbs) * args.steps,
         "clocks": clk,
     }

@@ -203,6 +203,25 @@ enum {
 };
 int asap_moe_set_tiling(asap_moe_t h, int32_t mode);
 
+/* Where asap_moe_layer and asap_moe_layer_dyn combine (bf16 layers): in a
+ * separate kernel after the down GEMM (ASAP_COMBINE_SEPARATE, the default), or
+ * inside the down GEMM (ASAP_COMBINE_FUSED, row f4 of the hot path): each
+ * warp that has stored its rows of an output tile counts one arrival per row
+ * for the row's token slice (token, 256 output columns), and the arrival that
+ * completes a slice (the token's k routed rows and its shared-expert row)
+ * sums that slice in slot order with the separate kernel's arithmetic, so
+ * the output bits are the same in both modes.  Measured slower at the
+ * DeepSeek-V3 shape (most slices complete in the launch's last tiles, whose
+ * warps then hold back the tensor core), hence not the default.  The other
+ * calls keep their separate combine.  FP8 handles return ASAP_ERR_UNSUPPORTED
+ * for ASAP_COMBINE_FUSED; another mode returns ASAP_ERR_INVALID.  Host state
+ * only; do not call it while another thread enqueues on the same handle. */
+enum {
+  ASAP_COMBINE_SEPARATE = 0,
+  ASAP_COMBINE_FUSED = 1
+};
+int asap_moe_set_combine(asap_moe_t h, int32_t mode);
+
 /* Free everything create allocated.  Synchronises the device first.  NULL is
  * accepted.  Refused with ASAP_ERR_INVALID (nothing freed) while a mailbox
  * created on h is alive: destroy the mailboxes first. */

@@ -44,6 +44,7 @@ SIGNATURES = {
     "asap_moe_n_layers": [_P, ctypes.POINTER(_I)],
     "asap_moe_destroy": [_P],
     "asap_moe_time_layer": [_I, ctypes.POINTER(_P)],
+    "asap_moe_set_combine": [_P, _I],
     "asap_moe_workspace_size": [ctypes.POINTER(AsapMoeConfig), _I, ctypes.POINTER(_SZ)],
     "asap_moe_check_config": [ctypes.POINTER(AsapMoeConfig)],
     "asap_moe_router_logits": [_P, _P, _I, _P, _P, _SZ, _P],

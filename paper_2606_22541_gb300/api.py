@@ -350,6 +350,16 @@ def asap_moe_mailbox_rounds(m, cap=4096):
     return n.value, list(buf[:min(cap, n.value)])
 
 
+COMBINE_SEPARATE, COMBINE_FUSED = 0, 1
+
+
+def asap_moe_set_combine(h, mode):
+    """Where asap_moe_layer combines on a bf16 handle: COMBINE_SEPARATE (a
+    kernel after the down GEMM, the default) or COMBINE_FUSED (inside the down
+    GEMM); bit-identical outputs."""
+    check("asap_moe_set_combine", lib().asap_moe_set_combine(h.ptr, int(mode)))
+
+
 TILING_AUTO, TILING_SINGLE, TILING_PAIRED = 0, 1, 2
 
 

@@ -42,6 +42,7 @@ struct asap_moe_s {
   bool tc_router = false;             // router GEMM on the tensor core (E == 256)
   bool fp8 = false;                   // e4m3 experts with fp32 128 x 128 block scales
   int tiling = ASAP_TILING_AUTO;       // BF16 grouped GEMM tile shape (asap_moe_set_tiling)
+  int combine = ASAP_COMBINE_SEPARATE;  // where asap_moe_layer combines (asap_moe_set_combine)
   std::atomic<int> mailboxes{0};      // live mailboxes created on this handle
 };
 
@@ -74,7 +75,7 @@ constexpr int kHintF8A = ASAP_HINT_FP8_A, kHintF8B = ASAP_HINT_FP8_B;
 struct Layout {
   size_t logits, idx, w, hist, chunk_base, counts, offsets, perm_src, perm_dst, tile_counters, ticket;
   // bf16: x_perm (also y_perm in asap_moe_layer), h, h_sh, y_sh
-  size_t x_perm, h, h_sh, y_sh;
+  size_t x_perm, h, h_sh, y_sh, comb_cnt;
   // fp8: quantised rows and their per-128-channel scales, bf16 expert outputs
   size_t xq, xs, xq_sh, xs_sh, hq, hs, hq_sh, hs_sh, y_perm;
   size_t total;
@@ -120,6 +121,7 @@ Layout layout(const asap_moe_config& c, long long n) {
     L.h = take(nk * I * 2);
     L.h_sh = take(N * Is * 2);
     L.y_sh = take(N * H * 2 * (Is ? 1 : 0));
+    L.comb_cnt = take(N * (H / asap::kGemmBN) * 4);  // slice arrivals of the fused combine
   }
   L.total = off;
   return L;
@@ -407,8 +409,20 @@ int run_gate_up(asap_moe_t h, const void* x_perm, const int32_t* offsets, const 
 }
 
 // GEMM2: y = h Wd^T on the routed segments, plus the shared expert.
+// The combine fused into the down GEMM (see combine_slices): slice arrival
+// counters (zeroed before the launch), the permutation and the routing
+// weights of the call, and its output.
+struct CombineFuse {
+  int* cnt = nullptr;
+  const int32_t* src = nullptr;
+  const int32_t* dst = nullptr;
+  const float* w = nullptr;
+  void* out = nullptr;
+};
+
 int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void* hsh, int n, void* y_perm,
-             void* y_sh, const int32_t* layer, int32_t* counter, cudaStream_t st, const int32_t* m1_dev = nullptr) {
+             void* y_sh, const int32_t* layer, int32_t* counter, cudaStream_t st, const int32_t* m1_dev = nullptr,
+             const CombineFuse& cf = CombineFuse()) {
   const asap_moe_config& c = h->cfg;
   const long long nk = static_cast<long long>(n) * c.top_k;
   const bool sh = c.n_shared != 0;
@@ -453,6 +467,13 @@ int run_down(asap_moe_t h, const void* hbuf, const int32_t* offsets, const void*
   a.k_splits = 1;
   a.tile_counter = counter;
   a.b_tiled = 1;  // weights in tile-contiguous order (pack_layer)
+  a.comb_cnt = cf.cnt;
+  a.comb_src = cf.src;
+  a.comb_dst = cf.dst;
+  a.comb_w = cf.w;
+  a.comb_out = cf.out;
+  a.comb_n = n;
+  a.comb_k = c.top_k;
   const long long tiles = static_cast<long long>(ub_mtiles(c, nk, bm)) * a.n_tiles0 +
                           (sh ? static_cast<long long>(asap::ceil_div(n, bm)) * a.n_tiles1 : 0);
   CU_TRY(asap::gemm_launch(asap::EPI_BF16, pair, maps, a, static_cast<int>(std::min<long long>(tiles, h->num_sms)), st),
@@ -1074,6 +1095,21 @@ int run_layer(asap_moe_t h, const void* x, int32_t n, void* out, void* ws, size_
   void* hsh = at<void>(ws, L.h_sh);
   if ((r = run_gate_up(h, x_perm, offsets, x, n, hbuf, hsh, layer, counters, st)) != ASAP_OK) return r;
   CU_TRY(tev.mark(3, st), "timing event");
+  if (h->combine == ASAP_COMBINE_FUSED) {
+    CombineFuse cf;
+    cf.cnt = at<int>(ws, L.comb_cnt);
+    cf.src = perm_src;
+    cf.dst = perm_dst;
+    cf.w = w;
+    cf.out = out;
+    CU_TRY(cudaMemsetAsync(cf.cnt, 0, sizeof(int) * static_cast<size_t>(n) * (c.hidden / asap::kGemmBN), st),
+           "slice counters");
+    if ((r = run_down(h, hbuf, offsets, hsh, n, x_perm, y_sh, layer, counters + 1, st, nullptr, cf)) != ASAP_OK)
+      return r;
+    CU_TRY(tev.mark(4, st), "timing event");
+    CU_TRY(tev.mark(5, st), "timing event");  // the combine ran inside the down GEMM
+    return ASAP_OK;
+  }
   if ((r = run_down(h, hbuf, offsets, hsh, n, x_perm, y_sh, layer, counters + 1, st)) != ASAP_OK) return r;
   CU_TRY(tev.mark(4, st), "timing event");
   CU_TRY(asap::launch_combine(x_perm, y_sh, w, perm_dst, n, c.hidden, c.top_k, out, h->status, st),
@@ -1266,6 +1302,16 @@ ASAP_API int asap_moe_set_tiling(asap_moe_t h, int32_t mode) {
   if (mode != ASAP_TILING_AUTO && mode != ASAP_TILING_SINGLE && mode != ASAP_TILING_PAIRED)
     return fail(ASAP_ERR_INVALID, "tiling mode must be ASAP_TILING_AUTO, _SINGLE or _PAIRED");
   h->tiling = mode;
+  return ASAP_OK;
+}
+
+ASAP_API int asap_moe_set_combine(asap_moe_t h, int32_t mode) {
+  if (!h) return fail(ASAP_ERR_INVALID, "NULL handle");
+  if (mode != ASAP_COMBINE_SEPARATE && mode != ASAP_COMBINE_FUSED)
+    return fail(ASAP_ERR_INVALID, "combine mode must be ASAP_COMBINE_SEPARATE or ASAP_COMBINE_FUSED");
+  if (mode == ASAP_COMBINE_FUSED && h->fp8)
+    return fail(ASAP_ERR_UNSUPPORTED, "the combine is fused into the bf16 down GEMM only");
+  h->combine = mode;
   return ASAP_OK;
 }
 

@@ -115,7 +115,7 @@ __device__ __forceinline__ void store_round(const uint32_t* pk, uint4* stage, in
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     stage[lane * 8 + (j ^ (lane & 7))] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
-  if (valid_rows == 32) {
+  if (valid_rows == 32 && tm) {
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
@@ -166,6 +166,95 @@ __device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t
   }
 }
 
+// Combine fused into the down GEMM: after a warp has stored its rows of a
+// tile (plain stores, so that a fence orders them before the arrivals), each
+// stored row adds one arrival to its token slice (token t, 256-column
+// n-tile); the arrival that completes a slice (its k routed rows and the
+// shared row) has the warp sum it, out[t, slice] = sum_j w[t,j]
+// y_perm[perm_dst[t,j], slice] in slot order, then + y_sh[t, slice], rounded
+// to bf16: the combine kernel's arithmetic, so the output bits are the
+// same.  No wait: the last arrival does the work.
+__device__ __forceinline__ void combine_slices(const Tile& T, const GemmArgs& a, long long r0, int lane,
+                                               int valid_rows) {
+  const int V = static_cast<int>(a.ldo0 / 8);  // 16-byte vectors per row
+  const int NT = V / 32;                        // 256-column slices per row
+  const int need = a.comb_k + (a.m1 > 0 ? 1 : 0);
+  int t = -1;
+  if (lane < valid_rows) {
+    const long long r = r0 + lane;
+    t = T.p1 ? static_cast<int>(r) : __ldg(a.comb_src + r);
+    if (t < 0 || t >= a.comb_n) {
+      record_status(a.status, ST_BAD_POSITION);
+      t = -1;
+    }
+  }
+  __threadfence();  // the warp's row stores (after its last __syncwarp) before the arrivals
+  bool last = false;
+  if (t >= 0) last = atomicAdd(a.comb_cnt + static_cast<long long>(t) * NT + T.n_tile, 1) == need - 1;
+  unsigned m = __ballot_sync(0xffffffffu, last);
+  if (!m) return;
+  __threadfence();  // the other rows of the completed slices, stored by other CTAs
+  const uint4* y = static_cast<const uint4*>(a.out0);
+  const uint4* ysh = static_cast<const uint4*>(a.out1);
+  uint4* out = static_cast<uint4*>(a.comb_out);
+  const int v = T.n_tile * 32 + lane;
+  while (m) {
+    const int src = __ffs(m) - 1;
+    m &= m - 1;
+    const int tt = __shfl_sync(0xffffffffu, t, src);
+    const long long tk = static_cast<long long>(tt) * a.comb_k;
+    int p[kMaxTopK];
+    float wj[kMaxTopK];
+    uint4 yv[kMaxTopK];
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j) {
+      p[j] = -1;
+      wj[j] = 0.f;
+      if (j < a.comb_k) {
+        p[j] = __ldcg(a.comb_dst + tk + j);
+        wj[j] = __ldg(a.comb_w + tk + j);
+        if (p[j] < 0 || p[j] >= a.m0) {
+          if (lane == 0) record_status(a.status, ST_BAD_POSITION);
+          p[j] = -1;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j)
+      if (p[j] >= 0) yv[j] = __ldcg(y + static_cast<long long>(p[j]) * V + v);
+    float acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j) {
+      if (p[j] >= 0) {
+        const float w = wj[j];
+        acc[0] = fmaf(w, bf16_lo(yv[j].x), acc[0]);
+        acc[1] = fmaf(w, bf16_hi(yv[j].x), acc[1]);
+        acc[2] = fmaf(w, bf16_lo(yv[j].y), acc[2]);
+        acc[3] = fmaf(w, bf16_hi(yv[j].y), acc[3]);
+        acc[4] = fmaf(w, bf16_lo(yv[j].z), acc[4]);
+        acc[5] = fmaf(w, bf16_hi(yv[j].z), acc[5]);
+        acc[6] = fmaf(w, bf16_lo(yv[j].w), acc[6]);
+        acc[7] = fmaf(w, bf16_hi(yv[j].w), acc[7]);
+      }
+    }
+    if (a.m1 > 0) {
+      const uint4 sv = __ldcg(ysh + static_cast<long long>(tt) * V + v);
+      acc[0] += bf16_lo(sv.x);
+      acc[1] += bf16_hi(sv.x);
+      acc[2] += bf16_lo(sv.y);
+      acc[3] += bf16_hi(sv.y);
+      acc[4] += bf16_lo(sv.z);
+      acc[5] += bf16_hi(sv.z);
+      acc[6] += bf16_lo(sv.w);
+      acc[7] += bf16_hi(sv.w);
+    }
+    out[static_cast<long long>(tt) * V + v] = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
+                                                         pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
+  }
+}
+
 // Epilogue of one tile for the thread owning TMEM lane ``row`` (taddr: that
 // lane, the accumulator's first column); it arrives on ``tempty`` once the
 // accumulator has been read.  lanes: the warp's lanes that hold rows (16 for
@@ -177,8 +266,10 @@ __device__ __forceinline__ void tmem_to_bf16_64(uint32_t taddr, int c0, uint32_t
 // (measured 1-2 % faster; for the gate/up GEMM it measured no faster and
 // spilled).  Otherwise rows are read and stored round by round (single
 // m-tiles' two accumulators already overlap the epilogue with the next main
-// loop).  The fp32 epilogue (router logits) stores as it reads.
-template <int EPI, bool EARLY>
+// loop).  The fp32 epilogue (router logits) stores as it reads.  COMB: the
+// combine is fused (combine_slices after the tile's stores, which are plain
+// stores: tm is nullptr).
+template <int EPI, bool EARLY, bool COMB>
 __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, uint32_t taddr, int row,
                                               uint32_t tempty, uint4* stage, int lane, int lanes,
                                               const CUtensorMap* tm) {
@@ -221,6 +312,7 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
 #pragma unroll
       for (int rd = 0; rd < kRounds; ++rd)
         store_round(pk + 32 * rd, stage, lane, out_w + 64 * rd, ldo, valid_rows, tm, bx + 64 * rd, by);
+      if constexpr (COMB) combine_slices(T, a, orow_t + wrow0, lane, valid_rows);
     } else {
 #pragma unroll 1
       for (int rd = 0; rd < kRounds; ++rd) {
@@ -230,11 +322,12 @@ __device__ __forceinline__ void epilogue_tile(const Tile& T, const GemmArgs& a, 
       }
       tc_fence_before();
       mbar_arrive(tempty);
+      if constexpr (COMB) combine_slices(T, a, orow_t + wrow0, lane, valid_rows);
     }
   }
 }
 
-template <int EPI, bool PAIR>
+template <int EPI, bool PAIR, bool COMB>
 __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                         const __grid_constant__ CUtensorMap tmO0, const __grid_constant__ CUtensorMap tmO1,
@@ -505,9 +598,9 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
         const bool m64 = EPI != EPI_F32 && half_rows <= kTailRows;
         const int erow = m64 ? half * kGemmBM + q * 16 + lane : row;
         // arrives on tempty itself
-        epilogue_tile<EPI, PAIR && EPI == EPI_BF16>(T, args, taddr, erow, tempty_bar(acc),
-                                                    stage_all + (warp - 2) * (kStageWarpBytes / 16), lane,
-                                                    m64 ? 16 : 32, T.p1 ? &tmO1 : &tmO0);
+        epilogue_tile<EPI, PAIR && EPI == EPI_BF16, COMB>(T, args, taddr, erow, tempty_bar(acc),
+                                                          stage_all + (warp - 2) * (kStageWarpBytes / 16), lane,
+                                                          m64 ? 16 : 32, COMB ? nullptr : (T.p1 ? &tmO1 : &tmO0));
       } else {
         tc_fence_before();
         mbar_arrive(tempty_bar(acc));
@@ -526,16 +619,17 @@ __global__ void __launch_bounds__(Gemm<EPI, PAIR>::kThreads, 1)
   }
 }
 
-template <int EPI, bool PAIR>
+template <int EPI, bool PAIR, bool COMB = false>
 cudaError_t set_attr() {
-  return cudaFuncSetAttribute(grouped_gemm_kernel<EPI, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(grouped_gemm_kernel<EPI, PAIR, COMB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(smem_bytes<EPI, PAIR>()));
 }
 
-template <int EPI, bool PAIR>
+template <int EPI, bool PAIR, bool COMB = false>
 void launch(const CUtensorMap* maps, const GemmArgs& args, int grid, cudaStream_t stream) {
-  grouped_gemm_kernel<EPI, PAIR><<<dim3(grid), dim3(Gemm<EPI, PAIR>::kThreads), smem_bytes<EPI, PAIR>(), stream>>>(
-      maps[0], maps[1], maps[2], maps[3], args);
+  grouped_gemm_kernel<EPI, PAIR, COMB>
+      <<<dim3(grid), dim3(Gemm<EPI, PAIR>::kThreads), smem_bytes<EPI, PAIR>(), stream>>>(maps[0], maps[1], maps[2],
+                                                                                        maps[3], args);
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -566,6 +660,8 @@ cudaError_t gemm_set_attributes() {
   if (e == cudaSuccess) e = set_attr<EPI_SWIGLU, true>();
   if (e == cudaSuccess) e = set_attr<EPI_BF16, false>();
   if (e == cudaSuccess) e = set_attr<EPI_BF16, true>();
+  if (e == cudaSuccess) e = set_attr<EPI_BF16, false, true>();
+  if (e == cudaSuccess) e = set_attr<EPI_BF16, true, true>();
   if (e == cudaSuccess) e = set_attr<EPI_F32, false>();
   return e;
 }
@@ -577,8 +673,14 @@ cudaError_t gemm_launch(int epi, bool pair, const CUtensorMap* maps, const GemmA
     if (pair) launch<EPI_SWIGLU, true>(maps, args, grid, stream);
     else launch<EPI_SWIGLU, false>(maps, args, grid, stream);
   } else if (epi == EPI_BF16) {
-    if (pair) launch<EPI_BF16, true>(maps, args, grid, stream);
-    else launch<EPI_BF16, false>(maps, args, grid, stream);
+    if (args.comb_cnt) {
+      if (pair) launch<EPI_BF16, true, true>(maps, args, grid, stream);
+      else launch<EPI_BF16, false, true>(maps, args, grid, stream);
+    } else if (pair) {
+      launch<EPI_BF16, true>(maps, args, grid, stream);
+    } else {
+      launch<EPI_BF16, false>(maps, args, grid, stream);
+    }
   } else {
     if (pair) return cudaErrorInvalidValue;
     launch<EPI_F32, false>(maps, args, grid, stream);

@@ -65,6 +65,13 @@ struct GemmArgs {
   int bmap0, bmap1;
   int* tile_counter;       // zero at launch: tiles are claimed dynamically; nullptr: static order
   int b_tiled;             // B in tile-contiguous order (launch_retile): box row ((b_row/256) k_iters + kb) 256
+  // combine fused into the down GEMM (EPI_BF16 only; comb_cnt == nullptr: off)
+  int* comb_cnt;             // [comb_n, n_tiles0] arrivals per token slice, zero at launch
+  const int32_t* comb_src;   // [m0] token of each routed row (perm_src)
+  const int32_t* comb_dst;   // [comb_n, comb_k] routed row of each token slot (perm_dst)
+  const float* comb_w;       // [comb_n, comb_k] routing weights
+  void* comb_out;            // [comb_n, ldo0] bf16 layer output
+  int comb_n, comb_k;        // tokens (problem 1's rows when it exists) and slots per token
 };
 
 constexpr int kTileCounters = 2;  // per call: gate/up GEMM, down GEMM

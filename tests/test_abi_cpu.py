@@ -122,3 +122,10 @@ def test_time_layer_validates_its_request(L):
     # failing layer call takes the request and records nothing
     assert L.asap_moe_time_layer(6, arr) == _native.ASAP_OK
     assert L.asap_moe_layer(None, None, 1, None, None, 0, None) == _native.ASAP_ERR_INVALID
+
+
+def test_combine_modes_match_the_header(L):
+    text = open(HEADER).read()
+    vals = {m: int(v) for m, v in re.findall(r"ASAP_COMBINE_(\w+)\s*=\s*(\d+)", text)}
+    assert vals == {"SEPARATE": api.COMBINE_SEPARATE, "FUSED": api.COMBINE_FUSED}
+    assert L.asap_moe_set_combine(None, api.COMBINE_FUSED) == _native.ASAP_ERR_INVALID

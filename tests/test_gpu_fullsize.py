@@ -120,3 +120,25 @@ def test_full_size_streams_against_oracle(cfg):
     code, word = api.asap_moe_status(h)
     assert code == 0 and word == 0, f"status {word:#x}"
     h.close()
+
+
+@pytest.mark.parametrize("cfg,n", [(DSV3, 4096), (MIXTRAL, 3584)], ids=["dsv3_4096", "mixtral_3584"])
+def test_fused_combine_full_size_bit_identical(cfg, n):
+    """The combine fused into the down GEMM at a full-size micro-batch (every
+    256-column slice of every token completed by its last arrival) gives the
+    separate combine's bits."""
+    w = inputs.make_weights(cfg, DEV)
+    h = api.asap_moe_create(cfg, w, n)
+    del w
+    x = inputs.make_tokens(cfg, n, 0, DEV)
+    ws = api.workspace(h, n)
+    ref = torch.empty_like(x)
+    api.asap_moe_layer(h, x, ref, ws)
+    api.asap_moe_set_combine(h, api.COMBINE_FUSED)
+    out = torch.full_like(x, 3.0)
+    api.asap_moe_layer(h, x, out, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(ref.view(torch.int16), out.view(torch.int16))
+    code, word = api.asap_moe_status(h)
+    assert code == 0 and word == 0, f"status {word:#x}"
+    h.close()

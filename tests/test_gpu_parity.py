@@ -499,6 +499,30 @@ def test_layer_timing_events_mark_its_steps_and_change_no_bit(cfg):
     h.close()
 
 
+@pytest.mark.parametrize("cfg", SMALL + ODD, ids=lambda c: c.name)
+def test_fused_combine_is_bit_identical(cfg):
+    """ASAP_COMBINE_FUSED (the combine inside the down GEMM's epilogue, the
+    last arrival of each token slice summing it) against the separate combine
+    kernel: every micro-batch of the configuration, the same bits; tiny
+    micro-batches too (1 and 2 tokens, single tiles with M = 64 tails)."""
+    c = Case.get(cfg)
+    H = cfg.hidden
+    for n in list(cfg.microbatches) + [1, 2]:
+        x = c.tokens(0, n)
+        ws = c.ws(n)
+        ref = torch.empty((n, H), dtype=torch.bfloat16, device=DEV)
+        api.asap_moe_layer(c.h, x, ref, ws)
+        api.asap_moe_set_combine(c.h, api.COMBINE_FUSED)
+        try:
+            out = torch.full_like(ref, 5.0)
+            api.asap_moe_layer(c.h, x, out, ws)
+            torch.cuda.synchronize()
+        finally:
+            api.asap_moe_set_combine(c.h, api.COMBINE_SEPARATE)
+        assert torch.equal(ref.view(torch.int16), out.view(torch.int16)), (cfg.name, n)
+    assert_clean(c)
+
+
 @pytest.mark.parametrize("cfg", [DS_SMALL, ST_SMALL], ids=lambda c: c.name)
 def test_streams_concurrent_equals_serial_and_token_independent(cfg):
     """Micro-batches submitted on their own streams with no host barrier give
