@@ -205,7 +205,7 @@ int asap_moe_set_tiling(asap_moe_t h, int32_t mode);
 
 /* Where asap_moe_layer and asap_moe_layer_dyn combine (bf16 layers): in a
  * separate kernel after the down GEMM (ASAP_COMBINE_SEPARATE, the default), or
- * inside the down GEMM (ASAP_COMBINE_FUSED, row f4 of the hot path): each
+ * inside the down GEMM's epilogue (ASAP_COMBINE_FUSED): each
  * warp that has stored its rows of an output tile counts one arrival per row
  * for the row's token slice (token, 256 output columns), and the arrival that
  * completes a slice (the token's k routed rows and its shared-expert row)
